@@ -1,0 +1,131 @@
+/*
+ * ecmoe.h -- C ABI of the GB300 expert-choice (EC) MoE layer, forward and backward.
+ *
+ * The layer (arXiv 2604.01622, Sec. 2.2 "Mixture-of-Experts Routing"):
+ *   S = softmax_e(X Wr + br)                              router scores, S in R^{N x E}
+ *   T_{e,g} = top-k_g tokens t of group g by S[t,e]        expert choice (Sec. 2.2), one group
+ *                                                          per sequence (Sec. 5.2), per-sequence
+ *                                                          capacity k_g (Sec. 4.2)
+ *   Y_t = sum_{e: t in T_e} S[t,e] * FFN_e(x_t)            gated combine (Sec. 2.2); tokens no
+ *                                                          expert picks get exactly 0
+ *   FFN_e(x) = (silu(x Wg_e) * (x Wu_e)) Wd_e               SwiGLU experts (appendix
+ *                                                          "Experimental Setup")
+ * Ties in the top-k go to the lower token index; the tokens of one (expert, group)
+ * are listed in ascending index. The backward pass treats the selection as fixed.
+ *
+ * Conventions shared by every call:
+ *   - All arrays are row-major and contiguous. Device pointers unless stated.
+ *   - dtype EC_F32: X, Y, dY, dX, Wr, Wg, Wu, Wd are float32.
+ *     dtype EC_BF16: the same arrays are bf16 (raw 16-bit), accumulation is fp32.
+ *     S, gates, br and every weight gradient are float32 in both modes.
+ *   - Shapes: X, Y, dY, dX [N][d]; Wr [d][E]; br [E]; Wg, Wu [E][d][d_ff];
+ *     Wd [E][d_ff][d]; S [E][N] (expert-major); idx, gate [E][M] with
+ *     M = sum_g k_g: row e holds expert e's tokens, group g at offsets
+ *     k_off[g] .. k_off[g+1]-1 where k_off is the prefix sum of k_g.
+ *   - Device pointers must be 16-byte aligned. On the bf16 path d and d_ff must be
+ *     multiples of 64.
+ *   - Every compute call is asynchronous on `stream` (a cudaStream_t, NULL for the
+ *     legacy default stream) and does no host synchronisation. Argument errors are
+ *     returned before anything is launched. A kernel that gives up on a bounded
+ *     wait records EC_ERR_TIMEOUT in a device status word; ec_check_device reads it.
+ *   - The library never allocates device memory: the caller provides one workspace
+ *     (ec_workspace_bytes) that holds the activations saved for the backward pass.
+ *     The library never frees caller memory.
+ *   - A context is not thread-safe; calls on one context must be ordered.
+ */
+#ifndef ECMOE_H
+#define ECMOE_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  EC_OK = 0,
+  EC_ERR_INVALID_ARG = 1, /* null pointer, misaligned pointer, bad enum */
+  EC_ERR_SHAPE = 2,       /* inconsistent sizes, k_g outside [0, L_g], bad group offsets */
+  EC_ERR_UNSUPPORTED = 3, /* valid but not implemented (e.g. bf16 with d % 64 != 0) */
+  EC_ERR_CUDA = 4,        /* a CUDA runtime error; message in ec_last_error */
+  EC_ERR_TIMEOUT = 5,     /* a device-side bounded wait expired (kernel returned early) */
+  EC_ERR_WORKSPACE = 6,   /* workspace missing, too small or misaligned */
+  EC_ERR_STATE = 7        /* call order violated (backward before forward, ...) */
+} ec_status;
+
+typedef enum { EC_F32 = 0, EC_BF16 = 1 } ec_dtype;
+
+typedef struct ec_ctx ec_ctx;
+
+/* Create a context for one layer shape.
+ *   N tokens in G groups: group g holds tokens group_off[g] .. group_off[g+1]-1
+ *   (host array of G+1 int32, group_off[0] = 0, non-decreasing, group_off[G] = N).
+ *   k_g: host array of G int32 capacities, 0 <= k_g[g] <= group size (Sec. 4.2: the
+ *   capacity may differ per sequence). M = sum k_g is the number of rows every expert
+ *   processes (Sec. 2.2: each expert takes exactly its capacity).
+ *   dtype: EC_F32 or EC_BF16.
+ * Host arrays are copied; the caller keeps ownership. Returns EC_ERR_SHAPE on bad sizes. */
+ec_status ec_ctx_create(ec_ctx** out, int32_t N, int32_t d, int32_t E, int32_t d_ff, int32_t G,
+                        const int32_t* group_off, const int32_t* k_g, int32_t dtype);
+
+/* Destroy a context (host memory only; the workspace stays the caller's). NULL is ignored. */
+void ec_ctx_destroy(ec_ctx* ctx);
+
+/* Replace the per-group capacities (Sec. 4.2: a new k_g per denoising step).
+ * sum(k_g) must not exceed the M the context was created with (the workspace is sized
+ * for it). Copies k_g to the device with a synchronous copy; call outside stream capture.
+ * Invalidates saved forward state. */
+ec_status ec_ctx_set_capacity(ec_ctx* ctx, const int32_t* k_g);
+
+/* Current rows per expert M = sum k_g. */
+int64_t ec_rows_per_expert(const ec_ctx* ctx);
+
+/* Bytes of device workspace the context needs (saved activations, scores, selection,
+ * backward scratch). Depends only on the creation-time sizes. */
+size_t ec_workspace_bytes(const ec_ctx* ctx);
+
+/* Attach a caller-owned device workspace of at least ec_workspace_bytes bytes, 256-byte
+ * aligned. Uploads the group table with a synchronous copy; call outside stream capture.
+ * The workspace must stay allocated while the context is used. */
+ec_status ec_ctx_set_workspace(ec_ctx* ctx, void* workspace, size_t bytes);
+
+/* Router and expert-choice selection only (Sec. 2.2).
+ *   X [N][d], Wr [d][E] (dtype of the context), br [E] float or NULL.
+ *   S_in: NULL to compute S from X and Wr; otherwise a float [E][N] score matrix to select
+ *   from (X, Wr, br are then ignored and may be NULL).
+ *   S_out: NULL or float [E][N], receives the scores used.
+ *   idx [E][M] int32 and gate [E][M] float receive the selection (gate = S[idx, e]). */
+ec_status ec_route(ec_ctx* ctx, const void* X, const void* Wr, const float* br,
+                   const float* S_in, float* S_out, int32_t* idx, float* gate, void* stream);
+
+/* Whole-layer forward (Sec. 2.2): Y [N][d] in the context's dtype. idx, gate, S_out as in
+ * ec_route (each may be NULL). Saves what ec_moe_backward needs in the workspace, and
+ * remembers the weight pointers, which must stay valid and unchanged until the backward
+ * call. Wg, Wu [E][d][d_ff]; Wd [E][d_ff][d]. */
+ec_status ec_moe_forward(ec_ctx* ctx, const void* X, const void* Wr, const float* br,
+                         const void* Wg, const void* Wu, const void* Wd, void* Y,
+                         int32_t* idx, float* gate, float* S_out, void* stream);
+
+/* Backward of the last ec_moe_forward on this context: gradients of <dY, Y>.
+ *   dY, dX [N][d] in the context's dtype (dX is overwritten).
+ *   dWr [d][E], dbr [E] (NULL allowed), dWg, dWu [E][d][d_ff], dWd [E][d_ff][d]: float32,
+ *   overwritten (not accumulated). The selection is held fixed; the gate gradient flows
+ *   through the softmax Jacobian into dX and dWr. */
+ec_status ec_moe_backward(ec_ctx* ctx, const void* dY, void* dX, float* dWr, float* dbr,
+                          float* dWg, float* dWu, float* dWd, void* stream);
+
+/* Synchronise `stream`, read and clear the device status word. Returns EC_ERR_TIMEOUT if a
+ * kernel gave up on a bounded wait since the last check, EC_ERR_CUDA on a CUDA error. */
+ec_status ec_check_device(ec_ctx* ctx, void* stream);
+
+/* Message of the last failed call on this context ("" if none). Owned by the context. */
+const char* ec_last_error(const ec_ctx* ctx);
+
+/* Static name of a status code. */
+const char* ec_status_string(ec_status s);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* ECMOE_H */

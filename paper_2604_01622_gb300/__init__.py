@@ -1,1 +1,136 @@
-"""GB300-native expert-choice MoE layer (placeholder; binding added with the library)."""
+"""GB300-native expert-choice (EC) MoE layer, forward and backward (arXiv 2604.01622).
+
+Thin ctypes binding of the C ABI in include/ecmoe.h: every function here has the name of
+the C entry point it calls and only marshals arguments (device pointers as Python ints,
+a CUDA stream handle, host int32 arrays). All compute runs in libecmoe.so's CUDA kernels;
+there is no fallback. `ECMoELayer` (layer.py) wraps a context with torch-allocated
+buffers for convenience.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import numpy as np
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "libecmoe.so")
+
+EC_OK, EC_ERR_INVALID_ARG, EC_ERR_SHAPE, EC_ERR_UNSUPPORTED = 0, 1, 2, 3
+EC_ERR_CUDA, EC_ERR_TIMEOUT, EC_ERR_WORKSPACE, EC_ERR_STATE = 4, 5, 6, 7
+EC_F32, EC_BF16 = 0, 1
+
+# C entry points declared in include/ecmoe.h
+EXPORTS = (
+    "ec_ctx_create", "ec_ctx_destroy", "ec_ctx_set_capacity", "ec_rows_per_expert",
+    "ec_workspace_bytes", "ec_ctx_set_workspace", "ec_route", "ec_moe_forward",
+    "ec_moe_backward", "ec_check_device", "ec_last_error", "ec_status_string",
+)
+
+_lib = None
+
+
+class ECError(RuntimeError):
+    def __init__(self, status: int, msg: str):
+        super().__init__(f"{status_string(status)}: {msg}")
+        self.status = status
+
+
+def load():
+    """Load libecmoe.so (built by build.py). Raises if it is missing: there is no fallback."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(LIB_PATH):
+        raise RuntimeError(f"{LIB_PATH} is missing: run paper_2604_01622_gb300.build.build() "
+                           "(the EC-MoE layer has no non-CUDA implementation)")
+    lib = ctypes.CDLL(LIB_PATH)
+    vp, i32, i64, sz = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_size_t
+    P32 = ctypes.POINTER(ctypes.c_int32)
+    sig = {
+        "ec_ctx_create": (i32, [ctypes.POINTER(vp), i32, i32, i32, i32, i32, P32, P32, i32]),
+        "ec_ctx_destroy": (None, [vp]),
+        "ec_ctx_set_capacity": (i32, [vp, P32]),
+        "ec_rows_per_expert": (i64, [vp]),
+        "ec_workspace_bytes": (sz, [vp]),
+        "ec_ctx_set_workspace": (i32, [vp, vp, sz]),
+        "ec_route": (i32, [vp, vp, vp, vp, vp, vp, vp, vp, vp]),
+        "ec_moe_forward": (i32, [vp] * 12),
+        "ec_moe_backward": (i32, [vp] * 9),
+        "ec_check_device": (i32, [vp, vp]),
+        "ec_last_error": (ctypes.c_char_p, [vp]),
+        "ec_status_string": (ctypes.c_char_p, [i32]),
+    }
+    for name, (res, args) in sig.items():
+        fn = getattr(lib, name)
+        fn.restype = res
+        fn.argtypes = args
+    _lib = lib
+    return lib
+
+
+def status_string(status: int) -> str:
+    return load().ec_status_string(int(status)).decode()
+
+
+def _check(ctx, status: int):
+    if status != EC_OK:
+        msg = load().ec_last_error(ctx).decode() if ctx else ""
+        raise ECError(status, msg)
+
+
+def _i32(a):
+    arr = np.ascontiguousarray(np.asarray(a, dtype=np.int32))
+    return arr, arr.ctypes.data_as(ctypes.POINTER(ctypes.c_int32))
+
+
+def ec_ctx_create(N, d, E, d_ff, G, group_off, k_g, dtype):
+    lib = load()
+    ctx = ctypes.c_void_p()
+    g_arr, g_ptr = _i32(group_off)
+    k_arr, k_ptr = _i32(k_g)
+    st = lib.ec_ctx_create(ctypes.byref(ctx), N, d, E, d_ff, G, g_ptr, k_ptr, dtype)
+    if st != EC_OK:
+        raise ECError(st, "ec_ctx_create rejected the sizes")
+    return ctx
+
+
+def ec_ctx_destroy(ctx):
+    load().ec_ctx_destroy(ctx)
+
+
+def ec_ctx_set_capacity(ctx, k_g):
+    k_arr, k_ptr = _i32(k_g)
+    _check(ctx, load().ec_ctx_set_capacity(ctx, k_ptr))
+
+
+def ec_rows_per_expert(ctx) -> int:
+    return int(load().ec_rows_per_expert(ctx))
+
+
+def ec_workspace_bytes(ctx) -> int:
+    return int(load().ec_workspace_bytes(ctx))
+
+
+def ec_ctx_set_workspace(ctx, ptr: int, nbytes: int):
+    _check(ctx, load().ec_ctx_set_workspace(ctx, ptr, nbytes))
+
+
+def ec_route(ctx, X, Wr, br, S_in, S_out, idx, gate, stream):
+    _check(ctx, load().ec_route(ctx, X, Wr, br, S_in, S_out, idx, gate, stream))
+
+
+def ec_moe_forward(ctx, X, Wr, br, Wg, Wu, Wd, Y, idx, gate, S_out, stream):
+    _check(ctx, load().ec_moe_forward(ctx, X, Wr, br, Wg, Wu, Wd, Y, idx, gate, S_out, stream))
+
+
+def ec_moe_backward(ctx, dY, dX, dWr, dbr, dWg, dWu, dWd, stream):
+    _check(ctx, load().ec_moe_backward(ctx, dY, dX, dWr, dbr, dWg, dWu, dWd, stream))
+
+
+def ec_check_device(ctx, stream):
+    _check(ctx, load().ec_check_device(ctx, stream))
+
+
+def ec_last_error(ctx) -> str:
+    return load().ec_last_error(ctx).decode()

@@ -1,0 +1,461 @@
+// C ABI of the EC-MoE layer: argument checks, workspace layout and the launch sequence of
+// the forward and backward passes (arXiv 2604.01622, Sec. 2.2; per-sequence capacity,
+// Sec. 4.2; one selection pool per sequence, Sec. 5.2).
+#include <string>
+#include <vector>
+#include <cstdio>
+#include <cstring>
+#include <cstdarg>
+
+#include "../../include/ecmoe.h"
+#include "common.cuh"
+#include "kernels.h"
+#include "gemm_tc.h"
+
+using namespace ecmoe;
+
+struct ec_ctx {
+  int N = 0, d = 0, E = 0, F = 0, G = 0, dtype = 0;
+  int M_cap = 0, M = 0, max_group = 0;
+  std::vector<int32_t> group_off, k_g, k_off;
+  char* ws = nullptr;
+  size_t ws_bytes = 0;
+  // workspace offsets (bytes)
+  size_t o_status, o_goff, o_kg, o_koff, o_ST, o_S, o_idx, o_gate, o_slot, o_H, o_A, o_B, o_U,
+      o_O, o_dO, o_dA, o_dB, o_dgate, o_dZ, o_wrpad, o_f32a, o_f32b, o_dXr, o_part, total;
+  int wr_splits = 1;
+  // state saved by the forward pass
+  bool have_fwd = false;
+  const void *X = nullptr, *Wr = nullptr, *Wg = nullptr, *Wu = nullptr, *Wd = nullptr;
+  const float* br = nullptr;
+  std::string err;
+};
+
+namespace {
+
+ec_status fail(ec_ctx* c, ec_status s, const char* fmt, ...) {
+  if (c) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    c->err = buf;
+  }
+  return s;
+}
+
+ec_status cuda_fail(ec_ctx* c, cudaError_t e, const char* where) {
+  return fail(c, EC_ERR_CUDA, "%s: %s", where, cudaGetErrorString(e));
+}
+
+#define EC_CUDA(call, where)                         \
+  do {                                               \
+    cudaError_t _e = (call);                         \
+    if (_e != cudaSuccess) return cuda_fail(c, _e, where); \
+  } while (0)
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+size_t up256(size_t x) { return (x + 255) & ~size_t(255); }
+
+template <typename P>
+P* at(ec_ctx* c, size_t off) { return reinterpret_cast<P*>(c->ws + off); }
+
+size_t esize(const ec_ctx* c) { return c->dtype == EC_BF16 ? 2 : 4; }
+
+bool use_tc(const ec_ctx* c) { return c->dtype == EC_BF16; }
+
+void layout(ec_ctx* c) {
+  const size_t N = c->N, d = c->d, E = c->E, F = c->F, M = c->M_cap, G = c->G, es = esize(c);
+  const size_t P = E * M;
+  size_t o = 0;
+  auto take = [&](size_t bytes) { size_t r = o; o = up256(o + bytes); return r; };
+  c->o_status = take(256);
+  c->o_goff = take((G + 1) * 4);
+  c->o_kg = take(G * 4);
+  c->o_koff = take((G + 1) * 4);
+  c->o_ST = take(E * N * 4);
+  c->o_S = take(N * E * 4);
+  c->o_idx = take(P * 4);
+  c->o_gate = take(P * 4);
+  c->o_slot = take(N * E * 4);
+  c->o_H = take(P * d * es);
+  c->o_A = take(P * F * es);
+  c->o_B = take(P * F * es);
+  c->o_U = take(P * F * es);
+  c->o_O = take(P * d * es);   // also holds dH in the backward pass
+  c->o_dO = take(P * d * es);
+  c->o_dA = take(P * F * es);
+  c->o_dB = take(P * F * es);
+  c->o_dgate = take(P * 4);
+  c->o_dZ = take(N * E * 4);
+  c->o_wrpad = take(d * ((E + 63) / 64 * 64) * 2);
+  // fp32 scratch: SIMT GEMM outputs (fp32 path) and router logits / router dX part
+  const size_t f32n = use_tc(c) ? N * E : std::max(std::max(P * F, P * d), N * E);
+  c->o_f32a = take(f32n * 4);
+  c->o_f32b = take((use_tc(c) ? 0 : std::max(P * F, P * d)) * 4);
+  c->o_dXr = take(N * d * 4);
+  // split-K partials of dWr = X^T dZ
+  c->wr_splits = (int)std::max<size_t>(1, std::min<size_t>(64, N / 512));
+  c->o_part = take((size_t)c->wr_splits * d * E * 4);
+  c->total = o;
+}
+
+ec_status check_ready(ec_ctx* c) {
+  if (!c) return EC_ERR_INVALID_ARG;
+  if (!c->ws) return fail(c, EC_ERR_WORKSPACE, "no workspace attached (ec_ctx_set_workspace)");
+  return EC_OK;
+}
+
+ec_status set_groups(ec_ctx* c, const int32_t* group_off, const int32_t* k_g, bool creating) {
+  if (!group_off && creating) return fail(c, EC_ERR_INVALID_ARG, "group_off is NULL");
+  if (!k_g) return fail(c, EC_ERR_INVALID_ARG, "k_g is NULL");
+  const int G = c->G;
+  if (creating) {
+    if (group_off[0] != 0 || group_off[G] != c->N)
+      return fail(c, EC_ERR_SHAPE, "group_off must start at 0 and end at N=%d", c->N);
+    for (int g = 0; g < G; ++g)
+      if (group_off[g + 1] < group_off[g])
+        return fail(c, EC_ERR_SHAPE, "group_off must be non-decreasing (group %d)", g);
+  }
+  const int32_t* off = creating ? group_off : c->group_off.data();
+  int64_t M = 0;
+  int maxL = 0;
+  for (int g = 0; g < G; ++g) {
+    const int L = off[g + 1] - off[g];
+    if (k_g[g] < 0 || k_g[g] > L)
+      return fail(c, EC_ERR_SHAPE, "k_g[%d]=%d outside [0, %d]", g, k_g[g], L);
+    M += k_g[g];
+    maxL = std::max(maxL, L);
+  }
+  if (M > (int64_t)1 << 30) return fail(c, EC_ERR_UNSUPPORTED, "sum(k_g) too large");
+  if (!creating && M > c->M_cap)
+    return fail(c, EC_ERR_SHAPE, "sum(k_g)=%lld exceeds the context's capacity %d", (long long)M,
+                c->M_cap);
+  if (creating) {
+    c->group_off.assign(group_off, group_off + G + 1);
+    c->M_cap = (int)M;
+    c->max_group = maxL;
+  }
+  c->k_g.assign(k_g, k_g + G);
+  c->k_off.assign(G + 1, 0);
+  for (int g = 0; g < G; ++g) c->k_off[g + 1] = c->k_off[g] + k_g[g];
+  c->M = (int)M;
+  c->have_fwd = false;
+  return EC_OK;
+}
+
+ec_status upload_groups(ec_ctx* c) {
+  if (!c->ws) return EC_OK;
+  EC_CUDA(cudaMemcpy(at<int>(c, c->o_goff), c->group_off.data(), (c->G + 1) * 4,
+                     cudaMemcpyHostToDevice), "upload group_off");
+  EC_CUDA(cudaMemcpy(at<int>(c, c->o_kg), c->k_g.data(), c->G * 4, cudaMemcpyHostToDevice),
+          "upload k_g");
+  EC_CUDA(cudaMemcpy(at<int>(c, c->o_koff), c->k_off.data(), (c->G + 1) * 4,
+                     cudaMemcpyHostToDevice), "upload k_off");
+  return EC_OK;
+}
+
+// ---------------------------------------------------------------- SIMT GEMM helpers
+// Batched over experts: C[e] = A[e] . B[e] (+ beta C[e]).
+SimtGemmArgs sg(const void* A, int64_t a_bs, int64_t a_ms, int64_t a_ks, const void* B,
+                int64_t b_bs, int64_t b_ks, int64_t b_ns, float* C, int64_t c_bs, int64_t c_ms,
+                int M, int N, int K, int batch, float beta = 0.f) {
+  SimtGemmArgs a;
+  a.A = A; a.a_bs = a_bs; a.a_ms = a_ms; a.a_ks = a_ks;
+  a.B = B; a.b_bs = b_bs; a.b_ks = b_ks; a.b_ns = b_ns;
+  a.C = C; a.c_bs = c_bs; a.c_ms = c_ms;
+  a.M = M; a.N = N; a.K = K; a.batch = batch; a.splits = 1; a.c_split = 0; a.beta = beta;
+  return a;
+}
+
+EType et(const ec_ctx* c) { return c->dtype == EC_BF16 ? EType::BF16 : EType::F32; }
+
+// ---------------------------------------------------------------- router + selection
+template <typename T>
+ec_status run_route(ec_ctx* c, const void* X, const void* Wr, const float* br, const float* S_in,
+                    cudaStream_t st) {
+  const int N = c->N, E = c->E, d = c->d;
+  float* ST = at<float>(c, c->o_ST);
+  float* S = at<float>(c, c->o_S);
+  if (S_in) {
+    EC_CUDA(cudaMemcpyAsync(ST, S_in, (size_t)E * N * 4, cudaMemcpyDeviceToDevice, st), "copy S_in");
+    EC_CUDA(launch_transpose_scores(ST, S, N, E, st), "transpose scores");
+  } else if (use_tc(c)) {
+    EC_CUDA(tc_router_softmax(X, Wr, at<void>(c, c->o_wrpad), br, S, ST, N, d, E, at<int>(c, c->o_status), st), "router");
+  } else {
+    float* Z = at<float>(c, c->o_f32a);
+    EC_CUDA(launch_simt_gemm(sg(X, 0, d, 1, Wr, 0, E, 1, Z, 0, E, N, E, d, 1), et(c), et(c), st),
+            "router gemm");
+    EC_CUDA(launch_softmax_rows(Z, br, S, ST, N, E, st), "router softmax");
+  }
+  EC_CUDA(launch_topk(ST, N, E, c->G, at<int>(c, c->o_goff), at<int>(c, c->o_kg),
+                      at<int>(c, c->o_koff), c->M, c->max_group, at<int>(c, c->o_idx),
+                      at<float>(c, c->o_gate), at<int>(c, c->o_slot), st),
+          "top-k");
+  return EC_OK;
+}
+
+ec_status copy_out(ec_ctx* c, int32_t* idx, float* gate, float* S_out, cudaStream_t st) {
+  const size_t P = (size_t)c->E * c->M;
+  if (idx && P)
+    EC_CUDA(cudaMemcpyAsync(idx, at<int>(c, c->o_idx), P * 4, cudaMemcpyDeviceToDevice, st), "idx out");
+  if (gate && P)
+    EC_CUDA(cudaMemcpyAsync(gate, at<float>(c, c->o_gate), P * 4, cudaMemcpyDeviceToDevice, st),
+            "gate out");
+  if (S_out)
+    EC_CUDA(cudaMemcpyAsync(S_out, at<float>(c, c->o_ST), (size_t)c->E * c->N * 4,
+                            cudaMemcpyDeviceToDevice, st), "S out");
+  return EC_OK;
+}
+
+// ---------------------------------------------------------------- forward
+template <typename T>
+ec_status run_forward(ec_ctx* c, const void* X, const void* Wg, const void* Wu, const void* Wd,
+                      void* Y, cudaStream_t st) {
+  const int N = c->N, d = c->d, E = c->E, F = c->F, M = c->M;
+  const int64_t P = (int64_t)E * M;
+  T* H = at<T>(c, c->o_H);
+  T* A = at<T>(c, c->o_A);
+  T* B = at<T>(c, c->o_B);
+  T* U = at<T>(c, c->o_U);
+  T* O = at<T>(c, c->o_O);
+  const int* idx = at<int>(c, c->o_idx);
+  EC_CUDA(launch_gather<T>(static_cast<const T*>(X), idx, H, P, d, st), "gather");
+  if (P > 0) {
+    if (use_tc(c)) {
+      EC_CUDA(tc_expert_up(H, Wg, Wu, A, B, U, E, M, d, F, at<int>(c, c->o_status), st), "gate/up gemm");
+      EC_CUDA(tc_expert_down(U, Wd, O, E, M, d, F, at<int>(c, c->o_status), st), "down gemm");
+    } else {
+      float* Ag = at<float>(c, c->o_f32a);
+      float* Bu = at<float>(c, c->o_f32b);
+      const int64_t hs = (int64_t)M * d, ws = (int64_t)d * F, os = (int64_t)M * F;
+      EC_CUDA(launch_simt_gemm(sg(H, hs, d, 1, Wg, ws, F, 1, Ag, os, F, M, F, d, E), et(c), et(c), st),
+              "gate gemm");
+      EC_CUDA(launch_simt_gemm(sg(H, hs, d, 1, Wu, ws, F, 1, Bu, os, F, M, F, d, E), et(c), et(c), st),
+              "up gemm");
+      EC_CUDA(launch_swiglu_fwd_ew<T>(Ag, Bu, A, B, U, P * F, st), "swiglu");
+      float* O32 = at<float>(c, c->o_f32a);
+      EC_CUDA(launch_simt_gemm(sg(U, os, F, 1, Wd, (int64_t)F * d, d, 1, O32, hs, d, M, d, F, E),
+                               et(c), et(c), st), "down gemm");
+      EC_CUDA(launch_convert<T>(O32, O, P * d, st), "convert O");
+    }
+  }
+  EC_CUDA(launch_combine<T>(O, at<float>(c, c->o_gate), at<int>(c, c->o_slot),
+                            static_cast<T*>(Y), N, E, M, d, st), "combine");
+  return EC_OK;
+}
+
+// ---------------------------------------------------------------- backward
+template <typename T>
+ec_status run_backward(ec_ctx* c, const void* dY, void* dX, float* dWr, float* dbr, float* dWg,
+                       float* dWu, float* dWd, cudaStream_t st) {
+  const int N = c->N, d = c->d, E = c->E, F = c->F, M = c->M;
+  const int64_t P = (int64_t)E * M;
+  T* H = at<T>(c, c->o_H);
+  T* A = at<T>(c, c->o_A);
+  T* B = at<T>(c, c->o_B);
+  T* U = at<T>(c, c->o_U);
+  T* O = at<T>(c, c->o_O);
+  T* dH = O;  // O is dead once dgate is formed
+  T* dO = at<T>(c, c->o_dO);
+  T* dA = at<T>(c, c->o_dA);
+  T* dB = at<T>(c, c->o_dB);
+  float* dgate = at<float>(c, c->o_dgate);
+  float* dZ = at<float>(c, c->o_dZ);
+  const int* idx = at<int>(c, c->o_idx);
+  const float* gate = at<float>(c, c->o_gate);
+  const int* slot = at<int>(c, c->o_slot);
+  const int64_t hs = (int64_t)M * d, fs = (int64_t)M * F, wgs = (int64_t)d * F;
+
+  EC_CUDA(launch_bwd_gather_scale<T>(static_cast<const T*>(dY), O, idx, gate, dO, dgate, P, d, st),
+          "dO/dgate");
+  if (P > 0) {
+    if (use_tc(c)) {
+      EC_CUDA(tc_expert_dgrad_up(dO, c->Wd, A, B, dA, dB, E, M, d, F, at<int>(c, c->o_status), st),
+              "dU gemm");
+      EC_CUDA(tc_expert_dgrad_h(dA, dB, c->Wg, c->Wu, dH, E, M, d, F, at<int>(c, c->o_status), st),
+              "dH gemm");
+      EC_CUDA(tc_expert_wgrad(H, U, dO, dA, dB, dWg, dWu, dWd, E, M, d, F,
+                              at<int>(c, c->o_status), st), "weight-grad gemm");
+    } else {
+      float* dU32 = at<float>(c, c->o_f32a);
+      float* dH32 = at<float>(c, c->o_f32b);
+      // dU = dO . Wd^T : B[k=i][n=j] = Wd[j][i]
+      EC_CUDA(launch_simt_gemm(sg(dO, hs, d, 1, c->Wd, (int64_t)F * d, 1, d, dU32, fs, F, M, F, d, E),
+                               et(c), et(c), st), "dU gemm");
+      EC_CUDA(launch_swiglu_bwd_ew<T>(dU32, A, B, dA, dB, P * F, st), "swiglu bwd");
+      // dH = dA . Wg^T + dB . Wu^T
+      EC_CUDA(launch_simt_gemm(sg(dA, fs, F, 1, c->Wg, wgs, 1, F, dH32, hs, d, M, d, F, E),
+                               et(c), et(c), st), "dH gemm (gate)");
+      EC_CUDA(launch_simt_gemm(sg(dB, fs, F, 1, c->Wu, wgs, 1, F, dH32, hs, d, M, d, F, E, 1.f),
+                               et(c), et(c), st), "dH gemm (up)");
+      EC_CUDA(launch_convert<T>(dH32, dH, P * d, st), "convert dH");
+      // dWd = U^T dO ; dWg = H^T dA ; dWu = H^T dB   (A[m][k] = U[k][m])
+      EC_CUDA(launch_simt_gemm(sg(U, fs, 1, F, dO, hs, d, 1, dWd, (int64_t)F * d, d, F, d, M, E),
+                               et(c), et(c), st), "dWd gemm");
+      EC_CUDA(launch_simt_gemm(sg(H, hs, 1, d, dA, fs, F, 1, dWg, wgs, F, d, F, M, E),
+                               et(c), et(c), st), "dWg gemm");
+      EC_CUDA(launch_simt_gemm(sg(H, hs, 1, d, dB, fs, F, 1, dWu, wgs, F, d, F, M, E),
+                               et(c), et(c), st), "dWu gemm");
+    }
+  } else {
+    EC_CUDA(cudaMemsetAsync(dWg, 0, (size_t)E * d * F * 4, st), "zero dWg");
+    EC_CUDA(cudaMemsetAsync(dWu, 0, (size_t)E * d * F * 4, st), "zero dWu");
+    EC_CUDA(cudaMemsetAsync(dWd, 0, (size_t)E * d * F * 4, st), "zero dWd");
+  }
+  // router: dZ = S (dS - <dS,S>), dX = dZ Wr^T + sum dH, dWr = X^T dZ, dbr = sum dZ
+  EC_CUDA(launch_softmax_bwd(at<float>(c, c->o_S), slot, dgate, dZ, N, E, M, st), "softmax bwd");
+  float* dXr = at<float>(c, c->o_dXr);
+  EC_CUDA(launch_simt_gemm(sg(dZ, 0, E, 1, c->Wr, 0, 1, E, dXr, 0, d, N, d, E, 1), EType::F32, et(c), st),
+          "dZ Wr^T");
+  EC_CUDA(launch_dx_combine<T>(dH, slot, dXr, static_cast<T*>(dX), N, E, M, d, st), "dX");
+  {
+    SimtGemmArgs a = sg(c->X, 0, 1, d, dZ, 0, E, 1, at<float>(c, c->o_part), 0, E, d, E, N, 1);
+    a.splits = c->wr_splits;
+    a.c_split = (int64_t)d * E;
+    EC_CUDA(launch_simt_gemm(a, et(c), EType::F32, st), "X^T dZ");
+    EC_CUDA(launch_reduce_splits(at<float>(c, c->o_part), dWr, (int64_t)d * E, c->wr_splits, st),
+            "dWr reduce");
+  }
+  if (dbr) EC_CUDA(launch_colsum(dZ, dbr, N, E, st), "dbr");
+  return EC_OK;
+}
+
+}  // namespace
+
+// ====================================================================== C ABI
+extern "C" {
+
+const char* ec_status_string(ec_status s) {
+  switch (s) {
+    case EC_OK: return "EC_OK";
+    case EC_ERR_INVALID_ARG: return "EC_ERR_INVALID_ARG";
+    case EC_ERR_SHAPE: return "EC_ERR_SHAPE";
+    case EC_ERR_UNSUPPORTED: return "EC_ERR_UNSUPPORTED";
+    case EC_ERR_CUDA: return "EC_ERR_CUDA";
+    case EC_ERR_TIMEOUT: return "EC_ERR_TIMEOUT";
+    case EC_ERR_WORKSPACE: return "EC_ERR_WORKSPACE";
+    case EC_ERR_STATE: return "EC_ERR_STATE";
+  }
+  return "EC_ERR_UNKNOWN";
+}
+
+ec_status ec_ctx_create(ec_ctx** out, int32_t N, int32_t d, int32_t E, int32_t d_ff, int32_t G,
+                        const int32_t* group_off, const int32_t* k_g, int32_t dtype) {
+  if (!out) return EC_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (dtype != EC_F32 && dtype != EC_BF16) return EC_ERR_INVALID_ARG;
+  if (N < 0 || d <= 0 || E <= 0 || d_ff <= 0 || G <= 0) return EC_ERR_SHAPE;
+  if (E > 512) return EC_ERR_UNSUPPORTED;
+  if (dtype == EC_BF16 && (d % 64 || d_ff % 64)) return EC_ERR_UNSUPPORTED;
+  if (dtype == EC_F32 && (d % 4 || d_ff % 4)) return EC_ERR_UNSUPPORTED;
+  if (dtype == EC_BF16 && E > 256) return EC_ERR_UNSUPPORTED;
+  ec_ctx* c = new ec_ctx();
+  c->N = N; c->d = d; c->E = E; c->F = d_ff; c->G = G; c->dtype = dtype;
+  ec_status s = set_groups(c, group_off, k_g, true);
+  if (s != EC_OK) { delete c; return s; }
+  layout(c);
+  *out = c;
+  return EC_OK;
+}
+
+void ec_ctx_destroy(ec_ctx* c) { delete c; }
+
+ec_status ec_ctx_set_capacity(ec_ctx* c, const int32_t* k_g) {
+  if (!c) return EC_ERR_INVALID_ARG;
+  ec_status s = set_groups(c, nullptr, k_g, false);
+  if (s != EC_OK) return s;
+  return upload_groups(c);
+}
+
+int64_t ec_rows_per_expert(const ec_ctx* c) { return c ? c->M : -1; }
+
+size_t ec_workspace_bytes(const ec_ctx* c) { return c ? c->total : 0; }
+
+ec_status ec_ctx_set_workspace(ec_ctx* c, void* ws, size_t bytes) {
+  if (!c) return EC_ERR_INVALID_ARG;
+  if (!ws) return fail(c, EC_ERR_WORKSPACE, "workspace is NULL");
+  if (reinterpret_cast<uintptr_t>(ws) & 255u)
+    return fail(c, EC_ERR_WORKSPACE, "workspace must be 256-byte aligned");
+  if (bytes < c->total)
+    return fail(c, EC_ERR_WORKSPACE, "workspace has %zu bytes, needs %zu", bytes, c->total);
+  c->ws = static_cast<char*>(ws);
+  c->ws_bytes = bytes;
+  c->have_fwd = false;
+  EC_CUDA(cudaMemset(c->ws + c->o_status, 0, 256), "clear status");
+  return upload_groups(c);
+}
+
+ec_status ec_route(ec_ctx* c, const void* X, const void* Wr, const float* br, const float* S_in,
+                   float* S_out, int32_t* idx, float* gate, void* stream) {
+  ec_status s = check_ready(c);
+  if (s != EC_OK) return s;
+  if (!S_in && (!X || !Wr)) return fail(c, EC_ERR_INVALID_ARG, "X and Wr are required without S_in");
+  if (!idx || !gate) return fail(c, EC_ERR_INVALID_ARG, "idx and gate are required");
+  if ((X && !aligned16(X)) || (Wr && !aligned16(Wr)) || (S_in && !aligned16(S_in)))
+    return fail(c, EC_ERR_INVALID_ARG, "inputs must be 16-byte aligned");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  c->have_fwd = false;
+  s = c->dtype == EC_BF16 ? run_route<bf16>(c, X, Wr, br, S_in, st)
+                          : run_route<float>(c, X, Wr, br, S_in, st);
+  if (s != EC_OK) return s;
+  return copy_out(c, idx, gate, S_out, st);
+}
+
+ec_status ec_moe_forward(ec_ctx* c, const void* X, const void* Wr, const float* br, const void* Wg,
+                         const void* Wu, const void* Wd, void* Y, int32_t* idx, float* gate,
+                         float* S_out, void* stream) {
+  ec_status s = check_ready(c);
+  if (s != EC_OK) return s;
+  if (!X || !Wr || !Wg || !Wu || !Wd || !Y)
+    return fail(c, EC_ERR_INVALID_ARG, "X, Wr, Wg, Wu, Wd and Y are required");
+  for (const void* p : {X, Wr, Wg, Wu, Wd, (const void*)Y})
+    if (!aligned16(p)) return fail(c, EC_ERR_INVALID_ARG, "tensors must be 16-byte aligned");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  c->have_fwd = false;
+  s = c->dtype == EC_BF16 ? run_route<bf16>(c, X, Wr, br, nullptr, st)
+                          : run_route<float>(c, X, Wr, br, nullptr, st);
+  if (s != EC_OK) return s;
+  s = c->dtype == EC_BF16 ? run_forward<bf16>(c, X, Wg, Wu, Wd, Y, st)
+                          : run_forward<float>(c, X, Wg, Wu, Wd, Y, st);
+  if (s != EC_OK) return s;
+  s = copy_out(c, idx, gate, S_out, st);
+  if (s != EC_OK) return s;
+  c->X = X; c->Wr = Wr; c->br = br; c->Wg = Wg; c->Wu = Wu; c->Wd = Wd;
+  c->have_fwd = true;
+  return EC_OK;
+}
+
+ec_status ec_moe_backward(ec_ctx* c, const void* dY, void* dX, float* dWr, float* dbr, float* dWg,
+                          float* dWu, float* dWd, void* stream) {
+  ec_status s = check_ready(c);
+  if (s != EC_OK) return s;
+  if (!c->have_fwd) return fail(c, EC_ERR_STATE, "ec_moe_backward needs a preceding ec_moe_forward");
+  if (!dY || !dX || !dWr || !dWg || !dWu || !dWd)
+    return fail(c, EC_ERR_INVALID_ARG, "dY, dX, dWr, dWg, dWu and dWd are required");
+  for (const void* p : {dY, (const void*)dX, (const void*)dWr, (const void*)dWg, (const void*)dWu,
+                        (const void*)dWd})
+    if (!aligned16(p)) return fail(c, EC_ERR_INVALID_ARG, "tensors must be 16-byte aligned");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  return c->dtype == EC_BF16 ? run_backward<bf16>(c, dY, dX, dWr, dbr, dWg, dWu, dWd, st)
+                             : run_backward<float>(c, dY, dX, dWr, dbr, dWg, dWu, dWd, st);
+}
+
+ec_status ec_check_device(ec_ctx* c, void* stream) {
+  ec_status s = check_ready(c);
+  if (s != EC_OK) return s;
+  EC_CUDA(cudaStreamSynchronize(static_cast<cudaStream_t>(stream)), "stream sync");
+  int word = 0;
+  EC_CUDA(cudaMemcpy(&word, c->ws + c->o_status, 4, cudaMemcpyDeviceToHost), "read status");
+  if (word != DEV_OK) {
+    EC_CUDA(cudaMemset(c->ws + c->o_status, 0, 256), "clear status");
+    return fail(c, EC_ERR_TIMEOUT, "a kernel gave up on a bounded wait (device status %d)", word);
+  }
+  return EC_OK;
+}
+
+const char* ec_last_error(const ec_ctx* c) { return c ? c->err.c_str() : ""; }
+
+}  // extern "C"

@@ -1,0 +1,742 @@
+// Persistent, warp-specialised tcgen05 GEMM for sm_103a with fused epilogues.
+//
+// One CTA per SM walks a static list of 128 x BN output tiles over a uniform batch of
+// problems (one per expert: expert choice gives every expert the same M rows, arXiv
+// 2604.01622 Sec. 2.2). Roles:
+//   warp 0      TMA producer: 3-D tensor-map loads of A and B k-slices (64 deep, 128-byte
+//               swizzle) into a STAGES-deep shared-memory ring, one mbarrier per slot.
+//   warp 1      allocates TMEM; one thread issues tcgen05.mma (kind::f16, bf16 in, fp32
+//               accumulate) into one of two TMEM accumulators and commits slot releases
+//               and "accumulator full" to mbarriers.
+//   warps 2..5  epilogue: tcgen05.ld of the accumulator (one TMEM lane = one output row),
+//               fused math (router softmax, SwiGLU, SwiGLU backward, casts), global
+//               stores; then release the accumulator so the next tile's MMAs can reuse it.
+// Operands may be K-major or MN-major in global memory (tensor-core transpose bits), so
+// no operand is ever repacked. Every mbarrier wait is bounded in time: on expiry the CTA
+// records DEV_TIMEOUT in the status word, all roles leave their loops, and TMEM is freed.
+#include <cuda.h>
+#include <cstdio>
+#include "common.cuh"
+#include "gemm_tc.h"
+
+namespace ecmoe {
+namespace {
+
+constexpr int BM = 128;   // rows per tile = TMEM lanes
+constexpr int BK = 64;    // k-slice per stage: one 128-byte swizzle atom of bf16
+constexpr unsigned long long WAIT_LIMIT_NS = 2000000000ull;  // 2 s
+
+enum Epi : int {
+  EPI_ROUTER = 0,        // softmax over the (valid) columns, S [rows][E] and S^T [E][rows]
+  EPI_SWIGLU_FWD = 1,    // cols [0,BN/2) gate, [BN/2,BN) up -> A, B, U bf16
+  EPI_STORE_BF16 = 2,    // plain bf16 store
+  EPI_SWIGLU_BWD = 3,    // acc = dU; reads A, B; writes dA, dB bf16
+  EPI_STORE_F32 = 4,     // plain fp32 store
+  EPI_STORE_F32_SPLIT = 5  // cols [0,BN/2) -> out0, [BN/2,BN) -> out1, fp32
+};
+
+struct Args {
+  int batch, M, N, K;           // C[b] is M x N (N per half for split-column epilogues)
+  int m_tiles, n_tiles, k_blocks, k_blocks0;
+  void* out0;
+  void* out1;
+  void* out2;
+  const void* in0;
+  const void* in1;
+  const float* bias;
+  int64_t ld;                   // output row stride (elements)
+  int64_t bstride;              // output batch stride (elements)
+  int n_valid;                  // router: number of experts
+  int* status;
+};
+
+// ------------------------------------------------------------------ PTX wrappers
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count));
+}
+__device__ __forceinline__ void fence_mbar_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)),
+               "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+__device__ __forceinline__ unsigned long long globaltimer() {
+  unsigned long long t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+// Wait for the phase of `bar` with parity `parity`. Gives up after `limit` ns or when
+// another role of the CTA has given up; on expiry records DEV_TIMEOUT.
+__device__ __noinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
+                                       int* status, unsigned long long limit = WAIT_LIMIT_NS) {
+  const uint32_t a = smem_u32(bar);
+  if (mbar_try_wait(a, parity)) return true;
+  const unsigned long long t0 = globaltimer();
+  while (true) {
+    for (int i = 0; i < 32; ++i)
+      if (mbar_try_wait(a, parity)) return true;
+    if (*abort_flag) return false;
+    if (globaltimer() - t0 > limit) {
+      *abort_flag = 1;
+      atomicExch(status, DEV_TIMEOUT);
+      return false;
+    }
+  }
+}
+__device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, uint64_t* bar,
+                                            int c0, int c1, int c2) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%3, %4, %5}], [%2];" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(c0), "r"(c1), "r"(c2)
+      : "memory");
+}
+__device__ __forceinline__ void prefetch_map(const CUtensorMap* map) {
+  asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_alloc(uint32_t* holder, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                   smem_u32(holder)),
+               "r"(ncols)
+               : "memory");
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
+                                         uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+__device__ __forceinline__ void mma_commit(uint64_t* bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+          smem_u32(bar))
+      : "memory");
+}
+// 32 consecutive fp32 columns of this thread's TMEM lane.
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t* v) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+      "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+      : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]),
+        "=r"(v[7]), "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]),
+        "=r"(v[14]), "=r"(v[15]), "=r"(v[16]), "=r"(v[17]), "=r"(v[18]), "=r"(v[19]),
+        "=r"(v[20]), "=r"(v[21]), "=r"(v[22]), "=r"(v[23]), "=r"(v[24]), "=r"(v[25]),
+        "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]), "=r"(v[31])
+      : "r"(taddr));
+}
+__device__ __forceinline__ void tmem_wait_ld() {
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+// Shared-memory matrix descriptor (tcgen05 format): start, leading/stride byte offsets,
+// descriptor version 1, 128-byte swizzle.
+__device__ __forceinline__ uint64_t smem_desc(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr >> 4) & 0x3FFFu);
+  d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;
+  d |= (uint64_t)((sbo >> 4) & 0x3FFFu) << 32;
+  d |= (uint64_t)1u << 46;
+  d |= (uint64_t)2u << 61;
+  return d;
+}
+
+// Instruction descriptor of kind::f16: fp32 accumulator, bf16 A and B, M = 128.
+template <int BN, bool A_MN, bool B_MN>
+__host__ __device__ constexpr uint32_t instr_desc() {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((A_MN ? 1u : 0u) << 15) |
+         ((B_MN ? 1u : 0u) << 16) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
+}
+
+template <int BN>
+__host__ __device__ constexpr uint32_t tmem_cols() {
+  return 2 * BN <= 32 ? 32 : 2 * BN <= 64 ? 64 : 2 * BN <= 128 ? 128 : 2 * BN <= 256 ? 256 : 512;
+}
+
+template <int BN, int STAGES>
+__host__ __device__ constexpr uint32_t smem_bytes() {
+  return 1024 /*align slack*/ + STAGES * (BM * BK * 2 + BN * BK * 2) + 256 /*barriers*/;
+}
+
+__device__ __forceinline__ float f32(uint32_t u) { return __uint_as_float(u); }
+
+__device__ __forceinline__ void store_bf16x32(void* dst, const float* v) {
+  uint4* d = reinterpret_cast<uint4*>(dst);
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+    d[i] = make_uint4(pack_bf16x2(v[8 * i], v[8 * i + 1]), pack_bf16x2(v[8 * i + 2], v[8 * i + 3]),
+                      pack_bf16x2(v[8 * i + 4], v[8 * i + 5]),
+                      pack_bf16x2(v[8 * i + 6], v[8 * i + 7]));
+}
+__device__ __forceinline__ void load_bf16x32(const void* src, float* v) {
+  const uint4* s = reinterpret_cast<const uint4*>(src);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) unpack16(__ldg(s + i), v + 8 * i, bf16());
+}
+
+// ------------------------------------------------------------------ the kernel
+template <int BN, bool A_MN, bool B_MN, bool B_SPLIT, bool K_SPLIT, int EPI, int STAGES>
+__global__ void __launch_bounds__(192, 1)
+tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ CUtensorMap mA1,
+               const __grid_constant__ CUtensorMap mB0, const __grid_constant__ CUtensorMap mB1,
+               const Args p) {
+  constexpr uint32_t A_BYTES = BM * BK * 2;
+  constexpr uint32_t B_BYTES = BN * BK * 2;
+  constexpr uint32_t TCOLS = tmem_cols<BN>();
+  constexpr uint32_t IDESC = instr_desc<BN, A_MN, B_MN>();
+  static_assert(BN % 64 == 0 && BN <= 256, "BN");
+
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~uintptr_t(1023));
+  uint8_t* sA = smem;
+  uint8_t* sB = smem + STAGES * A_BYTES;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sB + STAGES * B_BYTES);
+  uint64_t* full = bars;
+  uint64_t* empty = bars + STAGES;
+  uint64_t* tfull = bars + 2 * STAGES;
+  uint64_t* tempty = tfull + 2;
+  uint64_t* mma_done = tempty + 2;
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(mma_done + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(&tfull[a], 1);
+      mbar_init(&tempty[a], 4);
+    }
+    mbar_init(mma_done, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 0 && lane == 0) {
+    prefetch_map(&mA0);
+    prefetch_map(&mB0);
+    if (K_SPLIT) prefetch_map(&mA1);
+    if (K_SPLIT || B_SPLIT) prefetch_map(&mB1);
+  }
+  if (warp == 1) tmem_alloc(tmem_holder, TCOLS);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_holder;
+
+  const int tiles_per_b = p.m_tiles * p.n_tiles;
+  const int total = p.batch * tiles_per_b;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ TMA producer
+    if (lane == 0) {
+      int s = 0;
+      uint32_t ph = 0;
+      bool ok = true;
+      for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x) {
+        const int b = tile / tiles_per_b;
+        const int rem = tile - b * tiles_per_b;
+        const int mt = rem / p.n_tiles, nt = rem - mt * p.n_tiles;
+        const int m0 = mt * BM;
+        for (int kb = 0; kb < p.k_blocks; ++kb) {
+          if (!mbar_wait(&empty[s], ph ^ 1u, abort_flag, p.status)) { ok = false; break; }
+          mbar_arrive_expect_tx(&full[s], A_BYTES + B_BYTES);
+          const bool second = K_SPLIT && kb >= p.k_blocks0;
+          const CUtensorMap* mA = second ? &mA1 : &mA0;
+          const CUtensorMap* mB = second ? &mB1 : &mB0;
+          const int k0 = (second ? kb - p.k_blocks0 : kb) * BK;
+          uint8_t* a_dst = sA + s * A_BYTES;
+          uint8_t* b_dst = sB + s * B_BYTES;
+          if (!A_MN) {
+            tma_load_3d(a_dst, mA, &full[s], k0, m0, b);
+          } else {
+#pragma unroll
+            for (int j = 0; j < BM / 64; ++j)
+              tma_load_3d(a_dst + j * 8192, mA, &full[s], m0 + 64 * j, k0, b);
+          }
+          if (!B_MN) {
+            if (B_SPLIT) {
+              const int n0h = nt * (BN / 2);
+              tma_load_3d(b_dst, &mB0, &full[s], k0, n0h, b);
+              tma_load_3d(b_dst + (BN / 2) * 128, &mB1, &full[s], k0, n0h, b);
+            } else {
+              tma_load_3d(b_dst, mB, &full[s], k0, nt * BN, b);
+            }
+          } else {
+            constexpr int NB = BN / 64;
+#pragma unroll
+            for (int j = 0; j < NB; ++j) {
+              if (B_SPLIT) {
+                const int n0h = nt * (BN / 2);
+                const CUtensorMap* m = j < NB / 2 ? &mB0 : &mB1;
+                tma_load_3d(b_dst + j * 8192, m, &full[s], n0h + 64 * (j % (NB / 2)), k0, b);
+              } else {
+                tma_load_3d(b_dst + j * 8192, mB, &full[s], nt * BN + 64 * j, k0, b);
+              }
+            }
+          }
+          if (++s == STAGES) { s = 0; ph ^= 1u; }
+        }
+      }
+      if (!ok) {
+        // let copies already issued land before the CTA leaves
+        const unsigned long long t0 = globaltimer();
+        while (globaltimer() - t0 < 1000000ull) {}
+      }
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      int s = 0;
+      uint32_t ph = 0;
+      bool ok = true;
+      int it = 0;
+      for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x, ++it) {
+        const int a = it & 1;
+        const uint32_t use = (uint32_t)(it >> 1);
+        if (!mbar_wait(&tempty[a], (use & 1u) ^ 1u, abort_flag, p.status)) { ok = false; break; }
+        tc_fence_after();
+        const uint32_t tacc = tmem_base + (uint32_t)(a * BN);
+        for (int kb = 0; kb < p.k_blocks; ++kb) {
+          if (!mbar_wait(&full[s], ph, abort_flag, p.status)) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t sa = smem_u32(sA + s * A_BYTES);
+          const uint32_t sb = smem_u32(sB + s * B_BYTES);
+#pragma unroll
+          for (int j = 0; j < BK / 16; ++j) {
+            const uint64_t ad = A_MN ? smem_desc(sa + j * 2048, 8192, 1024)
+                                     : smem_desc(sa + j * 32, 16, 1024);
+            const uint64_t bd = B_MN ? smem_desc(sb + j * 2048, 8192, 1024)
+                                     : smem_desc(sb + j * 32, 16, 1024);
+            mma_bf16(tacc, ad, bd, IDESC, (kb | j) != 0 ? 1u : 0u);
+          }
+          mma_commit(&empty[s]);
+          if (++s == STAGES) { s = 0; ph ^= 1u; }
+        }
+        if (!ok) break;
+        mma_commit(&tfull[a]);
+      }
+      if (!ok) {
+        // wait for the MMAs already issued before TMEM is released
+        mma_commit(mma_done);
+        volatile int keep_waiting = 0;
+        mbar_wait(mma_done, 0, &keep_waiting, p.status, 100000000ull);
+      }
+    }
+    __syncwarp();
+  } else {
+    // ------------------------------------------------------------ epilogue (warps 2..5)
+    const int q = warp & 3;             // TMEM lane quarter this warp may access
+    const int r = q * 32 + lane;        // row within the tile
+    int it = 0;
+    for (int tile = blockIdx.x; tile < total; tile += gridDim.x, ++it) {
+      const int a = it & 1;
+      const uint32_t use = (uint32_t)(it >> 1);
+      if (!mbar_wait(&tfull[a], use & 1u, abort_flag, p.status)) break;
+      tc_fence_after();
+      const int b = tile / tiles_per_b;
+      const int rem = tile - b * tiles_per_b;
+      const int mt = rem / p.n_tiles, nt = rem - mt * p.n_tiles;
+      const int gm = mt * BM + r;
+      const bool row_ok = gm < p.M;
+      const uint32_t tacc = tmem_base + (uint32_t)(a * BN) + ((uint32_t)(q * 32) << 16);
+      const int64_t row_off = (int64_t)b * p.bstride + (int64_t)gm * p.ld;
+      uint32_t v[32];
+      float f[32];
+
+      if constexpr (EPI == EPI_STORE_BF16 || EPI == EPI_STORE_F32) {
+#pragma unroll 1
+        for (int c = 0; c < BN / 32; ++c) {
+          tmem_ld32(tacc + c * 32, v);
+          tmem_wait_ld();
+          const int n = nt * BN + c * 32;
+          if (row_ok && n < p.N) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) f[i] = f32(v[i]);
+            if constexpr (EPI == EPI_STORE_BF16) {
+              store_bf16x32(reinterpret_cast<bf16*>(p.out0) + row_off + n, f);
+            } else {
+              float4* d4 = reinterpret_cast<float4*>(reinterpret_cast<float*>(p.out0) + row_off + n);
+#pragma unroll
+              for (int i = 0; i < 8; ++i) d4[i] = make_float4(f[4 * i], f[4 * i + 1], f[4 * i + 2], f[4 * i + 3]);
+            }
+          }
+        }
+      } else if constexpr (EPI == EPI_STORE_F32_SPLIT) {
+#pragma unroll 1
+        for (int c = 0; c < BN / 32; ++c) {
+          tmem_ld32(tacc + c * 32, v);
+          tmem_wait_ld();
+          const int half = c >= BN / 64;
+          const int n = nt * (BN / 2) + (c % (BN / 64)) * 32;
+          if (row_ok && n < p.N) {
+            float* out = reinterpret_cast<float*>(half ? p.out1 : p.out0) + row_off + n;
+            float4* d4 = reinterpret_cast<float4*>(out);
+#pragma unroll
+            for (int i = 0; i < 8; ++i)
+              d4[i] = make_float4(f32(v[4 * i]), f32(v[4 * i + 1]), f32(v[4 * i + 2]), f32(v[4 * i + 3]));
+          }
+        }
+      } else if constexpr (EPI == EPI_SWIGLU_FWD) {
+        uint32_t w[32];
+#pragma unroll 1
+        for (int c = 0; c < BN / 64; ++c) {
+          tmem_ld32(tacc + c * 32, v);
+          tmem_ld32(tacc + BN / 2 + c * 32, w);
+          tmem_wait_ld();
+          const int n = nt * (BN / 2) + c * 32;
+          if (row_ok && n < p.N) {
+            float g[32];
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+              const float av = f32(v[i]), bv = f32(w[i]);
+              f[i] = av;
+              g[i] = bv;
+            }
+            store_bf16x32(reinterpret_cast<bf16*>(p.out0) + row_off + n, f);
+            store_bf16x32(reinterpret_cast<bf16*>(p.out1) + row_off + n, g);
+#pragma unroll
+            for (int i = 0; i < 32; ++i) f[i] = f[i] * sigmoidf_(f[i]) * g[i];
+            store_bf16x32(reinterpret_cast<bf16*>(p.out2) + row_off + n, f);
+          }
+        }
+      } else if constexpr (EPI == EPI_SWIGLU_BWD) {
+#pragma unroll 1
+        for (int c = 0; c < BN / 32; ++c) {
+          tmem_ld32(tacc + c * 32, v);
+          tmem_wait_ld();
+          const int n = nt * BN + c * 32;
+          if (row_ok && n < p.N) {
+            float av[32], bv[32];
+            load_bf16x32(reinterpret_cast<const bf16*>(p.in0) + row_off + n, av);
+            load_bf16x32(reinterpret_cast<const bf16*>(p.in1) + row_off + n, bv);
+            float db[32];
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+              const float du = f32(v[i]);
+              const float sg = sigmoidf_(av[i]);
+              f[i] = du * bv[i] * sg * (1.0f + av[i] * (1.0f - sg));
+              db[i] = du * av[i] * sg;
+            }
+            store_bf16x32(reinterpret_cast<bf16*>(p.out0) + row_off + n, f);
+            store_bf16x32(reinterpret_cast<bf16*>(p.out1) + row_off + n, db);
+          }
+        }
+      } else if constexpr (EPI == EPI_ROUTER) {
+        const int E = p.n_valid;
+        float mx = -INFINITY;
+#pragma unroll 1
+        for (int c = 0; c < BN / 32; ++c) {
+          tmem_ld32(tacc + c * 32, v);
+          tmem_wait_ld();
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            const int e = c * 32 + i;
+            if (e < E) mx = fmaxf(mx, f32(v[i]) + (p.bias ? p.bias[e] : 0.f));
+          }
+        }
+        float sum = 0.f;
+#pragma unroll 1
+        for (int c = 0; c < BN / 32; ++c) {
+          tmem_ld32(tacc + c * 32, v);
+          tmem_wait_ld();
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            const int e = c * 32 + i;
+            if (e < E) sum += expf(f32(v[i]) + (p.bias ? p.bias[e] : 0.f) - mx);
+          }
+        }
+        const float inv = 1.0f / sum;
+        float* S = reinterpret_cast<float*>(p.out0);
+        float* ST = reinterpret_cast<float*>(p.out1);
+#pragma unroll 1
+        for (int c = 0; c < BN / 32; ++c) {
+          tmem_ld32(tacc + c * 32, v);
+          tmem_wait_ld();
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            const int e = c * 32 + i;
+            if (e < E && row_ok) {
+              const float pr = expf(f32(v[i]) + (p.bias ? p.bias[e] : 0.f) - mx) * inv;
+              S[(int64_t)gm * E + e] = pr;
+              ST[(int64_t)e * p.M + gm] = pr;
+            }
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&tempty[a]);
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, TCOLS);
+  }
+}
+
+// ------------------------------------------------------------------ host side
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  if (!fn) {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(ptr);
+  }
+  return fn;
+}
+
+// 3-D bf16 tensor [batch][rows][cols] (cols contiguous), box {64, box_rows, 1}, 128B swizzle.
+cudaError_t make_map(CUtensorMap* m, const void* base, uint64_t cols, uint64_t rows,
+                     uint64_t batch, uint32_t box_rows) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return cudaErrorNotSupported;
+  cuuint64_t dims[3] = {cols, rows, batch};
+  cuuint64_t strides[2] = {cols * 2, cols * rows * 2};
+  cuuint32_t box[3] = {64, box_rows, 1};
+  cuuint32_t estr[3] = {1, 1, 1};
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides,
+                  box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
+int sm_count() {
+  static int n = 0;
+  if (!n) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    if (n <= 0) n = 1;
+  }
+  return n;
+}
+
+template <int BN, bool A_MN, bool B_MN, bool B_SPLIT, bool K_SPLIT, int EPI, int STAGES>
+cudaError_t launch(const CUtensorMap& a0, const CUtensorMap& a1, const CUtensorMap& b0,
+                   const CUtensorMap& b1, const Args& p, cudaStream_t st) {
+  auto kern = tc_gemm_kernel<BN, A_MN, B_MN, B_SPLIT, K_SPLIT, EPI, STAGES>;
+  constexpr uint32_t smem = smem_bytes<BN, STAGES>();
+  static bool attr = false;
+  if (!attr) {
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+    attr = true;
+  }
+  const int total = p.batch * p.m_tiles * p.n_tiles;
+  if (total == 0 || p.k_blocks == 0) return cudaSuccess;
+  const int grid = total < sm_count() ? total : sm_count();
+  kern<<<grid, 192, smem, st>>>(a0, a1, b0, b1, p);
+  return cudaGetLastError();
+}
+
+Args base_args(int batch, int M, int N, int K, int BN_tile, int* status) {
+  Args p{};
+  p.batch = batch;
+  p.M = M;
+  p.N = N;
+  p.K = K;
+  p.m_tiles = (M + BM - 1) / BM;
+  p.n_tiles = (N + BN_tile - 1) / BN_tile;
+  p.k_blocks = (K + BK - 1) / BK;
+  p.k_blocks0 = p.k_blocks;
+  p.status = status;
+  return p;
+}
+
+__global__ void pad_router_weights(const bf16* __restrict__ Wr, bf16* __restrict__ Wp, int d,
+                                   int E, int Ep) {
+  const int64_t n = (int64_t)d * Ep;
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+       i += (int64_t)gridDim.x * blockDim.x) {
+    const int e = (int)(i % Ep);
+    const int64_t k = i / Ep;
+    Wp[i] = e < E ? Wr[k * E + e] : __float2bfloat16_rn(0.f);
+  }
+}
+
+__global__ void wait_probe_kernel(int* status, unsigned long long limit) {
+  __shared__ uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    abort_flag = 0;
+    fence_mbar_init();
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) mbar_wait(&bar, 0, &abort_flag, status, limit);
+}
+
+}  // namespace
+
+#define TC_TRY(x)                        \
+  do {                                   \
+    cudaError_t _e = (x);                \
+    if (_e != cudaSuccess) return _e;    \
+  } while (0)
+
+cudaError_t tc_router_softmax(const void* X, const void* Wr, void* Wr_pad, const float* br,
+                              float* S, float* ST, int N, int d, int E, int* status,
+                              cudaStream_t st) {
+  if (N == 0) return cudaSuccess;
+  const int Ep = (E + 63) / 64 * 64;
+  pad_router_weights<<<256, 256, 0, st>>>(static_cast<const bf16*>(Wr), static_cast<bf16*>(Wr_pad),
+                                          d, E, Ep);
+  TC_TRY(cudaGetLastError());
+  CUtensorMap ma, mb;
+  TC_TRY(make_map(&ma, X, d, N, 1, BM));
+  TC_TRY(make_map(&mb, Wr_pad, Ep, d, 1, 64));
+  Args p = base_args(1, N, Ep, d, Ep, status);
+  p.out0 = S;
+  p.out1 = ST;
+  p.bias = br;
+  p.n_valid = E;
+  switch (Ep) {
+    case 64: return launch<64, false, true, false, false, EPI_ROUTER, 8>(ma, ma, mb, mb, p, st);
+    case 128: return launch<128, false, true, false, false, EPI_ROUTER, 6>(ma, ma, mb, mb, p, st);
+    case 192: return launch<192, false, true, false, false, EPI_ROUTER, 5>(ma, ma, mb, mb, p, st);
+    case 256: return launch<256, false, true, false, false, EPI_ROUTER, 4>(ma, ma, mb, mb, p, st);
+  }
+  return cudaErrorInvalidValue;
+}
+
+cudaError_t tc_expert_up(const void* H, const void* Wg, const void* Wu, void* A, void* B, void* U,
+                         int E, int M, int d, int F, int* status, cudaStream_t st) {
+  CUtensorMap ma, mg, mu;
+  TC_TRY(make_map(&ma, H, d, M, E, BM));
+  TC_TRY(make_map(&mg, Wg, F, d, E, 64));
+  TC_TRY(make_map(&mu, Wu, F, d, E, 64));
+  Args p = base_args(E, M, F, d, 128, status);
+  p.out0 = A;
+  p.out1 = B;
+  p.out2 = U;
+  p.ld = F;
+  p.bstride = (int64_t)M * F;
+  return launch<256, false, true, true, false, EPI_SWIGLU_FWD, 4>(ma, ma, mg, mu, p, st);
+}
+
+cudaError_t tc_expert_down(const void* U, const void* Wd, void* O, int E, int M, int d, int F,
+                           int* status, cudaStream_t st) {
+  CUtensorMap ma, mb;
+  TC_TRY(make_map(&ma, U, F, M, E, BM));
+  TC_TRY(make_map(&mb, Wd, d, F, E, 64));
+  Args p = base_args(E, M, d, F, 256, status);
+  p.out0 = O;
+  p.ld = d;
+  p.bstride = (int64_t)M * d;
+  return launch<256, false, true, false, false, EPI_STORE_BF16, 4>(ma, ma, mb, mb, p, st);
+}
+
+cudaError_t tc_expert_dgrad_up(const void* dO, const void* Wd, const void* A, const void* B,
+                               void* dA, void* dB, int E, int M, int d, int F, int* status,
+                               cudaStream_t st) {
+  CUtensorMap ma, mb;
+  TC_TRY(make_map(&ma, dO, d, M, E, BM));
+  TC_TRY(make_map(&mb, Wd, d, F, E, 256));   // B[n=f][k=i] = Wd[f][i]: K-major
+  Args p = base_args(E, M, F, d, 256, status);
+  p.in0 = A;
+  p.in1 = B;
+  p.out0 = dA;
+  p.out1 = dB;
+  p.ld = F;
+  p.bstride = (int64_t)M * F;
+  return launch<256, false, false, false, false, EPI_SWIGLU_BWD, 4>(ma, ma, mb, mb, p, st);
+}
+
+cudaError_t tc_expert_dgrad_h(const void* dA, const void* dB, const void* Wg, const void* Wu,
+                              void* dH, int E, int M, int d, int F, int* status, cudaStream_t st) {
+  CUtensorMap ma0, ma1, mb0, mb1;
+  TC_TRY(make_map(&ma0, dA, F, M, E, BM));
+  TC_TRY(make_map(&ma1, dB, F, M, E, BM));
+  TC_TRY(make_map(&mb0, Wg, F, d, E, 256));  // B[n=i][k=f] = Wg[i][f]: K-major
+  TC_TRY(make_map(&mb1, Wu, F, d, E, 256));
+  Args p = base_args(E, M, d, 2 * F, 256, status);
+  p.k_blocks0 = F / BK;
+  p.out0 = dH;
+  p.ld = d;
+  p.bstride = (int64_t)M * d;
+  return launch<256, false, false, false, true, EPI_STORE_BF16, 4>(ma0, ma1, mb0, mb1, p, st);
+}
+
+cudaError_t tc_expert_wgrad(const void* H, const void* U, const void* dO, const void* dA,
+                            const void* dB, float* dWg, float* dWu, float* dWd, int E, int M,
+                            int d, int F, int* status, cudaStream_t st) {
+  {
+    // dWd[e] [F][d] = U[e]^T . dO[e]: A[m=f][k=t] = U[t][f] (MN-major), B[k=t][n=i] = dO[t][i]
+    CUtensorMap ma, mb;
+    TC_TRY(make_map(&ma, U, F, M, E, 64));
+    TC_TRY(make_map(&mb, dO, d, M, E, 64));
+    Args p = base_args(E, F, d, M, 256, status);
+    p.out0 = dWd;
+    p.ld = d;
+    p.bstride = (int64_t)F * d;
+    TC_TRY((launch<256, true, true, false, false, EPI_STORE_F32, 4>(ma, ma, mb, mb, p, st)));
+  }
+  {
+    // [dWg | dWu][e] [d][F] = H[e]^T . [dA | dB][e]
+    CUtensorMap ma, mb0, mb1;
+    TC_TRY(make_map(&ma, H, d, M, E, 64));
+    TC_TRY(make_map(&mb0, dA, F, M, E, 64));
+    TC_TRY(make_map(&mb1, dB, F, M, E, 64));
+    Args p = base_args(E, d, F, M, 128, status);
+    p.out0 = dWg;
+    p.out1 = dWu;
+    p.ld = F;
+    p.bstride = (int64_t)d * F;
+    TC_TRY((launch<256, true, true, true, false, EPI_STORE_F32_SPLIT, 4>(ma, ma, mb0, mb1, p, st)));
+  }
+  return cudaSuccess;
+}
+
+cudaError_t tc_wait_probe(int* status, unsigned long long limit_ns, cudaStream_t st) {
+  wait_probe_kernel<<<1, 32, 0, st>>>(status, limit_ns);
+  return cudaGetLastError();
+}
+
+}  // namespace ecmoe

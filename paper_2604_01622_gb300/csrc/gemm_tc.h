@@ -1,0 +1,46 @@
+// Tensor-core (tcgen05 + TMEM + TMA) GEMMs of the bf16 EC-MoE path. Internal.
+//
+// Expert choice gives every expert the same row count M (arXiv 2604.01622, Sec. 2.2:
+// each expert processes exactly its capacity), so every expert GEMM is a uniform batch
+// over E experts with 3-D TMA tensor maps [E][rows][cols].
+#pragma once
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace ecmoe {
+
+// Router: Z = X.Wr (+br), S = row softmax over the E experts, written as S [N][E] and
+// S^T [E][N]. X [N][d] bf16, Wr [d][E] bf16. Wr_pad: device scratch of d*round_up(E,64)
+// bf16 (zero-padded copy of Wr made on the stream).
+cudaError_t tc_router_softmax(const void* X, const void* Wr, void* Wr_pad, const float* br,
+                              float* S, float* ST, int N, int d, int E, int* status,
+                              cudaStream_t st);
+
+// [A | B] = H.[Wg | Wu] per expert; U = silu(A) * B. H [E][M][d]; Wg, Wu [E][d][F];
+// A, B, U [E][M][F] bf16.
+cudaError_t tc_expert_up(const void* H, const void* Wg, const void* Wu, void* A, void* B, void* U,
+                         int E, int M, int d, int F, int* status, cudaStream_t st);
+
+// O = U.Wd per expert. U [E][M][F]; Wd [E][F][d]; O [E][M][d] bf16.
+cudaError_t tc_expert_down(const void* U, const void* Wd, void* O, int E, int M, int d, int F,
+                           int* status, cudaStream_t st);
+
+// dU = dO.Wd^T per expert, then dA = dU * B * silu'(A), dB = dU * silu(A) (bf16 out).
+cudaError_t tc_expert_dgrad_up(const void* dO, const void* Wd, const void* A, const void* B,
+                               void* dA, void* dB, int E, int M, int d, int F, int* status,
+                               cudaStream_t st);
+
+// dH = dA.Wg^T + dB.Wu^T per expert (one K loop over both halves). dH [E][M][d] bf16.
+cudaError_t tc_expert_dgrad_h(const void* dA, const void* dB, const void* Wg, const void* Wu,
+                              void* dH, int E, int M, int d, int F, int* status, cudaStream_t st);
+
+// Weight gradients per expert, fp32: dWd = U^T.dO, dWg = H^T.dA, dWu = H^T.dB.
+cudaError_t tc_expert_wgrad(const void* H, const void* U, const void* dO, const void* dA,
+                            const void* dB, float* dWg, float* dWu, float* dWd, int E, int M,
+                            int d, int F, int* status, cudaStream_t st);
+
+// Launch a kernel that waits, with the given limit, on an mbarrier nothing completes, so
+// the bounded-wait path (status word, early return) can be exercised without a hang.
+cudaError_t tc_wait_probe(int* status, unsigned long long limit_ns, cudaStream_t st);
+
+}  // namespace ecmoe

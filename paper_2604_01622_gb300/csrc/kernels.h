@@ -1,0 +1,61 @@
+// Internal launchers of the EC-MoE library. Not part of the C ABI.
+#pragma once
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace ecmoe {
+
+// ---------------------------------------------------------------- router + selection
+// Row softmax of fp32 logits Z [N][E] (+ br) -> S [N][E] and S^T [E][N].
+cudaError_t launch_softmax_rows(const float* Z, const float* br, float* S, float* ST, int N, int E,
+                                cudaStream_t st);
+// Transpose scores [E][N] -> [N][E] (used when the caller supplies S).
+cudaError_t launch_transpose_scores(const float* ST, float* S, int N, int E, cudaStream_t st);
+// Expert-choice top-k per (expert, group) over S^T [E][N]; writes idx/gate [E][M] and the
+// token->slot map slot [N][E] (m or -1).
+cudaError_t launch_topk(const float* ST, int N, int E, int G, const int* group_off, const int* k_g,
+                        const int* k_off, int M, int max_group, int* idx, float* gate, int* slot,
+                        cudaStream_t st);
+
+// ---------------------------------------------------------------- data movement
+template <typename T>
+cudaError_t launch_gather(const T* X, const int* idx, T* H, int64_t P, int d, cudaStream_t st);
+template <typename T>
+cudaError_t launch_combine(const T* O, const float* gate, const int* slot, T* Y, int N, int E,
+                           int M, int d, cudaStream_t st);
+template <typename T>
+cudaError_t launch_bwd_gather_scale(const T* dY, const T* O, const int* idx, const float* gate,
+                                    T* dO, float* dgate, int64_t P, int d, cudaStream_t st);
+cudaError_t launch_softmax_bwd(const float* S, const int* slot, const float* dgate, float* dZ,
+                               int N, int E, int M, cudaStream_t st);
+template <typename T>
+cudaError_t launch_dx_combine(const T* dH, const int* slot, const float* dXr, T* dX, int N, int E,
+                              int M, int d, cudaStream_t st);
+cudaError_t launch_colsum(const float* Z, float* out, int N, int E, cudaStream_t st);
+template <typename T>
+cudaError_t launch_swiglu_fwd_ew(const float* Ag, const float* Bu, T* A, T* B, T* U, int64_t n,
+                                 cudaStream_t st);
+template <typename T>
+cudaError_t launch_swiglu_bwd_ew(const float* dU, const T* A, const T* B, T* dA, T* dB,
+                                 int64_t n, cudaStream_t st);
+template <typename T>
+cudaError_t launch_convert(const float* in, T* out, int64_t n, cudaStream_t st);
+cudaError_t launch_reduce_splits(const float* part, float* out, int64_t n, int splits,
+                                 cudaStream_t st);
+
+// ---------------------------------------------------------------- fp32 SIMT GEMM
+// C[b] (+)= A[b] . B[b] with A logical [M][K], B logical [K][N], C [M][N] fp32 (unit column
+// stride). Element strides per operand; TA/TB are float or bf16.
+struct SimtGemmArgs {
+  const void* A; int64_t a_bs, a_ms, a_ks;
+  const void* B; int64_t b_bs, b_ks, b_ns;
+  float* C; int64_t c_bs, c_ms;
+  int M, N, K, batch;
+  int splits;                 // >1: split s writes C + s * c_split (beta ignored)
+  int64_t c_split;
+  float beta;                 // C = A.B + beta*C (splits == 1 only)
+};
+enum class EType { F32, BF16 };
+cudaError_t launch_simt_gemm(const SimtGemmArgs& a, EType ta, EType tb, cudaStream_t st);
+
+}  // namespace ecmoe

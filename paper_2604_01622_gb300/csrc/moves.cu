@@ -1,0 +1,340 @@
+// Bandwidth kernels of the EC-MoE layer: gather into expert-major rows, gated combine
+// (arXiv 2604.01622, Sec. 2.2: y_t = sum_{e: t in T_e} g_te FFN_e(x_t)), and their
+// backward (gate gradient, softmax Jacobian, scatter of the input gradient).
+//
+// The token->slot map slot[t][e] (row m of expert e, or -1) makes every per-token sum run
+// over experts in ascending order with no atomics, so results are deterministic.
+#include "common.cuh"
+#include "kernels.h"
+
+namespace ecmoe {
+
+// Grid of 256-thread blocks for a grid-stride loop over n elements, capped at `cap` blocks.
+static unsigned grid_for(int64_t n, int64_t cap) {
+  const int64_t b = (n + 255) / 256;
+  return (unsigned)(b < cap ? b : cap);
+}
+
+// ------------------------------------------------------------------ gather H[e][m] = X[idx[e][m]]
+template <typename T>
+__global__ void gather_kernel(const T* __restrict__ X, const int* __restrict__ idx,
+                              T* __restrict__ H, int64_t P, int d) {
+  const int64_t row = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (row >= P) return;
+  const int t = idx[row];
+  const int nv = d * (int)sizeof(T) / 16;
+  const uint4* src = reinterpret_cast<const uint4*>(X + (size_t)t * d);
+  uint4* dst = reinterpret_cast<uint4*>(H + (size_t)row * d);
+  for (int v = lane; v < nv; v += 32) dst[v] = __ldg(src + v);
+}
+
+template <typename T>
+cudaError_t launch_gather(const T* X, const int* idx, T* H, int64_t P, int d, cudaStream_t st) {
+  if (P == 0) return cudaSuccess;
+  const int warps = 8;
+  gather_kernel<T><<<(unsigned)((P + warps - 1) / warps), warps * 32, 0, st>>>(X, idx, H, P, d);
+  return cudaGetLastError();
+}
+
+// ------------------------------------------------------------------ per-token pair lists
+// Fills s_m/s_g (slot row, gate) of the experts that chose token t, ascending e. Returns count.
+__device__ __forceinline__ int token_pairs(const int* __restrict__ slot, const float* __restrict__ gate,
+                                           int t, int E, int M, int* s_e, int* s_m, float* s_g,
+                                           int* s_cnt) {
+  if (threadIdx.x < 32) {
+    const int lane = threadIdx.x;
+    int cnt = 0;
+    for (int e0 = 0; e0 < E; e0 += 32) {
+      const int e = e0 + lane;
+      const int m = e < E ? slot[(size_t)t * E + e] : -1;
+      const unsigned ball = __ballot_sync(0xffffffffu, m >= 0);
+      if (m >= 0) {
+        const int p = cnt + __popc(ball & ((1u << lane) - 1u));
+        s_e[p] = e;
+        s_m[p] = m;
+        if (s_g) s_g[p] = gate[(size_t)e * M + m];
+      }
+      cnt += __popc(ball);
+    }
+    if (lane == 0) *s_cnt = cnt;
+  }
+  __syncthreads();
+  return *s_cnt;
+}
+
+// ------------------------------------------------------------------ combine Y_t = sum g * O
+template <typename T>
+__global__ void combine_kernel(const T* __restrict__ O, const float* __restrict__ gate,
+                               const int* __restrict__ slot, T* __restrict__ Y, int N, int E, int M,
+                               int d) {
+  extern __shared__ int sh[];
+  int* s_e = sh;
+  int* s_m = sh + E;
+  float* s_g = reinterpret_cast<float*>(sh + 2 * E);
+  __shared__ int s_cnt;
+  const int t = blockIdx.x;
+  const int cnt = token_pairs(slot, gate, t, E, M, s_e, s_m, s_g, &s_cnt);
+  constexpr int VN = 16 / sizeof(T);
+  const int nv = d / VN;
+  for (int v = threadIdx.x; v < nv; v += blockDim.x) {
+    float acc[VN];
+#pragma unroll
+    for (int j = 0; j < VN; ++j) acc[j] = 0.f;
+    for (int p = 0; p < cnt; ++p) {
+      const size_t row = (size_t)s_e[p] * M + s_m[p];
+      const uint4 u = __ldg(reinterpret_cast<const uint4*>(O + row * d) + v);
+      float o[VN];
+      unpack16(u, o, T());
+      const float g = s_g[p];
+#pragma unroll
+      for (int j = 0; j < VN; ++j) acc[j] = fmaf(g, o[j], acc[j]);
+    }
+    reinterpret_cast<uint4*>(Y + (size_t)t * d)[v] = pack16(acc, T());
+  }
+}
+
+template <typename T>
+cudaError_t launch_combine(const T* O, const float* gate, const int* slot, T* Y, int N, int E,
+                           int M, int d, cudaStream_t st) {
+  if (N == 0) return cudaSuccess;
+  const size_t smem = (size_t)3 * E * sizeof(int);
+  combine_kernel<T><<<N, 128, smem, st>>>(O, gate, slot, Y, N, E, M, d);
+  return cudaGetLastError();
+}
+
+// ------------------------------------------------------------------ backward: dO = g dY_t, dgate = <dY_t, O>
+template <typename T>
+__global__ void bwd_gather_scale_kernel(const T* __restrict__ dY, const T* __restrict__ O,
+                                        const int* __restrict__ idx, const float* __restrict__ gate,
+                                        T* __restrict__ dO, float* __restrict__ dgate, int64_t P,
+                                        int d) {
+  const int64_t row = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (row >= P) return;
+  const int t = idx[row];
+  const float g = gate[row];
+  constexpr int VN = 16 / sizeof(T);
+  const int nv = d / VN;
+  const uint4* dy = reinterpret_cast<const uint4*>(dY + (size_t)t * d);
+  const uint4* o = reinterpret_cast<const uint4*>(O + (size_t)row * d);
+  uint4* out = reinterpret_cast<uint4*>(dO + (size_t)row * d);
+  float dot = 0.f;
+  for (int v = lane; v < nv; v += 32) {
+    float a[VN], b[VN], c[VN];
+    unpack16(__ldg(dy + v), a, T());
+    unpack16(__ldg(o + v), b, T());
+#pragma unroll
+    for (int j = 0; j < VN; ++j) {
+      dot = fmaf(a[j], b[j], dot);
+      c[j] = g * a[j];
+    }
+    out[v] = pack16(c, T());
+  }
+  dot = warp_sum(dot);
+  if (lane == 0) dgate[row] = dot;
+}
+
+template <typename T>
+cudaError_t launch_bwd_gather_scale(const T* dY, const T* O, const int* idx, const float* gate,
+                                    T* dO, float* dgate, int64_t P, int d, cudaStream_t st) {
+  if (P == 0) return cudaSuccess;
+  const int warps = 8;
+  bwd_gather_scale_kernel<T><<<(unsigned)((P + warps - 1) / warps), warps * 32, 0, st>>>(
+      dY, O, idx, gate, dO, dgate, P, d);
+  return cudaGetLastError();
+}
+
+// ------------------------------------------------------------------ softmax Jacobian
+// dS[t,e] = dgate of the pair (t chosen by e) else 0; dZ = S * (dS - <dS, S>).
+__global__ void softmax_bwd_kernel(const float* __restrict__ S, const int* __restrict__ slot,
+                                   const float* __restrict__ dgate, float* __restrict__ dZ, int N,
+                                   int E, int M) {
+  const int t = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (t >= N) return;
+  float dot = 0.f;
+  for (int e = lane; e < E; e += 32) {
+    const int m = slot[(size_t)t * E + e];
+    const float ds = m >= 0 ? dgate[(size_t)e * M + m] : 0.f;
+    dot = fmaf(ds, S[(size_t)t * E + e], dot);
+  }
+  dot = warp_sum(dot);
+  for (int e = lane; e < E; e += 32) {
+    const int m = slot[(size_t)t * E + e];
+    const float ds = m >= 0 ? dgate[(size_t)e * M + m] : 0.f;
+    const float s = S[(size_t)t * E + e];
+    dZ[(size_t)t * E + e] = s * (ds - dot);
+  }
+}
+
+cudaError_t launch_softmax_bwd(const float* S, const int* slot, const float* dgate, float* dZ,
+                               int N, int E, int M, cudaStream_t st) {
+  if (N == 0) return cudaSuccess;
+  softmax_bwd_kernel<<<(N + 7) / 8, 256, 0, st>>>(S, slot, dgate, dZ, N, E, M);
+  return cudaGetLastError();
+}
+
+// ------------------------------------------------------------------ dX_t = dXr_t + sum dH rows
+template <typename T>
+__global__ void dx_combine_kernel(const T* __restrict__ dH, const int* __restrict__ slot,
+                                  const float* __restrict__ dXr, T* __restrict__ dX, int N, int E,
+                                  int M, int d) {
+  extern __shared__ int sh[];
+  int* s_e = sh;
+  int* s_m = sh + E;
+  __shared__ int s_cnt;
+  const int t = blockIdx.x;
+  const int cnt = token_pairs(slot, nullptr, t, E, M, s_e, s_m, nullptr, &s_cnt);
+  constexpr int VN = 16 / sizeof(T);
+  const int nv = d / VN;
+  for (int v = threadIdx.x; v < nv; v += blockDim.x) {
+    float acc[VN];
+    if (dXr) {
+      const float4* r = reinterpret_cast<const float4*>(dXr + (size_t)t * d + (size_t)v * VN);
+#pragma unroll
+      for (int j = 0; j < VN / 4; ++j) {
+        float4 q = r[j];
+        acc[4 * j] = q.x; acc[4 * j + 1] = q.y; acc[4 * j + 2] = q.z; acc[4 * j + 3] = q.w;
+      }
+    } else {
+#pragma unroll
+      for (int j = 0; j < VN; ++j) acc[j] = 0.f;
+    }
+    for (int p = 0; p < cnt; ++p) {
+      const size_t row = (size_t)s_e[p] * M + s_m[p];
+      float h[VN];
+      unpack16(__ldg(reinterpret_cast<const uint4*>(dH + row * d) + v), h, T());
+#pragma unroll
+      for (int j = 0; j < VN; ++j) acc[j] += h[j];
+    }
+    reinterpret_cast<uint4*>(dX + (size_t)t * d)[v] = pack16(acc, T());
+  }
+}
+
+template <typename T>
+cudaError_t launch_dx_combine(const T* dH, const int* slot, const float* dXr, T* dX, int N, int E,
+                              int M, int d, cudaStream_t st) {
+  if (N == 0) return cudaSuccess;
+  const size_t smem = (size_t)2 * E * sizeof(int);
+  dx_combine_kernel<T><<<N, 128, smem, st>>>(dH, slot, dXr, dX, N, E, M, d);
+  return cudaGetLastError();
+}
+
+// ------------------------------------------------------------------ column sums of Z [N][E]
+__global__ void colsum_kernel(const float* __restrict__ Z, float* __restrict__ out, int N, int E) {
+  __shared__ float part[8][33];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int e = blockIdx.x * 32 + lane;
+  float s = 0.f;
+  if (e < E)
+    for (int t = warp; t < N; t += 8) s += Z[(size_t)t * E + e];
+  part[warp][lane] = s;
+  __syncthreads();
+  if (warp == 0 && e < E) {
+    float r = 0.f;
+    for (int w = 0; w < 8; ++w) r += part[w][lane];
+    out[e] = r;
+  }
+}
+
+cudaError_t launch_colsum(const float* Z, float* out, int N, int E, cudaStream_t st) {
+  colsum_kernel<<<(E + 31) / 32, 256, 0, st>>>(Z, out, N, E);
+  return cudaGetLastError();
+}
+
+// ------------------------------------------------------------------ SwiGLU elementwise (SIMT path)
+template <typename T>
+__global__ void swiglu_fwd_ew_kernel(const float* __restrict__ Ag, const float* __restrict__ Bu,
+                                     T* __restrict__ A, T* __restrict__ B, T* __restrict__ U,
+                                     int64_t n) {
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+       i += (int64_t)gridDim.x * blockDim.x) {
+    const float a = Ag[i], b = Bu[i];
+    A[i] = from_f32<T>(a);
+    B[i] = from_f32<T>(b);
+    U[i] = from_f32<T>(a * sigmoidf_(a) * b);
+  }
+}
+
+template <typename T>
+cudaError_t launch_swiglu_fwd_ew(const float* Ag, const float* Bu, T* A, T* B, T* U, int64_t n,
+                                 cudaStream_t st) {
+  if (n == 0) return cudaSuccess;
+  const unsigned blocks = grid_for(n, 152 * 64);
+  swiglu_fwd_ew_kernel<T><<<blocks, 256, 0, st>>>(Ag, Bu, A, B, U, n);
+  return cudaGetLastError();
+}
+
+template <typename T>
+__global__ void swiglu_bwd_ew_kernel(const float* __restrict__ dU, const T* __restrict__ A,
+                                     const T* __restrict__ B, T* __restrict__ dA,
+                                     T* __restrict__ dB, int64_t n) {
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+       i += (int64_t)gridDim.x * blockDim.x) {
+    const float a = to_f32(A[i]), b = to_f32(B[i]), du = dU[i];
+    const float s = sigmoidf_(a);
+    dA[i] = from_f32<T>(du * b * s * (1.0f + a * (1.0f - s)));
+    dB[i] = from_f32<T>(du * a * s);
+  }
+}
+
+template <typename T>
+cudaError_t launch_swiglu_bwd_ew(const float* dU, const T* A, const T* B, T* dA, T* dB,
+                                 int64_t n, cudaStream_t st) {
+  if (n == 0) return cudaSuccess;
+  const unsigned blocks = grid_for(n, 152 * 64);
+  swiglu_bwd_ew_kernel<T><<<blocks, 256, 0, st>>>(dU, A, B, dA, dB, n);
+  return cudaGetLastError();
+}
+
+template <typename T>
+__global__ void convert_kernel(const float* __restrict__ in, T* __restrict__ out, int64_t n) {
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+       i += (int64_t)gridDim.x * blockDim.x)
+    out[i] = from_f32<T>(in[i]);
+}
+
+template <typename T>
+cudaError_t launch_convert(const float* in, T* out, int64_t n, cudaStream_t st) {
+  if (n == 0) return cudaSuccess;
+  const unsigned blocks = grid_for(n, 152 * 64);
+  convert_kernel<T><<<blocks, 256, 0, st>>>(in, out, n);
+  return cudaGetLastError();
+}
+
+__global__ void reduce_splits_kernel(const float* __restrict__ part, float* __restrict__ out,
+                                     int64_t n, int splits) {
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+       i += (int64_t)gridDim.x * blockDim.x) {
+    float s = 0.f;
+    for (int k = 0; k < splits; ++k) s += part[(size_t)k * n + i];
+    out[i] = s;
+  }
+}
+
+cudaError_t launch_reduce_splits(const float* part, float* out, int64_t n, int splits,
+                                 cudaStream_t st) {
+  if (n == 0) return cudaSuccess;
+  const unsigned blocks = grid_for(n, 152 * 16);
+  reduce_splits_kernel<<<blocks, 256, 0, st>>>(part, out, n, splits);
+  return cudaGetLastError();
+}
+
+#define ECMOE_INST(T)                                                                            \
+  template cudaError_t launch_gather<T>(const T*, const int*, T*, int64_t, int, cudaStream_t);    \
+  template cudaError_t launch_combine<T>(const T*, const float*, const int*, T*, int, int, int,   \
+                                         int, cudaStream_t);                                      \
+  template cudaError_t launch_bwd_gather_scale<T>(const T*, const T*, const int*, const float*,   \
+                                                  T*, float*, int64_t, int, cudaStream_t);        \
+  template cudaError_t launch_dx_combine<T>(const T*, const int*, const float*, T*, int, int,     \
+                                            int, int, cudaStream_t);                              \
+  template cudaError_t launch_swiglu_fwd_ew<T>(const float*, const float*, T*, T*, T*, int64_t,   \
+                                               cudaStream_t);                                     \
+  template cudaError_t launch_swiglu_bwd_ew<T>(const float*, const T*, const T*, T*, T*,          \
+                                               int64_t, cudaStream_t);                            \
+  template cudaError_t launch_convert<T>(const float*, T*, int64_t, cudaStream_t);
+ECMOE_INST(float)
+ECMOE_INST(bf16)
+
+}  // namespace ecmoe

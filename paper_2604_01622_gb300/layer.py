@@ -1,0 +1,97 @@
+"""Torch-facing wrapper of one EC-MoE layer context (argument marshalling only).
+
+PyTorch supplies device memory and the current stream; every step of the layer runs in
+libecmoe.so. Tensor layouts are those of include/ecmoe.h.
+"""
+from __future__ import annotations
+
+import torch
+
+from . import (EC_BF16, EC_F32, ec_check_device, ec_ctx_create, ec_ctx_destroy,
+               ec_ctx_set_capacity, ec_ctx_set_workspace, ec_moe_backward, ec_moe_forward,
+               ec_route, ec_rows_per_expert, ec_workspace_bytes)
+
+_DT = {"f32": (EC_F32, torch.float32), "bf16": (EC_BF16, torch.bfloat16)}
+
+
+def _p(t):
+    return None if t is None else t.data_ptr()
+
+
+def _stream(stream):
+    return (stream or torch.cuda.current_stream()).cuda_stream
+
+
+class ECMoELayer:
+    """One layer shape: N tokens in groups `group_off`, E experts, capacities k_g."""
+
+    def __init__(self, N, d, E, d_ff, group_off, k_g, dtype="bf16", device="cuda"):
+        self.N, self.d, self.E, self.d_ff = int(N), int(d), int(E), int(d_ff)
+        self.G = len(group_off) - 1
+        self.code, self.tdtype = _DT[dtype]
+        self.device = torch.device(device)
+        self.ctx = ec_ctx_create(self.N, self.d, self.E, self.d_ff, self.G, group_off, k_g,
+                                 self.code)
+        self.ws_bytes = ec_workspace_bytes(self.ctx)
+        self.ws = torch.empty(self.ws_bytes, dtype=torch.uint8, device=self.device)
+        ec_ctx_set_workspace(self.ctx, self.ws.data_ptr(), self.ws_bytes)
+
+    @property
+    def M(self) -> int:
+        return ec_rows_per_expert(self.ctx)
+
+    def set_capacity(self, k_g):
+        ec_ctx_set_capacity(self.ctx, k_g)
+
+    def _empty(self, *shape, dtype=None):
+        return torch.empty(*shape, dtype=dtype or self.tdtype, device=self.device)
+
+    def route(self, X=None, Wr=None, br=None, S_in=None, stream=None):
+        """Selection only. Returns (idx [E][M] int32, gate [E][M] f32, S [E][N] f32)."""
+        idx = self._empty(self.E, self.M, dtype=torch.int32)
+        gate = self._empty(self.E, self.M, dtype=torch.float32)
+        S = self._empty(self.E, self.N, dtype=torch.float32)
+        ec_route(self.ctx, _p(X), _p(Wr), _p(br), _p(S_in), _p(S), _p(idx), _p(gate),
+                 _stream(stream))
+        return idx, gate, S
+
+    def forward(self, X, Wr, br, Wg, Wu, Wd, Y=None, stream=None, outputs=True):
+        """Y = EC-MoE(X). Returns (Y, idx, gate, S) (idx/gate/S None if outputs=False)."""
+        Y = self._empty(self.N, self.d) if Y is None else Y
+        idx = gate = S = None
+        if outputs:
+            idx = self._empty(self.E, self.M, dtype=torch.int32)
+            gate = self._empty(self.E, self.M, dtype=torch.float32)
+            S = self._empty(self.E, self.N, dtype=torch.float32)
+        ec_moe_forward(self.ctx, _p(X), _p(Wr), _p(br), _p(Wg), _p(Wu), _p(Wd), _p(Y),
+                       _p(idx), _p(gate), _p(S), _stream(stream))
+        return Y, idx, gate, S
+
+    def backward(self, dY, grads=None, stream=None, with_bias=False):
+        """Gradients of <dY, Y> for the last forward. Returns a dict of tensors."""
+        g = grads or {
+            "dX": self._empty(self.N, self.d),
+            "dWr": self._empty(self.d, self.E, dtype=torch.float32),
+            "dbr": self._empty(self.E, dtype=torch.float32) if with_bias else None,
+            "dWg": self._empty(self.E, self.d, self.d_ff, dtype=torch.float32),
+            "dWu": self._empty(self.E, self.d, self.d_ff, dtype=torch.float32),
+            "dWd": self._empty(self.E, self.d_ff, self.d, dtype=torch.float32),
+        }
+        ec_moe_backward(self.ctx, _p(dY), _p(g["dX"]), _p(g["dWr"]), _p(g.get("dbr")),
+                        _p(g["dWg"]), _p(g["dWu"]), _p(g["dWd"]), _stream(stream))
+        return g
+
+    def check(self, stream=None):
+        """Synchronise and raise if a kernel reported a device-side timeout."""
+        ec_check_device(self.ctx, _stream(stream))
+
+    def close(self):
+        if self.ctx is not None:
+            ec_ctx_destroy(self.ctx)
+            self.ctx = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass

@@ -1,0 +1,80 @@
+"""The C ABI library loads on a machine without a GPU and exports every declared entry
+point; host-side argument checks work without touching the device."""
+import ctypes
+import os
+import re
+
+import pytest
+
+import paper_2604_01622_gb300 as ec
+from paper_2604_01622_gb300 import build as B
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    if not os.path.exists(ec.LIB_PATH):
+        B.build()
+    return ec.load()
+
+
+def _declared():
+    names = set()
+    for f in os.listdir(os.path.join(ROOT, "include")):
+        if f.endswith(".h"):
+            src = open(os.path.join(ROOT, "include", f)).read()
+            src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+            names |= set(re.findall(r"^\s*(?:[\w\s\*]+?)\b(ec_\w+)\s*\(", src, flags=re.M))
+    return names
+
+
+def test_header_declares_the_boundary():
+    names = _declared()
+    for n in ("ec_route", "ec_moe_forward", "ec_moe_backward", "ec_ctx_create"):
+        assert n in names
+    assert names == set(ec.EXPORTS)
+
+
+def test_library_exports_every_declared_symbol(lib):
+    handle = ctypes.CDLL(ec.LIB_PATH)
+    for name in _declared():
+        assert hasattr(handle, name), name
+
+
+def test_status_strings(lib):
+    assert ec.status_string(ec.EC_OK) == "EC_OK"
+    assert ec.status_string(ec.EC_ERR_TIMEOUT) == "EC_ERR_TIMEOUT"
+
+
+def test_host_validation_without_device(lib):
+    # k_g larger than its group
+    with pytest.raises(ec.ECError) as e:
+        ec.ec_ctx_create(256, 64, 8, 128, 2, [0, 128, 256], [16, 129], ec.EC_F32)
+    assert e.value.status == ec.EC_ERR_SHAPE
+    # group offsets not covering N
+    with pytest.raises(ec.ECError):
+        ec.ec_ctx_create(256, 64, 8, 128, 2, [0, 128, 255], [16, 16], ec.EC_F32)
+    # bf16 path needs d, d_ff multiples of 64
+    with pytest.raises(ec.ECError) as e:
+        ec.ec_ctx_create(256, 96, 8, 128, 2, [0, 128, 256], [16, 16], ec.EC_BF16)
+    assert e.value.status == ec.EC_ERR_UNSUPPORTED
+    ctx = ec.ec_ctx_create(256, 64, 8, 128, 2, [0, 128, 256], [16, 16], ec.EC_F32)
+    try:
+        assert ec.ec_rows_per_expert(ctx) == 32
+        assert ec.ec_workspace_bytes(ctx) > 0
+        # capacities may change per step but not exceed the workspace's
+        ec.ec_ctx_set_capacity(ctx, [0, 20])
+        assert ec.ec_rows_per_expert(ctx) == 20
+        with pytest.raises(ec.ECError) as e:
+            ec.ec_ctx_set_capacity(ctx, [20, 20])
+        assert e.value.status == ec.EC_ERR_SHAPE
+        # compute calls without a workspace are refused before any launch
+        with pytest.raises(ec.ECError) as e:
+            ec.ec_route(ctx, 16, 16, None, None, None, 16, 16, None)
+        assert e.value.status == ec.EC_ERR_WORKSPACE
+        with pytest.raises(ec.ECError) as e:
+            ec.ec_ctx_set_workspace(ctx, 0x1001, 1 << 40)
+        assert e.value.status == ec.EC_ERR_WORKSPACE
+    finally:
+        ec.ec_ctx_destroy(ctx)

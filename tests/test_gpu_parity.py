@@ -1,0 +1,154 @@
+"""CUDA path vs the float64 oracle, through the C ABI.
+
+Rules: the selection is compared bit-exactly when both sides rank the same score tensor
+(the GPU's fp32 scores); the layer outputs and gradients are then compared with the
+oracle run on that selection: relative max-norm 1e-4 on the fp32 path, 2e-2 on bf16.
+"""
+import numpy as np
+import pytest
+import torch
+
+from oracle import ecmoe as O
+from paper_2604_01622_gb300 import inputs as I
+from tests._util import dev, gpu_layer, host, relmax, tol
+
+pytestmark = pytest.mark.gpu
+
+GRADS = [("Y", "Y"), ("dX", "dX"), ("dWr", "dWr"), ("dWg", "dWg"), ("dWu", "dWu"), ("dWd", "dWd")]
+
+
+def _oracle_full(inp, layer, idx):
+    L = inp.layers[layer]
+    fwd = O.forward(inp.X.f64(), L.Wr.f64(), L.br, L.Wg.f64(), L.Wu.f64(), L.Wd.f64(),
+                    inp.group_off, inp.k_g, forced_idx=idx)
+    bwd = O.backward(fwd, inp.dY.f64(), L.Wr.f64(), L.Wg.f64(), L.Wu.f64(), L.Wd.f64())
+    return fwd, bwd
+
+
+def _check_layer(inp, layer=0):
+    w = inp.w
+    lay, out = gpu_layer(inp, layer)
+    S_gpu = host(out["S"]).T                              # [N][E] fp32 values as float64
+    idx_gpu = out["idx"].cpu().numpy()
+    # selection: bit-exact on the GPU's own scores
+    idx_ref, gate_ref = O.ec_select(S_gpu, inp.group_off, inp.k_g)
+    assert np.array_equal(idx_gpu, idx_ref)
+    assert np.array_equal(host(out["gate"]), gate_ref)
+    fwd, bwd = _oracle_full(inp, layer, idx_gpu)
+    ref = {"Y": fwd["Y"], **bwd}
+    errs = {k: relmax(host(out[k]), ref[r]) for k, r in GRADS}
+    if inp.layers[layer].br is not None:
+        errs["dbr"] = relmax(host(out["dbr"]), ref["dbr"])
+    errs["S"] = relmax(S_gpu, fwd["S"])
+    bound = tol(w)
+    assert all(v <= bound for v in errs.values()), errs
+    # tokens no expert chose: exactly zero output and input gradient
+    picked = np.zeros(w.N, bool)
+    picked[idx_gpu.ravel()] = True
+    assert np.all(host(out["Y"])[~picked] == 0.0)
+    assert np.all(host(out["dX"])[~picked] == 0.0)
+    return errs
+
+
+# ------------------------------------------------------------------ selection on given scores
+@pytest.mark.parametrize("quant", [None, 8.0, 2.0])
+def test_selection_bit_exact_on_given_scores(quant):
+    from paper_2604_01622_gb300.layer import ECMoELayer
+    rng = np.random.default_rng(7)
+    N, E = 3000, 12
+    for trial in range(3):
+        S = rng.random((N, E)).astype(np.float32)
+        if quant is not None:
+            S = (np.round(S * quant) / quant).astype(np.float32)
+        S[rng.random((N, E)) < 0.03] = np.float32(-0.0)
+        S[rng.random((N, E)) < 0.03] = np.float32(0.0)
+        S[rng.random((N, E)) < 0.02] *= -1
+        group_off = I.random_groups(rng, N, 5)
+        sizes = np.diff(group_off)
+        k_g = np.array([rng.integers(0, s + 1) for s in sizes], dtype=np.int32)
+        k_g[0] = 0
+        k_g[-1] = sizes[-1]                                 # k = L edge
+        lay = ECMoELayer(N, 64, E, 64, group_off, k_g, dtype="f32")
+        ST = torch.from_numpy(np.ascontiguousarray(S.T)).cuda()
+        idx, gate, S_out = lay.route(S_in=ST)
+        lay.check()
+        ref_idx, ref_gate = O.ec_select(S.astype(np.float64), group_off, k_g)
+        assert np.array_equal(idx.cpu().numpy(), ref_idx)
+        assert np.array_equal(gate.cpu().numpy().astype(np.float64), ref_gate)
+        assert np.array_equal(S_out.cpu().numpy(), S.T)
+
+
+def test_selection_long_groups_beyond_shared_memory():
+    """Groups longer than the shared-memory key buffer take the global-memory path."""
+    from paper_2604_01622_gb300.layer import ECMoELayer
+    rng = np.random.default_rng(8)
+    N, E = 60000, 3
+    S = (np.round(rng.random((N, E)) * 64) / 64).astype(np.float32)
+    group_off = np.array([0, 55000, N], np.int32)
+    k_g = np.array([7001, 300], np.int32)
+    lay = ECMoELayer(N, 64, E, 64, group_off, k_g, dtype="f32")
+    idx, gate, _ = lay.route(S_in=torch.from_numpy(np.ascontiguousarray(S.T)).cuda())
+    lay.check()
+    ref_idx, _ = O.ec_select(S.astype(np.float64), group_off, k_g)
+    assert np.array_equal(idx.cpu().numpy(), ref_idx)
+
+
+# ------------------------------------------------------------------ fp32 path (1e-4)
+def test_tiny_f32_layer_matches_oracle():
+    _check_layer(I.make_inputs(I.WORKLOADS["tiny_f32"]))
+
+
+@pytest.mark.parametrize("seed", [11, 12])
+def test_f32_ragged_groups_and_capacity_edges(seed):
+    # N = 333 tokens, d = 68, d_ff = 36: no size is a multiple of a tile
+    w = I.scaled(I.WORKLOADS["tiny_f32"], G=1, L=333, d=68, E=11, d_ff=36, seed=seed,
+                 router_bias=True)
+    inp = I.make_inputs(w)
+    inp.group_off = np.array([0, 0, 150, 151, 333], np.int32)   # an empty and a 1-token group
+    inp.k_g = np.array([0, 150, 1, 17], np.int32)                # k = 0 and k = L
+    _check_layer(inp)
+
+
+# ------------------------------------------------------------------ bf16 path (2e-2), small shapes
+SMALL_BF16 = {
+    # d2048/e64-like: ragged M (2*80 = 160 rows: one full 128-row tile and a 32-row tail)
+    "ec_d2048_e64": dict(G=2, L=512, d=256, E=8, d_ff=128, k_base=80),
+    # timestep capacity with mask-vector ties
+    "ec_timestep_d2048_e64": dict(G=4, L=256, d=192, E=8, d_ff=192, k_base=48),
+    # many experts with router bias
+    "ec_many_small_e128": dict(G=4, L=256, d=128, E=128, d_ff=64, k_base=16),
+    # wide, few experts
+    "ec_wide_d4096_e32_x4": dict(G=2, L=1024, d=512, E=32, d_ff=256, k_base=64, layers=1),
+}
+
+
+@pytest.mark.parametrize("name", sorted(SMALL_BF16))
+def test_bf16_small_layers_match_oracle(name):
+    w = I.scaled(I.WORKLOADS[name], **SMALL_BF16[name])
+    _check_layer(I.make_inputs(w))
+
+
+def test_bf16_is_deterministic():
+    w = I.scaled(I.WORKLOADS["ec_d2048_e64"], **SMALL_BF16["ec_d2048_e64"])
+    inp = I.make_inputs(w)
+    _, a = gpu_layer(inp)
+    _, b = gpu_layer(inp)
+    for k in ("Y", "idx", "gate", "dX", "dWr", "dWg", "dWu", "dWd"):
+        assert torch.equal(a[k], b[k]), k
+
+
+def test_set_capacity_matches_fresh_context():
+    from paper_2604_01622_gb300.layer import ECMoELayer
+    w = I.scaled(I.WORKLOADS["ec_timestep_d2048_e64"], **SMALL_BF16["ec_timestep_d2048_e64"])
+    inp = I.make_inputs(w)
+    L = inp.layers[0]
+    args = (dev(inp.X), dev(L.Wr), None, dev(L.Wg), dev(L.Wu), dev(L.Wd))
+    lay = ECMoELayer(w.N, w.d, w.E, w.d_ff, inp.group_off, inp.k_g, dtype="bf16")
+    k2 = np.array([60, 10, 0, 100], np.int32)          # same total, new split
+    lay.set_capacity(k2)
+    Y1, idx1, _, _ = lay.forward(*args)
+    fresh = ECMoELayer(w.N, w.d, w.E, w.d_ff, inp.group_off, k2, dtype="bf16")
+    Y2, idx2, _, _ = fresh.forward(*args)
+    lay.check()
+    fresh.check()
+    assert torch.equal(idx1, idx2) and torch.equal(Y1, Y2)
