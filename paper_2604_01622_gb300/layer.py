@@ -65,6 +65,8 @@ class ECMoELayer:
             S = self._empty(self.E, self.N, dtype=torch.float32)
         ec_moe_forward(self.ctx, _p(X), _p(Wr), _p(br), _p(Wg), _p(Wu), _p(Wd), _p(Y),
                        _p(idx), _p(gate), _p(S), _stream(stream))
+        # the backward pass reads these through the pointers the context remembered
+        self._keep = (X, Wr, br, Wg, Wu, Wd)
         return Y, idx, gate, S
 
     def backward(self, dY, grads=None, stream=None, with_bias=False):
