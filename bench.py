@@ -1,0 +1,405 @@
+#!/usr/bin/env python3
+"""EC-MoE layer forward + backward throughput on GB300 (tokens/s).
+
+Default workload: 8 sequences x 4096 tokens (N = 32768), d_model 2048, 64 SwiGLU experts
+of d_ff 1024, capacity k_g = 512 per expert per sequence (top-8 equivalent), bf16 with
+fp32 accumulation, seeded synthetic inputs. One step = ec_moe_forward + ec_moe_backward
+through the C ABI on inputs resident in HBM. Inputs and saved activations (GBs) are far
+larger than the 129 MB L2, so no explicit flush is done between steps.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+With N > 1 (torchrun) every rank runs its own replica of the workload on its own GPU
+(the layer needs no exchange in the forward pass and this benchmark does not all-reduce
+weight gradients); value = tokens of all ranks / max over ranks of the step time.
+`--impl reference` times the float64 CPU oracle on the host cores instead.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "EC-MoE layer fwd+bwd tokens/sec on 1 GB300; expert-GEMM % BF16 peak; routing HBM GB/s"
+UNIT = "tokens/s"
+
+# DRAM traffic per launch of the grouped-GEMM kernels, from one ncu capture of this
+# workload (dram__bytes_read.sum + dram__bytes_write.sum), keyed by the hash of the
+# kernel source it was taken on; a changed kernel reports null until re-captured.
+TRAFFIC = {}
+
+
+def _peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return d["hbm_gbs"], d["bf16_tflops"], d["bf16_tflops_sustained"], "measured"
+    return 6800.0, 1900.0, 1700.0, "fallback"
+
+
+def _src_hash(path):
+    return hashlib.sha1(open(path, "rb").read()).hexdigest()[:12]
+
+
+def _cores():
+    for v in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS"):
+        if os.environ.get(v, "").isdigit():
+            return int(os.environ[v])
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count()
+
+
+# ------------------------------------------------------------------ clocks
+class Clocks:
+    """nvidia-smi sampler running during the timed region."""
+    Q = ("timestamp,clocks.sm,clocks.max.sm,power.draw,utilization.gpu,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+        self.f = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+
+    def start(self):
+        self.t_begin = None
+        self.t_end = None
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.Q}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=self.f, stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+
+    def mark_begin(self):
+        self.t_begin = time.time()
+
+    def mark_end(self):
+        self.t_end = time.time()
+
+    def stop(self):
+        import datetime
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        time.sleep(0.25)
+        self.proc.terminate()
+        self.proc.wait()
+        self.f.flush()
+        rows = [r.split(",") for r in open(self.f.name).read().strip().splitlines() if r]
+        os.unlink(self.f.name)
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        sm, smax, reasons, load = [], [], set(), []
+        for r in rows:
+            r = [x.strip() for x in r]
+            if len(r) < 10:
+                continue
+            try:
+                ts = datetime.datetime.strptime(r[0], "%Y/%m/%d %H:%M:%S.%f").timestamp()
+                if self.t_begin and self.t_end and not (self.t_begin - 0.05 <= ts <= self.t_end + 0.05):
+                    continue
+                sm.append(float(r[1]))
+                smax.append(float(r[2]))
+                load.append(float(r[4]))
+            except ValueError:
+                continue
+            for n, v in zip(names, r[6:10]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        busy = [s for s, u in zip(sm, load) if u >= 50] or sm
+        busy.sort()
+        return {"sm_mhz": busy[len(busy) // 2] if busy else None,
+                "sm_max_mhz": max(smax) if smax else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ------------------------------------------------------------------ CPU oracle sample
+class OracleSample:
+    """A bounded sample of the workload for the float64 oracle (as it stands): whole
+    sequences of the workload when `tokens` >= its sequence length, else one shorter
+    sequence with the capacity scaled to keep the workload's capacity factor."""
+
+    def __init__(self, tokens: int, w):
+        from paper_2604_01622_gb300 import inputs as I
+        if tokens >= w.L:
+            G, L, k = max(1, tokens // w.L), w.L, w.k_base
+        else:
+            G, L, k = 1, tokens, max(1, w.k_base * tokens // w.L)
+        self.tokens = G * L
+        ws = I.scaled(w, G=G, L=L, k_base=k, timestep_capacity=False, layers=1)
+        inp = I.make_inputs(ws)
+        Ld = inp.layers[0]
+        self.args = (inp.X.f64(), Ld.Wr.f64(), Ld.br, Ld.Wg.f64(), Ld.Wu.f64(), Ld.Wd.f64(),
+                     inp.group_off, inp.k_g)
+        self.dY = inp.dY.f64()
+        self.desc = (f"{G} sequence(s) x {L} tokens of the workload (k_g={k}, capacity factor "
+                     f"{w.E * k / L:g}, E={w.E}, d={w.d}, d_ff={w.d_ff}), oracle fwd+bwd")
+
+    def run(self):
+        """Returns (tokens/s, seconds)."""
+        from oracle import ecmoe as O
+        X, Wr, br, Wg, Wu, Wd, goff, kg = self.args
+        t0 = time.perf_counter()
+        f = O.forward(X, Wr, br, Wg, Wu, Wd, goff, kg)
+        O.backward(f, self.dY, Wr, Wg, Wu, Wd)
+        dt = time.perf_counter() - t0
+        return self.tokens / dt, dt
+
+
+# ------------------------------------------------------------------ distributed
+def _dist():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def _max_over_ranks(x: float, ws: int, device) -> float:
+    if ws == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def _barrier(ws):
+    if ws > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+# ------------------------------------------------------------------ our arm
+def run_ours(args):
+    import numpy as np
+    import torch
+    ws, rank, local = _dist()
+    if ws > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", init_method="env://")
+    torch.cuda.set_device(local)
+    device = torch.device("cuda", local)
+
+    from paper_2604_01622_gb300 import build as B
+    if rank == 0 or ws == 1:
+        B.build()
+    _barrier(ws)
+    from paper_2604_01622_gb300 import inputs as I
+    from paper_2604_01622_gb300.layer import ECMoELayer
+    w = I.WORKLOADS[args.workload]
+    if args.seqs:
+        w = I.scaled(w, G=args.seqs)
+    inp = I.make_inputs(w)
+    Ld = inp.layers[0]
+
+    def to_dev(t):
+        if t.dtype == "bf16":
+            return torch.from_numpy(t.data.view(np.int16)).to(device).view(torch.bfloat16)
+        return torch.from_numpy(t.data).to(device)
+
+    X, dY = to_dev(inp.X), to_dev(inp.dY)
+    Wr, Wg, Wu, Wd = to_dev(Ld.Wr), to_dev(Ld.Wg), to_dev(Ld.Wu), to_dev(Ld.Wd)
+    br = None if Ld.br is None else torch.from_numpy(Ld.br).to(device)
+    lay = ECMoELayer(w.N, w.d, w.E, w.d_ff, inp.group_off, inp.k_g, dtype=w.dtype, device=device)
+    Y = torch.empty_like(X)
+    grads = {"dX": torch.empty_like(X),
+             "dWr": torch.empty(w.d, w.E, dtype=torch.float32, device=device),
+             "dbr": None if br is None else torch.empty(w.E, dtype=torch.float32, device=device),
+             "dWg": torch.empty(w.E, w.d, w.d_ff, dtype=torch.float32, device=device),
+             "dWu": torch.empty(w.E, w.d, w.d_ff, dtype=torch.float32, device=device),
+             "dWd": torch.empty(w.E, w.d_ff, w.d, dtype=torch.float32, device=device)}
+    stream = torch.cuda.current_stream(device)
+
+    def step(x=X, dy=dY, y=Y, g=grads):
+        lay.forward(x, Wr, br, Wg, Wu, Wd, Y=y, outputs=False)
+        lay.backward(dy, grads=g)
+
+    for _ in range(args.warmup):
+        step()
+    lay.check()
+
+    # ---- device-timed steps (inputs resident), per-kernel events on the same stream
+    lay.set_profiling(True)
+    launches0 = lay.launches
+    clocks = Clocks(local)
+    clocks.start()
+    time.sleep(0.5)       # let the sampler come up before the timed region
+    _barrier(ws)
+    torch.cuda.synchronize(device)
+    clocks.mark_begin()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        step()
+    e1.record(stream)
+    torch.cuda.synchronize(device)
+    clocks.mark_end()
+    _barrier(ws)
+    clk = clocks.stop()
+    launches = lay.launches - launches0
+    phases = lay.profile()
+    lay.set_profiling(False)
+    lay.check()
+    ms = e0.elapsed_time(e1) / args.steps
+    ms_max = _max_over_ranks(ms, ws, device)
+
+    # ---- end to end: host inputs copied in, results copied out, every step
+    hX = torch.empty(X.shape, dtype=X.dtype, pin_memory=True)
+    hdY = torch.empty(dY.shape, dtype=dY.dtype, pin_memory=True)
+    hX.copy_(X)
+    hdY.copy_(dY)
+    hY = torch.empty(Y.shape, dtype=Y.dtype, pin_memory=True)
+    hdX = torch.empty(X.shape, dtype=X.dtype, pin_memory=True)
+    Xe, dYe = torch.empty_like(X), torch.empty_like(dY)
+    e_steps = max(3, args.steps // 2)
+    _barrier(ws)
+    torch.cuda.synchronize(device)
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record(stream)
+    for _ in range(e_steps):
+        Xe.copy_(hX, non_blocking=True)
+        dYe.copy_(hdY, non_blocking=True)
+        step(x=Xe, dy=dYe)
+        hY.copy_(Y, non_blocking=True)
+        hdX.copy_(grads["dX"], non_blocking=True)
+    t1.record(stream)
+    torch.cuda.synchronize(device)
+    e2e_ms = _max_over_ranks(t0.elapsed_time(t1) / e_steps, ws, device)
+    lay.check()
+
+    # ---- roofline of the dominant kernel (the tcgen05 grouped GEMM)
+    hbm, bf16_burst, bf16_sust, peak_src = _peaks()
+    per = {}
+    for name, t in phases:
+        per.setdefault(name, []).append(t)
+    gemm = {k: v for k, v in per.items() if k.startswith("gemm_")}
+    gemm_launches = sum(len(v) for v in gemm.values()) + len(per.get("gemm_wgrad", []))
+    gemm_ms_step = sum(sum(v) for v in gemm.values()) / args.steps
+    P = w.E * int(inp.k_g.sum())
+    flops_step = 18.0 * P * w.d * w.d_ff
+    gemm_tflops = flops_step / (gemm_ms_step * 1e-3) / 1e12
+    gemm_per_launch = flops_step / max(1, gemm_launches / args.steps)
+    b = 2 if w.dtype == "bf16" else 4
+    N, d, E = w.N, w.d, w.E
+    mem_bytes = {
+        "router_gemm_softmax": N * d * b + 2 * N * E * 4,
+        "topk": 2 * N * E * 4 + 2 * P * 4,
+        "gather": 2 * P * d * b,
+        "combine": P * d * b + N * d * b,
+        "bwd_gather_scale": 3 * P * d * b,
+        "softmax_bwd": 3 * N * E * 4,
+        "dx_combine": P * d * b + N * d * 4 + N * d * b,
+    }
+    mem_ms = sum(sum(per.get(k, [])) for k in mem_bytes) / args.steps
+    mem_gbs = sum(mem_bytes.values()) / (mem_ms * 1e-3) / 1e9 if mem_ms > 0 else None
+    src = os.path.join(ROOT, "paper_2604_01622_gb300", "csrc", "gemm_tc.cu")
+    tr = TRAFFIC.get(_src_hash(src))
+    roofline = {
+        "kernel": "tc_gemm_kernel (tcgen05 grouped expert GEMMs: gate/up, down, dU, dH, dW)",
+        "bound": "tensor", "achieved": round(gemm_tflops, 1),
+        "peak": bf16_sust, "unit": "TFLOP/s", "frac": round(gemm_tflops / bf16_sust, 4),
+        "peak_kind": f"bf16 sustained, {peak_src}",
+        "frac_of_burst": round(gemm_tflops / bf16_burst, 4),
+        "flops_per_launch": gemm_per_launch,
+        "traffic": tr,
+    }
+    out = {
+        "metric": METRIC, "value": None, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": round(ms_max, 4), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
+        "config": {"workload": w.name, "sequences": w.G, "seq_len": w.L, "tokens": w.N,
+                   "d_model": w.d, "experts": w.E, "d_ff": w.d_ff, "k_per_seq": w.k_base,
+                   "parallelism": f"replicas{ws}" if ws > 1 else "single",
+                   "l2": "inputs and activations larger than L2 (no flush)"},
+    }
+    out["value"] = round(ws * w.N / (ms_max * 1e-3), 1)
+    out["expert_gemm_pct_bf16_peak"] = round(100 * gemm_tflops / bf16_burst, 2)
+    out["routing_hbm_gbs"] = None if mem_gbs is None else round(mem_gbs, 1)
+    out["routing_hbm_frac"] = None if mem_gbs is None else round(mem_gbs / hbm, 4)
+    out["e2e"] = {"value": round(ws * w.N / (e2e_ms * 1e-3), 1), "unit": UNIT,
+                  "h2d_bytes_per_step": int(X.numel() * X.element_size() * 2),
+                  "d2h_bytes_per_step": int(X.numel() * X.element_size() * 2)}
+    out["roofline"] = roofline
+    out["gpu_launches"] = int(launches)
+    out["kernel_ms_per_step"] = {k: round(sum(v) / args.steps, 4) for k, v in per.items()}
+    out["clocks"] = clk
+    if rank == 0 and not args.no_cpu_baseline:
+        smp = OracleSample(args.cpu_tokens, w)
+        v, dt = smp.run()
+        out["cpu_baseline"] = {"value": round(v, 2), "unit": UNIT, "cores": _cores(),
+                               "kind": "oracle", "sample": smp.desc, "seconds": round(dt, 2)}
+    if rank == 0:
+        print(json.dumps(out), flush=True)
+    if ws > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+# ------------------------------------------------------------------ reference arm (oracle)
+def run_reference(args):
+    ws, rank, local = _dist()
+    if rank != 0:
+        return
+    from paper_2604_01622_gb300 import inputs as I
+    w = I.WORKLOADS[args.workload]
+    smp = OracleSample(args.ref_tokens, w)
+    for _ in range(args.warmup):
+        smp.run()
+    total_t = 0.0
+    for _ in range(args.steps):
+        total_t += smp.run()[1]
+    desc = smp.desc
+    v = args.steps * smp.tokens / total_t
+    out = {"impl": "reference", "metric": METRIC, "value": round(v, 2), "unit": UNIT,
+           "n_gpus": 1, "steps": args.steps, "warmup": args.warmup,
+           "ms_per_step": round(1e3 * total_t / args.steps, 2), "higher_is_better": True,
+           "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+           "config": {"workload": w.name, "sequences": w.G, "seq_len": w.L, "tokens": w.N,
+                      "d_model": w.d, "experts": w.E, "d_ff": w.d_ff, "k_per_seq": w.k_base,
+                      "parallelism": "host cores"},
+           "cpu_baseline": {"value": round(v, 2), "unit": UNIT, "cores": _cores(),
+                            "kind": "oracle", "sample": desc + " per step"},
+           "e2e": {"value": round(v, 2), "unit": UNIT, "h2d_bytes_per_step": 0,
+                   "d2h_bytes_per_step": 0}}
+    print(json.dumps(out), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="ec_d2048_e64")
+    ap.add_argument("--seqs", type=int, default=0,
+                    help="run only this many sequences of the workload (small profiling cases)")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-tokens", type=int, default=8192,
+                    help="tokens of the oracle's CPU baseline sample")
+    ap.add_argument("--ref-tokens", type=int, default=128,
+                    help="tokens per step of the reference (oracle) arm")
+    args = ap.parse_args()
+    if args.warmup < 3 and args.impl == "ours":
+        ap.error("--warmup must be at least 3")
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

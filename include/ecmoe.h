@@ -119,6 +119,19 @@ ec_status ec_moe_backward(ec_ctx* ctx, const void* dY, void* dX, float* dWr, flo
  * kernel gave up on a bounded wait since the last check, EC_ERR_CUDA on a CUDA error. */
 ec_status ec_check_device(ec_ctx* ctx, void* stream);
 
+/* Per-kernel timing. With profiling on, every kernel launch of the following calls is
+ * bracketed by CUDA events recorded on the call's stream (one event record per kernel;
+ * off by default). Phases accumulate over calls; ec_ctx_set_profiling clears them. */
+ec_status ec_ctx_set_profiling(ec_ctx* ctx, int32_t on);
+
+/* Phases recorded since profiling was last switched: up to `cap` kernel names (static
+ * strings) and durations in ms, in launch order. Waits for the last recorded event.
+ * Returns the number of phases (which may exceed cap), 0 if none, -1 on a CUDA error. */
+int32_t ec_ctx_profile(ec_ctx* ctx, const char** names, float* ms, int32_t cap);
+
+/* Number of CUDA kernels the library has launched through this context so far. */
+int64_t ec_kernel_launches(const ec_ctx* ctx);
+
 /* Message of the last failed call on this context ("" if none). Owned by the context. */
 const char* ec_last_error(const ec_ctx* ctx);
 

@@ -25,6 +25,7 @@ EXPORTS = (
     "ec_ctx_create", "ec_ctx_destroy", "ec_ctx_set_capacity", "ec_rows_per_expert",
     "ec_workspace_bytes", "ec_ctx_set_workspace", "ec_route", "ec_moe_forward",
     "ec_moe_backward", "ec_check_device", "ec_last_error", "ec_status_string",
+    "ec_ctx_set_profiling", "ec_ctx_profile", "ec_kernel_launches",
 )
 
 _lib = None
@@ -60,6 +61,10 @@ def load():
         "ec_check_device": (i32, [vp, vp]),
         "ec_last_error": (ctypes.c_char_p, [vp]),
         "ec_status_string": (ctypes.c_char_p, [i32]),
+        "ec_ctx_set_profiling": (i32, [vp, i32]),
+        "ec_ctx_profile": (i32, [vp, ctypes.POINTER(ctypes.c_char_p),
+                                 ctypes.POINTER(ctypes.c_float), i32]),
+        "ec_kernel_launches": (i64, [vp]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -130,6 +135,24 @@ def ec_moe_backward(ctx, dY, dX, dWr, dbr, dWg, dWu, dWd, stream):
 
 def ec_check_device(ctx, stream):
     _check(ctx, load().ec_check_device(ctx, stream))
+
+
+def ec_ctx_set_profiling(ctx, on: bool):
+    _check(ctx, load().ec_ctx_set_profiling(ctx, 1 if on else 0))
+
+
+def ec_ctx_profile(ctx, cap: int = 4096):
+    """[(kernel name, ms), ...] of the phases recorded since profiling was switched on."""
+    names = (ctypes.c_char_p * cap)()
+    ms = (ctypes.c_float * cap)()
+    n = load().ec_ctx_profile(ctx, names, ms, cap)
+    if n < 0:
+        raise ECError(EC_ERR_CUDA, "ec_ctx_profile: CUDA error while reading events")
+    return [(names[i].decode(), float(ms[i])) for i in range(min(n, cap))]
+
+
+def ec_kernel_launches(ctx) -> int:
+    return int(load().ec_kernel_launches(ctx))
 
 
 def ec_last_error(ctx) -> str:

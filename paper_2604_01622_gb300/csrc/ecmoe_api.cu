@@ -24,6 +24,12 @@ struct ec_ctx {
   size_t o_status, o_goff, o_kg, o_koff, o_ST, o_S, o_idx, o_gate, o_slot, o_H, o_A, o_B, o_U,
       o_O, o_dO, o_dA, o_dB, o_dgate, o_dZ, o_wrpad, o_f32a, o_f32b, o_dXr, o_part, total;
   int wr_splits = 1;
+  // per-kernel event timing (off by default) and kernel launch counter
+  bool prof = false;
+  std::vector<cudaEvent_t> ev;
+  std::vector<const char*> ev_name;
+  int ev_n = 0;
+  int64_t launches = 0;
   // state saved by the forward pass
   bool have_fwd = false;
   const void *X = nullptr, *Wr = nullptr, *Wg = nullptr, *Wu = nullptr, *Wd = nullptr;
@@ -53,6 +59,29 @@ ec_status cuda_fail(ec_ctx* c, cudaError_t e, const char* where) {
   do {                                               \
     cudaError_t _e = (call);                         \
     if (_e != cudaSuccess) return cuda_fail(c, _e, where); \
+  } while (0)
+
+// Phase marker: with profiling on, records an event named after the kernel about to be
+// launched (or "end" after the last one) on the call's stream.
+void mark(ec_ctx* c, const char* name, cudaStream_t st) {
+  if (!c->prof) return;
+  if (c->ev_n == (int)c->ev.size()) {
+    cudaEvent_t e;
+    if (cudaEventCreate(&e) != cudaSuccess) return;
+    c->ev.push_back(e);
+    c->ev_name.push_back(nullptr);
+  }
+  cudaEventRecord(c->ev[c->ev_n], st);
+  c->ev_name[c->ev_n] = name;
+  ++c->ev_n;
+}
+
+// Launch `nk` kernels through `call` as one named phase.
+#define EC_KERNEL(name, nk, call)            \
+  do {                                       \
+    mark(c, name, st);                       \
+    c->launches += (nk);                     \
+    EC_CUDA(call, name);                     \
   } while (0)
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
@@ -179,21 +208,24 @@ ec_status run_route(ec_ctx* c, const void* X, const void* Wr, const float* br, c
   const int N = c->N, E = c->E, d = c->d;
   float* ST = at<float>(c, c->o_ST);
   float* S = at<float>(c, c->o_S);
+  const int nz = N > 0;
   if (S_in) {
     EC_CUDA(cudaMemcpyAsync(ST, S_in, (size_t)E * N * 4, cudaMemcpyDeviceToDevice, st), "copy S_in");
-    EC_CUDA(launch_transpose_scores(ST, S, N, E, st), "transpose scores");
+    EC_KERNEL("transpose_scores", nz, launch_transpose_scores(ST, S, N, E, st));
   } else if (use_tc(c)) {
-    EC_CUDA(tc_router_softmax(X, Wr, at<void>(c, c->o_wrpad), br, S, ST, N, d, E, at<int>(c, c->o_status), st), "router");
+    EC_KERNEL("router_gemm_softmax", 2 * nz,
+              tc_router_softmax(X, Wr, at<void>(c, c->o_wrpad), br, S, ST, N, d, E,
+                                at<int>(c, c->o_status), st));
   } else {
     float* Z = at<float>(c, c->o_f32a);
-    EC_CUDA(launch_simt_gemm(sg(X, 0, d, 1, Wr, 0, E, 1, Z, 0, E, N, E, d, 1), et(c), et(c), st),
-            "router gemm");
-    EC_CUDA(launch_softmax_rows(Z, br, S, ST, N, E, st), "router softmax");
+    EC_KERNEL("router_gemm", nz,
+              launch_simt_gemm(sg(X, 0, d, 1, Wr, 0, E, 1, Z, 0, E, N, E, d, 1), et(c), et(c), st));
+    EC_KERNEL("router_softmax", nz, launch_softmax_rows(Z, br, S, ST, N, E, st));
   }
-  EC_CUDA(launch_topk(ST, N, E, c->G, at<int>(c, c->o_goff), at<int>(c, c->o_kg),
-                      at<int>(c, c->o_koff), c->M, c->max_group, at<int>(c, c->o_idx),
-                      at<float>(c, c->o_gate), at<int>(c, c->o_slot), st),
-          "top-k");
+  EC_KERNEL("topk", 1,
+            launch_topk(ST, N, E, c->G, at<int>(c, c->o_goff), at<int>(c, c->o_kg),
+                        at<int>(c, c->o_koff), c->M, c->max_group, at<int>(c, c->o_idx),
+                        at<float>(c, c->o_gate), at<int>(c, c->o_slot), st));
   return EC_OK;
 }
 
@@ -216,34 +248,38 @@ ec_status run_forward(ec_ctx* c, const void* X, const void* Wg, const void* Wu, 
                       void* Y, cudaStream_t st) {
   const int N = c->N, d = c->d, E = c->E, F = c->F, M = c->M;
   const int64_t P = (int64_t)E * M;
+  const int pz = P > 0;
   T* H = at<T>(c, c->o_H);
   T* A = at<T>(c, c->o_A);
   T* B = at<T>(c, c->o_B);
   T* U = at<T>(c, c->o_U);
   T* O = at<T>(c, c->o_O);
+  int* status = at<int>(c, c->o_status);
   const int* idx = at<int>(c, c->o_idx);
-  EC_CUDA(launch_gather<T>(static_cast<const T*>(X), idx, H, P, d, st), "gather");
+  EC_KERNEL("gather", pz, launch_gather<T>(static_cast<const T*>(X), idx, H, P, d, st));
   if (P > 0) {
     if (use_tc(c)) {
-      EC_CUDA(tc_expert_up(H, Wg, Wu, A, B, U, E, M, d, F, at<int>(c, c->o_status), st), "gate/up gemm");
-      EC_CUDA(tc_expert_down(U, Wd, O, E, M, d, F, at<int>(c, c->o_status), st), "down gemm");
+      EC_KERNEL("gemm_gate_up_swiglu", 1, tc_expert_up(H, Wg, Wu, A, B, U, E, M, d, F, status, st));
+      EC_KERNEL("gemm_down", 1, tc_expert_down(U, Wd, O, E, M, d, F, status, st));
     } else {
       float* Ag = at<float>(c, c->o_f32a);
       float* Bu = at<float>(c, c->o_f32b);
       const int64_t hs = (int64_t)M * d, ws = (int64_t)d * F, os = (int64_t)M * F;
-      EC_CUDA(launch_simt_gemm(sg(H, hs, d, 1, Wg, ws, F, 1, Ag, os, F, M, F, d, E), et(c), et(c), st),
-              "gate gemm");
-      EC_CUDA(launch_simt_gemm(sg(H, hs, d, 1, Wu, ws, F, 1, Bu, os, F, M, F, d, E), et(c), et(c), st),
-              "up gemm");
-      EC_CUDA(launch_swiglu_fwd_ew<T>(Ag, Bu, A, B, U, P * F, st), "swiglu");
+      EC_KERNEL("gemm_gate", 1,
+                launch_simt_gemm(sg(H, hs, d, 1, Wg, ws, F, 1, Ag, os, F, M, F, d, E), et(c), et(c), st));
+      EC_KERNEL("gemm_up", 1,
+                launch_simt_gemm(sg(H, hs, d, 1, Wu, ws, F, 1, Bu, os, F, M, F, d, E), et(c), et(c), st));
+      EC_KERNEL("swiglu", 1, launch_swiglu_fwd_ew<T>(Ag, Bu, A, B, U, P * F, st));
       float* O32 = at<float>(c, c->o_f32a);
-      EC_CUDA(launch_simt_gemm(sg(U, os, F, 1, Wd, (int64_t)F * d, d, 1, O32, hs, d, M, d, F, E),
-                               et(c), et(c), st), "down gemm");
-      EC_CUDA(launch_convert<T>(O32, O, P * d, st), "convert O");
+      EC_KERNEL("gemm_down", 1,
+                launch_simt_gemm(sg(U, os, F, 1, Wd, (int64_t)F * d, d, 1, O32, hs, d, M, d, F, E),
+                                 et(c), et(c), st));
+      EC_KERNEL("convert_o", 1, launch_convert<T>(O32, O, P * d, st));
     }
   }
-  EC_CUDA(launch_combine<T>(O, at<float>(c, c->o_gate), at<int>(c, c->o_slot),
-                            static_cast<T*>(Y), N, E, M, d, st), "combine");
+  EC_KERNEL("combine", N > 0,
+            launch_combine<T>(O, at<float>(c, c->o_gate), at<int>(c, c->o_slot),
+                              static_cast<T*>(Y), N, E, M, d, st));
   return EC_OK;
 }
 
@@ -253,6 +289,7 @@ ec_status run_backward(ec_ctx* c, const void* dY, void* dX, float* dWr, float* d
                        float* dWu, float* dWd, cudaStream_t st) {
   const int N = c->N, d = c->d, E = c->E, F = c->F, M = c->M;
   const int64_t P = (int64_t)E * M;
+  const int pz = P > 0, nz = N > 0;
   T* H = at<T>(c, c->o_H);
   T* A = at<T>(c, c->o_A);
   T* B = at<T>(c, c->o_B);
@@ -264,41 +301,47 @@ ec_status run_backward(ec_ctx* c, const void* dY, void* dX, float* dWr, float* d
   T* dB = at<T>(c, c->o_dB);
   float* dgate = at<float>(c, c->o_dgate);
   float* dZ = at<float>(c, c->o_dZ);
+  int* status = at<int>(c, c->o_status);
   const int* idx = at<int>(c, c->o_idx);
   const float* gate = at<float>(c, c->o_gate);
   const int* slot = at<int>(c, c->o_slot);
   const int64_t hs = (int64_t)M * d, fs = (int64_t)M * F, wgs = (int64_t)d * F;
 
-  EC_CUDA(launch_bwd_gather_scale<T>(static_cast<const T*>(dY), O, idx, gate, dO, dgate, P, d, st),
-          "dO/dgate");
+  EC_KERNEL("bwd_gather_scale", pz,
+            launch_bwd_gather_scale<T>(static_cast<const T*>(dY), O, idx, gate, dO, dgate, P, d, st));
   if (P > 0) {
     if (use_tc(c)) {
-      EC_CUDA(tc_expert_dgrad_up(dO, c->Wd, A, B, dA, dB, E, M, d, F, at<int>(c, c->o_status), st),
-              "dU gemm");
-      EC_CUDA(tc_expert_dgrad_h(dA, dB, c->Wg, c->Wu, dH, E, M, d, F, at<int>(c, c->o_status), st),
-              "dH gemm");
-      EC_CUDA(tc_expert_wgrad(H, U, dO, dA, dB, dWg, dWu, dWd, E, M, d, F,
-                              at<int>(c, c->o_status), st), "weight-grad gemm");
+      EC_KERNEL("gemm_dgrad_up_swiglu", 1,
+                tc_expert_dgrad_up(dO, c->Wd, A, B, dA, dB, E, M, d, F, status, st));
+      EC_KERNEL("gemm_dgrad_h", 1, tc_expert_dgrad_h(dA, dB, c->Wg, c->Wu, dH, E, M, d, F, status, st));
+      EC_KERNEL("gemm_wgrad", 2,
+                tc_expert_wgrad(H, U, dO, dA, dB, dWg, dWu, dWd, E, M, d, F, status, st));
     } else {
       float* dU32 = at<float>(c, c->o_f32a);
       float* dH32 = at<float>(c, c->o_f32b);
       // dU = dO . Wd^T : B[k=i][n=j] = Wd[j][i]
-      EC_CUDA(launch_simt_gemm(sg(dO, hs, d, 1, c->Wd, (int64_t)F * d, 1, d, dU32, fs, F, M, F, d, E),
-                               et(c), et(c), st), "dU gemm");
-      EC_CUDA(launch_swiglu_bwd_ew<T>(dU32, A, B, dA, dB, P * F, st), "swiglu bwd");
+      EC_KERNEL("gemm_dgrad_u", 1,
+                launch_simt_gemm(sg(dO, hs, d, 1, c->Wd, (int64_t)F * d, 1, d, dU32, fs, F, M, F, d, E),
+                                 et(c), et(c), st));
+      EC_KERNEL("swiglu_bwd", 1, launch_swiglu_bwd_ew<T>(dU32, A, B, dA, dB, P * F, st));
       // dH = dA . Wg^T + dB . Wu^T
-      EC_CUDA(launch_simt_gemm(sg(dA, fs, F, 1, c->Wg, wgs, 1, F, dH32, hs, d, M, d, F, E),
-                               et(c), et(c), st), "dH gemm (gate)");
-      EC_CUDA(launch_simt_gemm(sg(dB, fs, F, 1, c->Wu, wgs, 1, F, dH32, hs, d, M, d, F, E, 1.f),
-                               et(c), et(c), st), "dH gemm (up)");
-      EC_CUDA(launch_convert<T>(dH32, dH, P * d, st), "convert dH");
+      EC_KERNEL("gemm_dgrad_h_gate", 1,
+                launch_simt_gemm(sg(dA, fs, F, 1, c->Wg, wgs, 1, F, dH32, hs, d, M, d, F, E),
+                                 et(c), et(c), st));
+      EC_KERNEL("gemm_dgrad_h_up", 1,
+                launch_simt_gemm(sg(dB, fs, F, 1, c->Wu, wgs, 1, F, dH32, hs, d, M, d, F, E, 1.f),
+                                 et(c), et(c), st));
+      EC_KERNEL("convert_dh", 1, launch_convert<T>(dH32, dH, P * d, st));
       // dWd = U^T dO ; dWg = H^T dA ; dWu = H^T dB   (A[m][k] = U[k][m])
-      EC_CUDA(launch_simt_gemm(sg(U, fs, 1, F, dO, hs, d, 1, dWd, (int64_t)F * d, d, F, d, M, E),
-                               et(c), et(c), st), "dWd gemm");
-      EC_CUDA(launch_simt_gemm(sg(H, hs, 1, d, dA, fs, F, 1, dWg, wgs, F, d, F, M, E),
-                               et(c), et(c), st), "dWg gemm");
-      EC_CUDA(launch_simt_gemm(sg(H, hs, 1, d, dB, fs, F, 1, dWu, wgs, F, d, F, M, E),
-                               et(c), et(c), st), "dWu gemm");
+      EC_KERNEL("gemm_wgrad_down", 1,
+                launch_simt_gemm(sg(U, fs, 1, F, dO, hs, d, 1, dWd, (int64_t)F * d, d, F, d, M, E),
+                                 et(c), et(c), st));
+      EC_KERNEL("gemm_wgrad_gate", 1,
+                launch_simt_gemm(sg(H, hs, 1, d, dA, fs, F, 1, dWg, wgs, F, d, F, M, E),
+                                 et(c), et(c), st));
+      EC_KERNEL("gemm_wgrad_up", 1,
+                launch_simt_gemm(sg(H, hs, 1, d, dB, fs, F, 1, dWu, wgs, F, d, F, M, E),
+                                 et(c), et(c), st));
     }
   } else {
     EC_CUDA(cudaMemsetAsync(dWg, 0, (size_t)E * d * F * 4, st), "zero dWg");
@@ -306,20 +349,21 @@ ec_status run_backward(ec_ctx* c, const void* dY, void* dX, float* dWr, float* d
     EC_CUDA(cudaMemsetAsync(dWd, 0, (size_t)E * d * F * 4, st), "zero dWd");
   }
   // router: dZ = S (dS - <dS,S>), dX = dZ Wr^T + sum dH, dWr = X^T dZ, dbr = sum dZ
-  EC_CUDA(launch_softmax_bwd(at<float>(c, c->o_S), slot, dgate, dZ, N, E, M, st), "softmax bwd");
+  EC_KERNEL("softmax_bwd", nz, launch_softmax_bwd(at<float>(c, c->o_S), slot, dgate, dZ, N, E, M, st));
   float* dXr = at<float>(c, c->o_dXr);
-  EC_CUDA(launch_simt_gemm(sg(dZ, 0, E, 1, c->Wr, 0, 1, E, dXr, 0, d, N, d, E, 1), EType::F32, et(c), st),
-          "dZ Wr^T");
-  EC_CUDA(launch_dx_combine<T>(dH, slot, dXr, static_cast<T*>(dX), N, E, M, d, st), "dX");
+  EC_KERNEL("router_dgrad_gemm", nz,
+            launch_simt_gemm(sg(dZ, 0, E, 1, c->Wr, 0, 1, E, dXr, 0, d, N, d, E, 1), EType::F32,
+                             et(c), st));
+  EC_KERNEL("dx_combine", nz, launch_dx_combine<T>(dH, slot, dXr, static_cast<T*>(dX), N, E, M, d, st));
   {
     SimtGemmArgs a = sg(c->X, 0, 1, d, dZ, 0, E, 1, at<float>(c, c->o_part), 0, E, d, E, N, 1);
     a.splits = c->wr_splits;
     a.c_split = (int64_t)d * E;
-    EC_CUDA(launch_simt_gemm(a, et(c), EType::F32, st), "X^T dZ");
-    EC_CUDA(launch_reduce_splits(at<float>(c, c->o_part), dWr, (int64_t)d * E, c->wr_splits, st),
-            "dWr reduce");
+    EC_KERNEL("router_wgrad_gemm", 1, launch_simt_gemm(a, et(c), EType::F32, st));
+    EC_KERNEL("router_wgrad_reduce", 1,
+              launch_reduce_splits(at<float>(c, c->o_part), dWr, (int64_t)d * E, c->wr_splits, st));
   }
-  if (dbr) EC_CUDA(launch_colsum(dZ, dbr, N, E, st), "dbr");
+  if (dbr) EC_KERNEL("router_dbias", 1, launch_colsum(dZ, dbr, N, E, st));
   return EC_OK;
 }
 
@@ -361,7 +405,11 @@ ec_status ec_ctx_create(ec_ctx** out, int32_t N, int32_t d, int32_t E, int32_t d
   return EC_OK;
 }
 
-void ec_ctx_destroy(ec_ctx* c) { delete c; }
+void ec_ctx_destroy(ec_ctx* c) {
+  if (!c) return;
+  for (cudaEvent_t e : c->ev) cudaEventDestroy(e);
+  delete c;
+}
 
 ec_status ec_ctx_set_capacity(ec_ctx* c, const int32_t* k_g) {
   if (!c) return EC_ERR_INVALID_ARG;
@@ -401,6 +449,7 @@ ec_status ec_route(ec_ctx* c, const void* X, const void* Wr, const float* br, co
   s = c->dtype == EC_BF16 ? run_route<bf16>(c, X, Wr, br, S_in, st)
                           : run_route<float>(c, X, Wr, br, S_in, st);
   if (s != EC_OK) return s;
+  mark(c, "end", st);
   return copy_out(c, idx, gate, S_out, st);
 }
 
@@ -421,6 +470,7 @@ ec_status ec_moe_forward(ec_ctx* c, const void* X, const void* Wr, const float* 
   s = c->dtype == EC_BF16 ? run_forward<bf16>(c, X, Wg, Wu, Wd, Y, st)
                           : run_forward<float>(c, X, Wg, Wu, Wd, Y, st);
   if (s != EC_OK) return s;
+  mark(c, "end", st);
   s = copy_out(c, idx, gate, S_out, st);
   if (s != EC_OK) return s;
   c->X = X; c->Wr = Wr; c->br = br; c->Wg = Wg; c->Wu = Wu; c->Wd = Wd;
@@ -439,9 +489,38 @@ ec_status ec_moe_backward(ec_ctx* c, const void* dY, void* dX, float* dWr, float
                         (const void*)dWd})
     if (!aligned16(p)) return fail(c, EC_ERR_INVALID_ARG, "tensors must be 16-byte aligned");
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  return c->dtype == EC_BF16 ? run_backward<bf16>(c, dY, dX, dWr, dbr, dWg, dWu, dWd, st)
-                             : run_backward<float>(c, dY, dX, dWr, dbr, dWg, dWu, dWd, st);
+  s = c->dtype == EC_BF16 ? run_backward<bf16>(c, dY, dX, dWr, dbr, dWg, dWu, dWd, st)
+                          : run_backward<float>(c, dY, dX, dWr, dbr, dWg, dWu, dWd, st);
+  if (s != EC_OK) return s;
+  mark(c, "end", st);
+  return EC_OK;
 }
+
+ec_status ec_ctx_set_profiling(ec_ctx* c, int32_t on) {
+  if (!c) return EC_ERR_INVALID_ARG;
+  c->prof = on != 0;
+  c->ev_n = 0;
+  return EC_OK;
+}
+
+int32_t ec_ctx_profile(ec_ctx* c, const char** names, float* ms, int32_t cap) {
+  if (!c || c->ev_n == 0) return 0;
+  if (cudaEventSynchronize(c->ev[c->ev_n - 1]) != cudaSuccess) return -1;
+  int32_t n = 0;
+  for (int i = 0; i + 1 < c->ev_n; ++i) {
+    if (std::strcmp(c->ev_name[i], "end") == 0) continue;
+    if (n < cap) {
+      float t = 0.f;
+      cudaEventElapsedTime(&t, c->ev[i], c->ev[i + 1]);
+      if (names) names[n] = c->ev_name[i];
+      if (ms) ms[n] = t;
+    }
+    ++n;
+  }
+  return n;
+}
+
+int64_t ec_kernel_launches(const ec_ctx* c) { return c ? c->launches : -1; }
 
 ec_status ec_check_device(ec_ctx* c, void* stream) {
   ec_status s = check_ready(c);

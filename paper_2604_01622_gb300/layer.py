@@ -8,8 +8,9 @@ from __future__ import annotations
 import torch
 
 from . import (EC_BF16, EC_F32, ec_check_device, ec_ctx_create, ec_ctx_destroy,
-               ec_ctx_set_capacity, ec_ctx_set_workspace, ec_moe_backward, ec_moe_forward,
-               ec_route, ec_rows_per_expert, ec_workspace_bytes)
+               ec_ctx_profile, ec_ctx_set_capacity, ec_ctx_set_profiling, ec_ctx_set_workspace,
+               ec_kernel_launches, ec_moe_backward, ec_moe_forward, ec_route,
+               ec_rows_per_expert, ec_workspace_bytes)
 
 _DT = {"f32": (EC_F32, torch.float32), "bf16": (EC_BF16, torch.bfloat16)}
 
@@ -82,6 +83,17 @@ class ECMoELayer:
         ec_moe_backward(self.ctx, _p(dY), _p(g["dX"]), _p(g["dWr"]), _p(g.get("dbr")),
                         _p(g["dWg"]), _p(g["dWu"]), _p(g["dWd"]), _stream(stream))
         return g
+
+    def set_profiling(self, on: bool):
+        ec_ctx_set_profiling(self.ctx, on)
+
+    def profile(self):
+        """[(kernel, ms)] of every launch since profiling was switched on."""
+        return ec_ctx_profile(self.ctx)
+
+    @property
+    def launches(self) -> int:
+        return ec_kernel_launches(self.ctx)
 
     def check(self, stream=None):
         """Synchronise and raise if a kernel reported a device-side timeout."""
