@@ -132,6 +132,30 @@ int32_t ec_ctx_profile(ec_ctx* ctx, const char** names, float* ms, int32_t cap);
 /* Number of CUDA kernels the library has launched through this context so far. */
 int64_t ec_kernel_launches(const ec_ctx* ctx);
 
+/* Expert-choice selection for callers that cannot allocate device memory (the paper has no
+ * counterpart: this is a deployment variant of the selection in ec_route).
+ *
+ * Some callers cannot call cudaMalloc where they need a selection: a runtime that hands
+ * out a fixed memory budget, or code that must not grow the device footprint once it is
+ * serving. This call needs no context and no workspace: its scratch (the token->slot map
+ * and the group tables) lives in one file-scope device array of
+ * EC_STATIC_SELECT_MAX_SCORES + 3*(EC_STATIC_SELECT_MAX_GROUPS+1) int32 (about 16 MB), which
+ * every GPU that loads the library holds until the process exits. It calls no allocator.
+ *   S [E][N] float scores (device), N tokens in G groups given by the host arrays
+ *   group_off [G+1] and k_g [G] (same rules as ec_ctx_create); idx [E][M] int32 and
+ *   gate [E][M] float (device, M = sum k_g) receive the same selection as ec_route with S_in.
+ * Returns EC_ERR_UNSUPPORTED if N*E > EC_STATIC_SELECT_MAX_SCORES or
+ * G > EC_STATIC_SELECT_MAX_GROUPS, EC_ERR_SHAPE / EC_ERR_INVALID_ARG on bad arguments,
+ * EC_ERR_CUDA if a CUDA call fails. Asynchronous on `stream` (the host tables are copied
+ * before the call returns). The first call on each device looks up the array's device
+ * address; make that first call before any stream capture. All calls share the array:
+ * calls that overlap on the GPU (other streams, other threads) race and must be ordered. */
+#define EC_STATIC_SELECT_MAX_SCORES 4194304
+#define EC_STATIC_SELECT_MAX_GROUPS 4096
+ec_status ec_select_static(const float* S, int32_t N, int32_t E, int32_t G,
+                           const int32_t* group_off, const int32_t* k_g, int32_t* idx,
+                           float* gate, void* stream);
+
 /* Message of the last failed call on this context ("" if none). Owned by the context. */
 const char* ec_last_error(const ec_ctx* ctx);
 

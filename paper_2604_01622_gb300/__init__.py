@@ -25,7 +25,7 @@ EXPORTS = (
     "ec_ctx_create", "ec_ctx_destroy", "ec_ctx_set_capacity", "ec_rows_per_expert",
     "ec_workspace_bytes", "ec_ctx_set_workspace", "ec_route", "ec_moe_forward",
     "ec_moe_backward", "ec_check_device", "ec_last_error", "ec_status_string",
-    "ec_ctx_set_profiling", "ec_ctx_profile", "ec_kernel_launches",
+    "ec_ctx_set_profiling", "ec_ctx_profile", "ec_kernel_launches", "ec_select_static",
 )
 
 _lib = None
@@ -65,6 +65,7 @@ def load():
         "ec_ctx_profile": (i32, [vp, ctypes.POINTER(ctypes.c_char_p),
                                  ctypes.POINTER(ctypes.c_float), i32]),
         "ec_kernel_launches": (i64, [vp]),
+        "ec_select_static": (i32, [vp, i32, i32, i32, P32, P32, vp, vp, vp]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -153,6 +154,15 @@ def ec_ctx_profile(ctx, cap: int = 4096):
 
 def ec_kernel_launches(ctx) -> int:
     return int(load().ec_kernel_launches(ctx))
+
+
+def ec_select_static(S, N, E, group_off, k_g, idx, gate, stream):
+    """Selection with no workspace (scratch in the library's static device array)."""
+    g_arr, g_ptr = _i32(group_off)
+    k_arr, k_ptr = _i32(k_g)
+    st = load().ec_select_static(S, N, E, len(g_arr) - 1, g_ptr, k_ptr, idx, gate, stream)
+    if st != EC_OK:
+        raise ECError(st, "ec_select_static rejected the call")
 
 
 def ec_last_error(ctx) -> str:
