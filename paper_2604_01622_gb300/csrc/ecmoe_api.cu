@@ -22,8 +22,9 @@ struct ec_ctx {
   size_t ws_bytes = 0;
   // workspace offsets (bytes)
   size_t o_status, o_goff, o_kg, o_koff, o_ST, o_S, o_idx, o_gate, o_slot, o_H, o_A, o_B, o_U,
-      o_O, o_dO, o_dA, o_dB, o_dgate, o_dZ, o_wrpad, o_f32a, o_f32b, o_dXr, o_part, total;
-  int wr_splits = 1;
+      o_O, o_dO, o_dA, o_dB, o_dgate, o_dZ, o_dZb, o_wrpad, o_f32a, o_f32b, o_dXr, o_part, total;
+  int wr_splits = 1;   // split-K factor of dWr = X^T dZ
+  int Ep = 64;         // experts rounded up to 64 (tensor-core router operands)
   // per-kernel event timing (off by default) and kernel launch counter
   bool prof = false;
   std::vector<cudaEvent_t> ev;
@@ -119,15 +120,24 @@ void layout(ec_ctx* c) {
   c->o_dB = take(P * F * es);
   c->o_dgate = take(P * 4);
   c->o_dZ = take(N * E * 4);
-  c->o_wrpad = take(d * ((E + 63) / 64 * 64) * 2);
+  c->Ep = (c->E + 63) / 64 * 64;
+  c->o_dZb = take(use_tc(c) ? 2 * N * c->Ep * 2 : 0);
+  c->o_wrpad = take(d * c->Ep * 2);
   // fp32 scratch: SIMT GEMM outputs (fp32 path) and router logits / router dX part
   const size_t f32n = use_tc(c) ? N * E : std::max(std::max(P * F, P * d), N * E);
   c->o_f32a = take(f32n * 4);
   c->o_f32b = take((use_tc(c) ? 0 : std::max(P * F, P * d)) * 4);
   c->o_dXr = take(N * d * 4);
-  // split-K partials of dWr = X^T dZ
-  c->wr_splits = (int)std::max<size_t>(1, std::min<size_t>(64, N / 512));
-  c->o_part = take((size_t)c->wr_splits * d * E * 4);
+  // split-K partials of dWr = X^T dZ (tensor cores: equal token blocks, so N % splits == 0)
+  if (use_tc(c)) {
+    c->wr_splits = 1;
+    for (int s = 16; s > 1; s >>= 1)
+      if (N % s == 0 && N / s >= 256) { c->wr_splits = s; break; }
+    c->o_part = take((size_t)2 * c->wr_splits * d * c->Ep * 4);
+  } else {
+    c->wr_splits = (int)std::max<size_t>(1, std::min<size_t>(64, N / 512));
+    c->o_part = take((size_t)c->wr_splits * d * E * 4);
+  }
   c->total = o;
 }
 
@@ -349,19 +359,34 @@ ec_status run_backward(ec_ctx* c, const void* dY, void* dX, float* dWr, float* d
     EC_CUDA(cudaMemsetAsync(dWd, 0, (size_t)E * d * F * 4, st), "zero dWd");
   }
   // router: dZ = S (dS - <dS,S>), dX = dZ Wr^T + sum dH, dWr = X^T dZ, dbr = sum dZ
-  EC_KERNEL("softmax_bwd", nz, launch_softmax_bwd(at<float>(c, c->o_S), slot, dgate, dZ, N, E, M, st));
   float* dXr = at<float>(c, c->o_dXr);
-  EC_KERNEL("router_dgrad_gemm", nz,
-            launch_simt_gemm(sg(dZ, 0, E, 1, c->Wr, 0, 1, E, dXr, 0, d, N, d, E, 1), EType::F32,
-                             et(c), st));
-  EC_KERNEL("dx_combine", nz, launch_dx_combine<T>(dH, slot, dXr, static_cast<T*>(dX), N, E, M, d, st));
-  {
-    SimtGemmArgs a = sg(c->X, 0, 1, d, dZ, 0, E, 1, at<float>(c, c->o_part), 0, E, d, E, N, 1);
+  float* part = at<float>(c, c->o_part);
+  if (use_tc(c)) {
+    bf16* dZb = at<bf16>(c, c->o_dZb);
+    EC_KERNEL("softmax_bwd", nz,
+              launch_softmax_bwd(at<float>(c, c->o_S), slot, dgate, dZ, dZb, N, E, c->Ep, M, st));
+    EC_KERNEL("router_dgrad_gemm", nz,
+              tc_router_dgrad(dZb, at<void>(c, c->o_wrpad), dXr, N, d, c->Ep, status, st));
+    EC_KERNEL("dx_combine", nz,
+              launch_dx_combine<T>(dH, slot, dXr, static_cast<T*>(dX), N, E, M, d, st));
+    EC_KERNEL("router_wgrad_gemm", nz,
+              tc_router_wgrad(c->X, dZb, part, N, d, c->Ep, c->wr_splits, status, st));
+    EC_KERNEL("router_wgrad_reduce", 1,
+              launch_reduce_partials(part, dWr, d, E, c->Ep, 2 * c->wr_splits, st));
+  } else {
+    EC_KERNEL("softmax_bwd", nz,
+              launch_softmax_bwd(at<float>(c, c->o_S), slot, dgate, dZ, nullptr, N, E, E, M, st));
+    EC_KERNEL("router_dgrad_gemm", nz,
+              launch_simt_gemm(sg(dZ, 0, E, 1, c->Wr, 0, 1, E, dXr, 0, d, N, d, E, 1), EType::F32,
+                               et(c), st));
+    EC_KERNEL("dx_combine", nz,
+              launch_dx_combine<T>(dH, slot, dXr, static_cast<T*>(dX), N, E, M, d, st));
+    SimtGemmArgs a = sg(c->X, 0, 1, d, dZ, 0, E, 1, part, 0, E, d, E, N, 1);
     a.splits = c->wr_splits;
     a.c_split = (int64_t)d * E;
     EC_KERNEL("router_wgrad_gemm", 1, launch_simt_gemm(a, et(c), EType::F32, st));
     EC_KERNEL("router_wgrad_reduce", 1,
-              launch_reduce_splits(at<float>(c, c->o_part), dWr, (int64_t)d * E, c->wr_splits, st));
+              launch_reduce_splits(part, dWr, (int64_t)d * E, c->wr_splits, st));
   }
   if (dbr) EC_KERNEL("router_dbias", 1, launch_colsum(dZ, dbr, N, E, st));
   return EC_OK;

@@ -201,15 +201,10 @@ __device__ __forceinline__ void store_bf16x32(void* dst, const float* v) {
                       pack_bf16x2(v[8 * i + 4], v[8 * i + 5]),
                       pack_bf16x2(v[8 * i + 6], v[8 * i + 7]));
 }
-__device__ __forceinline__ void load_bf16x32(const void* src, float* v) {
-  const uint4* s = reinterpret_cast<const uint4*>(src);
-#pragma unroll
-  for (int i = 0; i < 4; ++i) unpack16(__ldg(s + i), v + 8 * i, bf16());
-}
 
 // ------------------------------------------------------------------ the kernel
-template <int BN, bool A_MN, bool B_MN, bool B_SPLIT, bool K_SPLIT, int EPI, int STAGES>
-__global__ void __launch_bounds__(192, 1)
+template <int BN, bool A_MN, bool B_MN, bool B_SPLIT, bool K_SPLIT, int EPI, int STAGES, int EPW>
+__global__ void __launch_bounds__(64 + 32 * EPW, 1)
 tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ CUtensorMap mA1,
                const __grid_constant__ CUtensorMap mB0, const __grid_constant__ CUtensorMap mB1,
                const Args p) {
@@ -218,6 +213,8 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
   constexpr uint32_t TCOLS = tmem_cols<BN>();
   constexpr uint32_t IDESC = instr_desc<BN, A_MN, B_MN>();
   static_assert(BN % 64 == 0 && BN <= 256, "BN");
+  static_assert(EPW == 4 || EPW == 8, "epilogue warps: one or two per TMEM lane quarter");
+  static_assert(EPI != EPI_ROUTER || EPW == 4, "the row softmax needs whole rows per thread");
 
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -241,7 +238,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(&tfull[a], 1);
-      mbar_init(&tempty[a], 4);
+      mbar_init(&tempty[a], EPW);
     }
     mbar_init(mma_done, 1);
     *abort_flag = 0;
@@ -290,7 +287,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
               tma_load_3d(a_dst + j * 8192, mA, &full[s], m0 + 64 * j, k0, b);
           }
           if (!B_MN) {
-            if (B_SPLIT) {
+            if constexpr (B_SPLIT) {
               const int n0h = nt * (BN / 2);
               tma_load_3d(b_dst, &mB0, &full[s], k0, n0h, b);
               tma_load_3d(b_dst + (BN / 2) * 128, &mB1, &full[s], k0, n0h, b);
@@ -301,7 +298,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
             constexpr int NB = BN / 64;
 #pragma unroll
             for (int j = 0; j < NB; ++j) {
-              if (B_SPLIT) {
+              if constexpr (B_SPLIT) {
                 const int n0h = nt * (BN / 2);
                 const CUtensorMap* m = j < NB / 2 ? &mB0 : &mB1;
                 tma_load_3d(b_dst + j * 8192, m, &full[s], n0h + 64 * (j % (NB / 2)), k0, b);
@@ -361,9 +358,11 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
     }
     __syncwarp();
   } else {
-    // ------------------------------------------------------------ epilogue (warps 2..5)
+    // ------------------------------------------------------------ epilogue (warps 2..)
     const int q = warp & 3;             // TMEM lane quarter this warp may access
     const int r = q * 32 + lane;        // row within the tile
+    constexpr int NPART = EPW / 4;      // warps sharing a lane quarter split the columns
+    const int part = (warp - 2) / 4;
     int it = 0;
     for (int tile = blockIdx.x; tile < total; tile += gridDim.x, ++it) {
       const int a = it & 1;
@@ -380,9 +379,11 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
       uint32_t v[32];
       float f[32];
 
+      constexpr int NC32 = BN / 32 / NPART;   // 32-column chunks per warp
+      const int c32 = part * NC32;
       if constexpr (EPI == EPI_STORE_BF16 || EPI == EPI_STORE_F32) {
 #pragma unroll 1
-        for (int c = 0; c < BN / 32; ++c) {
+        for (int c = c32; c < c32 + NC32; ++c) {
           tmem_ld32(tacc + c * 32, v);
           tmem_wait_ld();
           const int n = nt * BN + c * 32;
@@ -400,7 +401,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
         }
       } else if constexpr (EPI == EPI_STORE_F32_SPLIT) {
 #pragma unroll 1
-        for (int c = 0; c < BN / 32; ++c) {
+        for (int c = c32; c < c32 + NC32; ++c) {
           tmem_ld32(tacc + c * 32, v);
           tmem_wait_ld();
           const int half = c >= BN / 64;
@@ -415,8 +416,9 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
         }
       } else if constexpr (EPI == EPI_SWIGLU_FWD) {
         uint32_t w[32];
+        constexpr int NC64 = BN / 64 / NPART;
 #pragma unroll 1
-        for (int c = 0; c < BN / 64; ++c) {
+        for (int c = part * NC64; c < (part + 1) * NC64; ++c) {
           tmem_ld32(tacc + c * 32, v);
           tmem_ld32(tacc + BN / 2 + c * 32, w);
           tmem_wait_ld();
@@ -437,16 +439,34 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
           }
         }
       } else if constexpr (EPI == EPI_SWIGLU_BWD) {
+        // A and B of the next chunk are requested before the current one is computed
+        const bf16* pa = reinterpret_cast<const bf16*>(p.in0) + row_off + nt * BN;
+        const bf16* pb = reinterpret_cast<const bf16*>(p.in1) + row_off + nt * BN;
+        uint4 ra[4], rb[4], na[4], nb[4];
+        auto fetch = [&](int c, uint4* xa, uint4* xb) {
+          const int n = nt * BN + c * 32;
+          if (row_ok && n < p.N) {
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              xa[i] = __ldg(reinterpret_cast<const uint4*>(pa + c * 32) + i);
+              xb[i] = __ldg(reinterpret_cast<const uint4*>(pb + c * 32) + i);
+            }
+          }
+        };
+        fetch(c32, ra, rb);
 #pragma unroll 1
-        for (int c = 0; c < BN / 32; ++c) {
+        for (int c = c32; c < c32 + NC32; ++c) {
+          if (c + 1 < c32 + NC32) fetch(c + 1, na, nb);
           tmem_ld32(tacc + c * 32, v);
           tmem_wait_ld();
           const int n = nt * BN + c * 32;
           if (row_ok && n < p.N) {
-            float av[32], bv[32];
-            load_bf16x32(reinterpret_cast<const bf16*>(p.in0) + row_off + n, av);
-            load_bf16x32(reinterpret_cast<const bf16*>(p.in1) + row_off + n, bv);
-            float db[32];
+            float av[32], bv[32], db[32];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              unpack16(ra[i], av + 8 * i, bf16());
+              unpack16(rb[i], bv + 8 * i, bf16());
+            }
 #pragma unroll
             for (int i = 0; i < 32; ++i) {
               const float du = f32(v[i]);
@@ -457,6 +477,8 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
             store_bf16x32(reinterpret_cast<bf16*>(p.out0) + row_off + n, f);
             store_bf16x32(reinterpret_cast<bf16*>(p.out1) + row_off + n, db);
           }
+#pragma unroll
+          for (int i = 0; i < 4; ++i) { ra[i] = na[i]; rb[i] = nb[i]; }
         }
       } else if constexpr (EPI == EPI_ROUTER) {
         const int E = p.n_valid;
@@ -558,10 +580,11 @@ int sm_count() {
   return n;
 }
 
-template <int BN, bool A_MN, bool B_MN, bool B_SPLIT, bool K_SPLIT, int EPI, int STAGES>
+template <int BN, bool A_MN, bool B_MN, bool B_SPLIT, bool K_SPLIT, int EPI, int STAGES,
+          int EPW = 8>
 cudaError_t launch(const CUtensorMap& a0, const CUtensorMap& a1, const CUtensorMap& b0,
                    const CUtensorMap& b1, const Args& p, cudaStream_t st) {
-  auto kern = tc_gemm_kernel<BN, A_MN, B_MN, B_SPLIT, K_SPLIT, EPI, STAGES>;
+  auto kern = tc_gemm_kernel<BN, A_MN, B_MN, B_SPLIT, K_SPLIT, EPI, STAGES, EPW>;
   constexpr uint32_t smem = smem_bytes<BN, STAGES>();
   static bool attr = false;
   if (!attr) {
@@ -572,7 +595,7 @@ cudaError_t launch(const CUtensorMap& a0, const CUtensorMap& a1, const CUtensorM
   const int total = p.batch * p.m_tiles * p.n_tiles;
   if (total == 0 || p.k_blocks == 0) return cudaSuccess;
   const int grid = total < sm_count() ? total : sm_count();
-  kern<<<grid, 192, smem, st>>>(a0, a1, b0, b1, p);
+  kern<<<grid, 64 + 32 * EPW, smem, st>>>(a0, a1, b0, b1, p);
   return cudaGetLastError();
 }
 
@@ -638,10 +661,10 @@ cudaError_t tc_router_softmax(const void* X, const void* Wr, void* Wr_pad, const
   p.bias = br;
   p.n_valid = E;
   switch (Ep) {
-    case 64: return launch<64, false, true, false, false, EPI_ROUTER, 8>(ma, ma, mb, mb, p, st);
-    case 128: return launch<128, false, true, false, false, EPI_ROUTER, 6>(ma, ma, mb, mb, p, st);
-    case 192: return launch<192, false, true, false, false, EPI_ROUTER, 5>(ma, ma, mb, mb, p, st);
-    case 256: return launch<256, false, true, false, false, EPI_ROUTER, 4>(ma, ma, mb, mb, p, st);
+    case 64: return launch<64, false, true, false, false, EPI_ROUTER, 8, 4>(ma, ma, mb, mb, p, st);
+    case 128: return launch<128, false, true, false, false, EPI_ROUTER, 6, 4>(ma, ma, mb, mb, p, st);
+    case 192: return launch<192, false, true, false, false, EPI_ROUTER, 5, 4>(ma, ma, mb, mb, p, st);
+    case 256: return launch<256, false, true, false, false, EPI_ROUTER, 4, 4>(ma, ma, mb, mb, p, st);
   }
   return cudaErrorInvalidValue;
 }
@@ -732,6 +755,46 @@ cudaError_t tc_expert_wgrad(const void* H, const void* U, const void* dO, const 
     TC_TRY((launch<256, true, true, true, false, EPI_STORE_F32_SPLIT, 4>(ma, ma, mb0, mb1, p, st)));
   }
   return cudaSuccess;
+}
+
+cudaError_t tc_router_dgrad(const void* dZb, const void* Wr_pad, float* dXr, int N, int d, int Ep,
+                            int* status, cudaStream_t st) {
+  if (N == 0) return cudaSuccess;
+  // dXr [N][d] = (dZ_hi + dZ_lo) [N][Ep] . Wr^T as one K loop over both planes;
+  // B[n=i][k=e] = Wr_pad[i][e] is K-major
+  const bf16* hi = static_cast<const bf16*>(dZb);
+  CUtensorMap ma0, ma1, mb;
+  TC_TRY(make_map(&ma0, hi, Ep, N, 1, BM));
+  TC_TRY(make_map(&ma1, hi + (size_t)N * Ep, Ep, N, 1, BM));
+  TC_TRY(make_map(&mb, Wr_pad, Ep, d, 1, 256));
+  Args p = base_args(1, N, d, 2 * Ep, 256, status);
+  p.k_blocks0 = Ep / BK;
+  p.out0 = dXr;
+  p.ld = d;
+  p.bstride = 0;
+  return launch<256, false, false, false, true, EPI_STORE_F32, 4>(ma0, ma1, mb, mb, p, st);
+}
+
+cudaError_t tc_router_wgrad(const void* X, const void* dZb, float* part, int N, int d, int Ep,
+                            int splits, int* status, cudaStream_t st) {
+  if (N == 0) return cudaSuccess;
+  // part[h][s] [d][Ep] = X_s^T . dZ_h,s over the s-th block of N/splits tokens (split K as the
+  // batch), h = hi / lo plane of dZ (the two column halves of each tile)
+  const int rows = N / splits;
+  const bf16* hi = static_cast<const bf16*>(dZb);
+  CUtensorMap ma, mb0, mb1;
+  TC_TRY(make_map(&ma, X, d, rows, splits, 64));
+  TC_TRY(make_map(&mb0, hi, Ep, rows, splits, 64));
+  TC_TRY(make_map(&mb1, hi + (size_t)N * Ep, Ep, rows, splits, 64));
+  const int BNt = Ep > 64 ? 256 : 128;
+  Args p = base_args(splits, d, Ep, rows, BNt / 2, status);
+  p.out0 = part;
+  p.out1 = part + (size_t)splits * d * Ep;
+  p.ld = Ep;
+  p.bstride = (int64_t)d * Ep;
+  if (BNt == 128)
+    return launch<128, true, true, true, false, EPI_STORE_F32_SPLIT, 6>(ma, ma, mb0, mb1, p, st);
+  return launch<256, true, true, true, false, EPI_STORE_F32_SPLIT, 4>(ma, ma, mb0, mb1, p, st);
 }
 
 cudaError_t tc_wait_probe(int* status, unsigned long long limit_ns, cudaStream_t st) {

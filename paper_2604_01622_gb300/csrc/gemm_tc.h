@@ -39,6 +39,16 @@ cudaError_t tc_expert_wgrad(const void* H, const void* U, const void* dO, const 
                             const void* dB, float* dWg, float* dWu, float* dWd, int E, int M,
                             int d, int F, int* status, cudaStream_t st);
 
+// Router backward on the tensor cores. dZb [2][N][Ep] bf16: hi and lo planes of the
+// zero-padded softmax gradient (dZ ~ hi + lo); Wr_pad [d][Ep] bf16 (the padded router
+// weights of the forward pass). dXr [N][d] fp32 = dZ . Wr^T.
+cudaError_t tc_router_dgrad(const void* dZb, const void* Wr_pad, float* dXr, int N, int d, int Ep,
+                            int* status, cudaStream_t st);
+// part [2][splits][d][Ep] fp32: X^T . dZ_plane over `splits` equal blocks of tokens
+// (N % splits == 0); dWr is the sum of all 2*splits partials.
+cudaError_t tc_router_wgrad(const void* X, const void* dZb, float* part, int N, int d, int Ep,
+                            int splits, int* status, cudaStream_t st);
+
 // Launch a kernel that waits, with the given limit, on an mbarrier nothing completes, so
 // the bounded-wait path (status word, early return) can be exercised without a hang.
 cudaError_t tc_wait_probe(int* status, unsigned long long limit_ns, cudaStream_t st);

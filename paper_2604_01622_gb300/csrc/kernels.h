@@ -2,6 +2,7 @@
 #pragma once
 #include <cuda_runtime.h>
 #include <stdint.h>
+#include <cuda_bf16.h>
 
 namespace ecmoe {
 
@@ -27,7 +28,9 @@ template <typename T>
 cudaError_t launch_bwd_gather_scale(const T* dY, const T* O, const int* idx, const float* gate,
                                     T* dO, float* dgate, int64_t P, int d, cudaStream_t st);
 cudaError_t launch_softmax_bwd(const float* S, const int* slot, const float* dgate, float* dZ,
-                               int N, int E, int M, cudaStream_t st);
+                               __nv_bfloat16* dZb, int N, int E, int Ep, int M, cudaStream_t st);
+cudaError_t launch_reduce_partials(const float* part, float* out, int rows, int cols, int ld,
+                                   int splits, cudaStream_t st);
 template <typename T>
 cudaError_t launch_dx_combine(const T* dH, const int* slot, const float* dXr, T* dX, int N, int E,
                               int M, int d, cudaStream_t st);

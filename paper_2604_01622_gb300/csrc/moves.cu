@@ -147,9 +147,13 @@ cudaError_t launch_bwd_gather_scale(const T* dY, const T* O, const int* idx, con
 
 // ------------------------------------------------------------------ softmax Jacobian
 // dS[t,e] = dgate of the pair (t chosen by e) else 0; dZ = S * (dS - <dS, S>).
+// Optionally also writes dZ as two bf16 planes [2][N][Ep], hi = bf16(dZ) and
+// lo = bf16(dZ - hi), zero in the padding columns E..Ep-1: the tensor-core operands of the
+// router-gradient GEMMs, which sum the products of both planes (hi + lo carries dZ to
+// about 16 significant bits, so the GEMMs keep near-fp32 accuracy).
 __global__ void softmax_bwd_kernel(const float* __restrict__ S, const int* __restrict__ slot,
-                                   const float* __restrict__ dgate, float* __restrict__ dZ, int N,
-                                   int E, int M) {
+                                   const float* __restrict__ dgate, float* __restrict__ dZ,
+                                   bf16* __restrict__ dZb, int N, int E, int Ep, int M) {
   const int t = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (t >= N) return;
@@ -164,14 +168,46 @@ __global__ void softmax_bwd_kernel(const float* __restrict__ S, const int* __res
     const int m = slot[(size_t)t * E + e];
     const float ds = m >= 0 ? dgate[(size_t)e * M + m] : 0.f;
     const float s = S[(size_t)t * E + e];
-    dZ[(size_t)t * E + e] = s * (ds - dot);
+    const float z = s * (ds - dot);
+    dZ[(size_t)t * E + e] = z;
+    if (dZb) {
+      const bf16 hi = __float2bfloat16_rn(z);
+      dZb[(size_t)t * Ep + e] = hi;
+      dZb[(size_t)N * Ep + (size_t)t * Ep + e] = __float2bfloat16_rn(z - __bfloat162float(hi));
+    }
   }
+  if (dZb)
+    for (int e = E + lane; e < Ep; e += 32) {
+      dZb[(size_t)t * Ep + e] = __float2bfloat16_rn(0.f);
+      dZb[(size_t)N * Ep + (size_t)t * Ep + e] = __float2bfloat16_rn(0.f);
+    }
 }
 
 cudaError_t launch_softmax_bwd(const float* S, const int* slot, const float* dgate, float* dZ,
-                               int N, int E, int M, cudaStream_t st) {
+                               bf16* dZb, int N, int E, int Ep, int M, cudaStream_t st) {
   if (N == 0) return cudaSuccess;
-  softmax_bwd_kernel<<<(N + 7) / 8, 256, 0, st>>>(S, slot, dgate, dZ, N, E, M);
+  softmax_bwd_kernel<<<(N + 7) / 8, 256, 0, st>>>(S, slot, dgate, dZ, dZb, N, E, Ep, M);
+  return cudaGetLastError();
+}
+
+// out[i][e] = sum_s part[s][i][e] for the first `cols` of `ld` columns.
+__global__ void reduce_partials_kernel(const float* __restrict__ part, float* __restrict__ out,
+                                       int rows, int cols, int ld, int splits) {
+  const int64_t n = (int64_t)rows * cols;
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+       i += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t r = i / cols, c = i % cols;
+    float s = 0.f;
+    for (int k = 0; k < splits; ++k) s += part[((int64_t)k * rows + r) * ld + c];
+    out[i] = s;
+  }
+}
+
+cudaError_t launch_reduce_partials(const float* part, float* out, int rows, int cols, int ld,
+                                   int splits, cudaStream_t st) {
+  if (rows == 0 || cols == 0) return cudaSuccess;
+  reduce_partials_kernel<<<grid_for((int64_t)rows * cols, 152 * 16), 256, 0, st>>>(
+      part, out, rows, cols, ld, splits);
   return cudaGetLastError();
 }
 
