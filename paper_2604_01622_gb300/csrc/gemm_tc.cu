@@ -72,7 +72,7 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
   uint32_t ok;
   asm volatile(
       "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
       "selp.u32 %0, 1, 0, p;\n\t}"
       : "=r"(ok)
       : "r"(bar), "r"(parity)
@@ -145,6 +145,65 @@ __device__ __forceinline__ void mma_commit(uint64_t* bar) {
           smem_u32(bar))
       : "memory");
 }
+// ---- CTA-pair (cluster of 2) forms: one MMA spans the two SMs' tensor cores, M = 256
+__device__ __forceinline__ uint32_t cluster_ctarank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+// Shared-memory address of the same variable in CTA `rank` of the cluster.
+__device__ __forceinline__ uint32_t mapa_shared(uint32_t addr, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" :::
+                   "memory");
+}
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr)
+               : "memory");
+}
+// TMA load whose completion is signalled on an mbarrier of either CTA of the pair.
+__device__ __forceinline__ void tma_load_3d_pair(void* dst, const CUtensorMap* map, uint32_t bar,
+                                                 int c0, int c1, int c2) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%3, %4, %5}], [%2];" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(c0), "r"(c1), "r"(c2)
+      : "memory");
+}
+__device__ __forceinline__ void tmem_alloc_pair(uint32_t* holder, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                   smem_u32(holder)),
+               "r"(ncols)
+               : "memory");
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc_pair(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void mma_bf16_pair(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
+                                              uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+// Arrive on the mbarrier at this shared offset in every CTA of `mask` once the MMAs issued
+// so far have completed.
+__device__ __forceinline__ void mma_commit_pair(uint64_t* bar, uint16_t mask) {
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
+      " [%0], %1;" ::"r"(smem_u32(bar)),
+      "h"(mask)
+      : "memory");
+}
+
 // 32 consecutive fp32 columns of this thread's TMEM lane.
 __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t* v) {
   asm volatile(
@@ -174,11 +233,12 @@ __device__ __forceinline__ uint64_t smem_desc(uint32_t saddr, uint32_t lbo, uint
   return d;
 }
 
-// Instruction descriptor of kind::f16: fp32 accumulator, bf16 A and B, M = 128.
-template <int BN, bool A_MN, bool B_MN>
+// Instruction descriptor of kind::f16: fp32 accumulator, bf16 A and B, M x BN (M = 128 for
+// one CTA, 256 for a CTA pair).
+template <int BN, bool A_MN, bool B_MN, int MMA_M>
 __host__ __device__ constexpr uint32_t instr_desc() {
   return (1u << 4) | (1u << 7) | (1u << 10) | ((A_MN ? 1u : 0u) << 15) |
-         ((B_MN ? 1u : 0u) << 16) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
+         ((B_MN ? 1u : 0u) << 16) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(MMA_M >> 4) << 24);
 }
 
 template <int BN>
@@ -186,9 +246,10 @@ __host__ __device__ constexpr uint32_t tmem_cols() {
   return 2 * BN <= 32 ? 32 : 2 * BN <= 64 ? 64 : 2 * BN <= 128 ? 128 : 2 * BN <= 256 ? 256 : 512;
 }
 
-template <int BN, int STAGES>
+template <int BN, int STAGES, bool PAIR>
 __host__ __device__ constexpr uint32_t smem_bytes() {
-  return 1024 /*align slack*/ + STAGES * (BM * BK * 2 + BN * BK * 2) + 256 /*barriers*/;
+  return 1024 /*align slack*/ + STAGES * (BM * BK * 2 + (PAIR ? BN / 2 : BN) * BK * 2) +
+         256 /*barriers*/;
 }
 
 __device__ __forceinline__ float f32(uint32_t u) { return __uint_as_float(u); }
@@ -203,16 +264,24 @@ __device__ __forceinline__ void store_bf16x32(void* dst, const float* v) {
 }
 
 // ------------------------------------------------------------------ the kernel
-template <int BN, bool A_MN, bool B_MN, bool B_SPLIT, bool K_SPLIT, int EPI, int STAGES, int EPW>
+// PAIR: the CTAs of a 2-CTA cluster share each 256 x BN tile. Each CTA loads its own 128 rows
+// of A and half (BN/2 columns) of B; the leader CTA (rank 0) issues M = 256 MMAs that read
+// both CTAs' shared memory and write each CTA's 128 rows into that CTA's TMEM. Per SM this
+// halves the B traffic into shared memory.
+template <int BN, bool A_MN, bool B_MN, bool B_SPLIT, bool K_SPLIT, int EPI, int STAGES, int EPW,
+          bool PAIR>
 __global__ void __launch_bounds__(64 + 32 * EPW, 1)
 tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ CUtensorMap mA1,
                const __grid_constant__ CUtensorMap mB0, const __grid_constant__ CUtensorMap mB1,
                const Args p) {
+  constexpr int BNL = PAIR ? BN / 2 : BN;     // B columns held by this CTA
+  constexpr int TM = PAIR ? 2 * BM : BM;      // tile rows
   constexpr uint32_t A_BYTES = BM * BK * 2;
-  constexpr uint32_t B_BYTES = BN * BK * 2;
+  constexpr uint32_t B_BYTES = BNL * BK * 2;
   constexpr uint32_t TCOLS = tmem_cols<BN>();
-  constexpr uint32_t IDESC = instr_desc<BN, A_MN, B_MN>();
+  constexpr uint32_t IDESC = instr_desc<BN, A_MN, B_MN, TM>();
   static_assert(BN % 64 == 0 && BN <= 256, "BN");
+  static_assert(!PAIR || BN % 128 == 0, "pair tiles split B in two 64-column multiples");
   static_assert(EPW == 4 || EPW == 8, "epilogue warps: one or two per TMEM lane quarter");
   static_assert(EPI != EPI_ROUTER || EPW == 4, "the row softmax needs whole rows per thread");
 
@@ -231,6 +300,10 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t rank = PAIR ? cluster_ctarank() : 0u;
+  const bool leader = rank == 0;
+  const int cid = PAIR ? (int)(blockIdx.x >> 1) : (int)blockIdx.x;  // tile walker index
+  const int nwalk = PAIR ? (int)(gridDim.x >> 1) : (int)gridDim.x;
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
       mbar_init(&full[s], 1);
@@ -238,7 +311,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(&tfull[a], 1);
-      mbar_init(&tempty[a], EPW);
+      mbar_init(&tempty[a], PAIR ? 2 * EPW : EPW);
     }
     mbar_init(mma_done, 1);
     *abort_flag = 0;
@@ -250,9 +323,13 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
     if (K_SPLIT) prefetch_map(&mA1);
     if (K_SPLIT || B_SPLIT) prefetch_map(&mB1);
   }
-  if (warp == 1) tmem_alloc(tmem_holder, TCOLS);
+  if (warp == 1) {
+    if constexpr (PAIR) tmem_alloc_pair(tmem_holder, TCOLS);
+    else tmem_alloc(tmem_holder, TCOLS);
+  }
   tc_fence_before();
   __syncthreads();
+  if constexpr (PAIR) cluster_sync();   // the peer's barriers are initialised before use
   tc_fence_after();
   const uint32_t tmem_base = *tmem_holder;
 
@@ -265,14 +342,20 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
       int s = 0;
       uint32_t ph = 0;
       bool ok = true;
-      for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x) {
+      for (int tile = cid; tile < total && ok; tile += nwalk) {
         const int b = tile / tiles_per_b;
         const int rem = tile - b * tiles_per_b;
         const int mt = rem / p.n_tiles, nt = rem - mt * p.n_tiles;
-        const int m0 = mt * BM;
+        const int m0 = mt * TM + (int)rank * BM;
         for (int kb = 0; kb < p.k_blocks; ++kb) {
           if (!mbar_wait(&empty[s], ph ^ 1u, abort_flag, p.status)) { ok = false; break; }
-          mbar_arrive_expect_tx(&full[s], A_BYTES + B_BYTES);
+          if (!PAIR || leader) mbar_arrive_expect_tx(&full[s], (A_BYTES + B_BYTES) * (PAIR ? 2 : 1));
+          // completion goes to the leader's barrier: it gates the pair's MMAs
+          const uint32_t fb = PAIR ? mapa_shared(smem_u32(&full[s]), 0) : smem_u32(&full[s]);
+          auto load = [&](void* dst, const CUtensorMap* m, int c0, int c1) {
+            if constexpr (PAIR) tma_load_3d_pair(dst, m, fb, c0, c1, b);
+            else tma_load_3d(dst, m, &full[s], c0, c1, b);
+          };
           const bool second = K_SPLIT && kb >= p.k_blocks0;
           const CUtensorMap* mA = second ? &mA1 : &mA0;
           const CUtensorMap* mB = second ? &mB1 : &mB0;
@@ -280,19 +363,28 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
           uint8_t* a_dst = sA + s * A_BYTES;
           uint8_t* b_dst = sB + s * B_BYTES;
           if (!A_MN) {
-            tma_load_3d(a_dst, mA, &full[s], k0, m0, b);
+            load(a_dst, mA, k0, m0);
           } else {
 #pragma unroll
-            for (int j = 0; j < BM / 64; ++j)
-              tma_load_3d(a_dst + j * 8192, mA, &full[s], m0 + 64 * j, k0, b);
+            for (int j = 0; j < BM / 64; ++j) load(a_dst + j * 8192, mA, m0 + 64 * j, k0);
           }
-          if (!B_MN) {
+          if constexpr (PAIR) {
+            // this CTA's half of the B tile: for split tiles the gate (rank 0) or up half
+            const CUtensorMap* mb = B_SPLIT ? (rank ? &mB1 : &mB0) : mB;
+            const int n0 = B_SPLIT ? nt * (BN / 2) : nt * BN + (int)rank * BNL;
+            if (!B_MN) {
+              load(b_dst, mb, k0, n0);
+            } else {
+#pragma unroll
+              for (int j = 0; j < BNL / 64; ++j) load(b_dst + j * 8192, mb, n0 + 64 * j, k0);
+            }
+          } else if (!B_MN) {
             if constexpr (B_SPLIT) {
               const int n0h = nt * (BN / 2);
-              tma_load_3d(b_dst, &mB0, &full[s], k0, n0h, b);
-              tma_load_3d(b_dst + (BN / 2) * 128, &mB1, &full[s], k0, n0h, b);
+              load(b_dst, &mB0, k0, n0h);
+              load(b_dst + (BN / 2) * 128, &mB1, k0, n0h);
             } else {
-              tma_load_3d(b_dst, mB, &full[s], k0, nt * BN, b);
+              load(b_dst, mB, k0, nt * BN);
             }
           } else {
             constexpr int NB = BN / 64;
@@ -301,9 +393,9 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
               if constexpr (B_SPLIT) {
                 const int n0h = nt * (BN / 2);
                 const CUtensorMap* m = j < NB / 2 ? &mB0 : &mB1;
-                tma_load_3d(b_dst + j * 8192, m, &full[s], n0h + 64 * (j % (NB / 2)), k0, b);
+                load(b_dst + j * 8192, m, n0h + 64 * (j % (NB / 2)), k0);
               } else {
-                tma_load_3d(b_dst + j * 8192, mB, &full[s], nt * BN + 64 * j, k0, b);
+                load(b_dst + j * 8192, mB, nt * BN + 64 * j, k0);
               }
             }
           }
@@ -318,13 +410,13 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
     }
     __syncwarp();
   } else if (warp == 1) {
-    // ------------------------------------------------------------ MMA issuer
-    if (lane == 0) {
+    // ------------------------------------------------------------ MMA issuer (leader CTA)
+    if (lane == 0 && leader) {
       int s = 0;
       uint32_t ph = 0;
       bool ok = true;
       int it = 0;
-      for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x, ++it) {
+      for (int tile = cid; tile < total && ok; tile += nwalk, ++it) {
         const int a = it & 1;
         const uint32_t use = (uint32_t)(it >> 1);
         if (!mbar_wait(&tempty[a], (use & 1u) ^ 1u, abort_flag, p.status)) { ok = false; break; }
@@ -341,17 +433,21 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
                                      : smem_desc(sa + j * 32, 16, 1024);
             const uint64_t bd = B_MN ? smem_desc(sb + j * 2048, 8192, 1024)
                                      : smem_desc(sb + j * 32, 16, 1024);
-            mma_bf16(tacc, ad, bd, IDESC, (kb | j) != 0 ? 1u : 0u);
+            if constexpr (PAIR) mma_bf16_pair(tacc, ad, bd, IDESC, (kb | j) != 0 ? 1u : 0u);
+            else mma_bf16(tacc, ad, bd, IDESC, (kb | j) != 0 ? 1u : 0u);
           }
-          mma_commit(&empty[s]);
+          if constexpr (PAIR) mma_commit_pair(&empty[s], 0x3);
+          else mma_commit(&empty[s]);
           if (++s == STAGES) { s = 0; ph ^= 1u; }
         }
         if (!ok) break;
-        mma_commit(&tfull[a]);
+        if constexpr (PAIR) mma_commit_pair(&tfull[a], 0x3);
+        else mma_commit(&tfull[a]);
       }
       if (!ok) {
         // wait for the MMAs already issued before TMEM is released
-        mma_commit(mma_done);
+        if constexpr (PAIR) mma_commit_pair(mma_done, 0x1);
+        else mma_commit(mma_done);
         volatile int keep_waiting = 0;
         mbar_wait(mma_done, 0, &keep_waiting, p.status, 100000000ull);
       }
@@ -364,7 +460,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
     constexpr int NPART = EPW / 4;      // warps sharing a lane quarter split the columns
     const int part = (warp - 2) / 4;
     int it = 0;
-    for (int tile = blockIdx.x; tile < total; tile += gridDim.x, ++it) {
+    for (int tile = cid; tile < total; tile += nwalk, ++it) {
       const int a = it & 1;
       const uint32_t use = (uint32_t)(it >> 1);
       if (!mbar_wait(&tfull[a], use & 1u, abort_flag, p.status)) break;
@@ -372,7 +468,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
       const int b = tile / tiles_per_b;
       const int rem = tile - b * tiles_per_b;
       const int mt = rem / p.n_tiles, nt = rem - mt * p.n_tiles;
-      const int gm = mt * BM + r;
+      const int gm = mt * TM + (int)rank * BM + r;
       const bool row_ok = gm < p.M;
       const uint32_t tacc = tmem_base + (uint32_t)(a * BN) + ((uint32_t)(q * 32) << 16);
       const int64_t row_off = (int64_t)b * p.bstride + (int64_t)gm * p.ld;
@@ -524,14 +620,20 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
       }
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&tempty[a]);
+      if (lane == 0) {
+        // the accumulator is free again: tell the CTA that issues the MMAs
+        if constexpr (PAIR) mbar_arrive_cluster(mapa_shared(smem_u32(&tempty[a]), 0));
+        else mbar_arrive(&tempty[a]);
+      }
     }
   }
   tc_fence_before();
   __syncthreads();
+  if constexpr (PAIR) cluster_sync();   // the pair's MMAs and remote arrivals are done
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem_base, TCOLS);
+    if constexpr (PAIR) tmem_dealloc_pair(tmem_base, TCOLS);
+    else tmem_dealloc(tmem_base, TCOLS);
   }
 }
 
@@ -581,21 +683,48 @@ int sm_count() {
 }
 
 template <int BN, bool A_MN, bool B_MN, bool B_SPLIT, bool K_SPLIT, int EPI, int STAGES,
-          int EPW = 8>
+          int EPW = 8, bool PAIR = false>
 cudaError_t launch(const CUtensorMap& a0, const CUtensorMap& a1, const CUtensorMap& b0,
-                   const CUtensorMap& b1, const Args& p, cudaStream_t st) {
-  auto kern = tc_gemm_kernel<BN, A_MN, B_MN, B_SPLIT, K_SPLIT, EPI, STAGES, EPW>;
-  constexpr uint32_t smem = smem_bytes<BN, STAGES>();
+                   const CUtensorMap& b1, Args p, cudaStream_t st) {
+  auto kern = tc_gemm_kernel<BN, A_MN, B_MN, B_SPLIT, K_SPLIT, EPI, STAGES, EPW, PAIR>;
+  constexpr uint32_t smem = smem_bytes<BN, STAGES, PAIR>();
+  constexpr int threads = 64 + 32 * EPW;
   static bool attr = false;
+  static int max_clusters = 0;
+  cudaLaunchAttribute cl[1];
+  cl[0].id = cudaLaunchAttributeClusterDimension;
+  cl[0].val.clusterDim.x = 2;
+  cl[0].val.clusterDim.y = 1;
+  cl[0].val.clusterDim.z = 1;
+  cudaLaunchConfig_t cfg = {};
+  cfg.blockDim = dim3(threads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  if (PAIR) {
+    cfg.attrs = cl;
+    cfg.numAttrs = 1;
+  }
   if (!attr) {
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
+    if (PAIR) {
+      cfg.gridDim = dim3(2 * sm_count());
+      e = cudaOccupancyMaxActiveClusters(&max_clusters, kern, &cfg);
+      if (e != cudaSuccess) return e;
+      if (max_clusters <= 0) return cudaErrorNotSupported;
+    }
     attr = true;
   }
+  if (PAIR) p.m_tiles = (p.M + 2 * BM - 1) / (2 * BM);
   const int total = p.batch * p.m_tiles * p.n_tiles;
   if (total == 0 || p.k_blocks == 0) return cudaSuccess;
+  if (PAIR) {
+    const int clusters = total < max_clusters ? total : max_clusters;
+    cfg.gridDim = dim3(2 * clusters);
+    return cudaLaunchKernelEx(&cfg, kern, a0, a1, b0, b1, p);
+  }
   const int grid = total < sm_count() ? total : sm_count();
-  kern<<<grid, 64 + 32 * EPW, smem, st>>>(a0, a1, b0, b1, p);
+  kern<<<grid, threads, smem, st>>>(a0, a1, b0, b1, p);
   return cudaGetLastError();
 }
 
@@ -681,7 +810,7 @@ cudaError_t tc_expert_up(const void* H, const void* Wg, const void* Wu, void* A,
   p.out2 = U;
   p.ld = F;
   p.bstride = (int64_t)M * F;
-  return launch<256, false, true, true, false, EPI_SWIGLU_FWD, 4>(ma, ma, mg, mu, p, st);
+  return launch<256, false, true, true, false, EPI_SWIGLU_FWD, 6, 8, true>(ma, ma, mg, mu, p, st);
 }
 
 cudaError_t tc_expert_down(const void* U, const void* Wd, void* O, int E, int M, int d, int F,
@@ -693,7 +822,7 @@ cudaError_t tc_expert_down(const void* U, const void* Wd, void* O, int E, int M,
   p.out0 = O;
   p.ld = d;
   p.bstride = (int64_t)M * d;
-  return launch<256, false, true, false, false, EPI_STORE_BF16, 4>(ma, ma, mb, mb, p, st);
+  return launch<256, false, true, false, false, EPI_STORE_BF16, 6, 8, true>(ma, ma, mb, mb, p, st);
 }
 
 cudaError_t tc_expert_dgrad_up(const void* dO, const void* Wd, const void* A, const void* B,
@@ -701,7 +830,7 @@ cudaError_t tc_expert_dgrad_up(const void* dO, const void* Wd, const void* A, co
                                cudaStream_t st) {
   CUtensorMap ma, mb;
   TC_TRY(make_map(&ma, dO, d, M, E, BM));
-  TC_TRY(make_map(&mb, Wd, d, F, E, 256));   // B[n=f][k=i] = Wd[f][i]: K-major
+  TC_TRY(make_map(&mb, Wd, d, F, E, 128));   // B[n=f][k=i] = Wd[f][i]: K-major, half per CTA
   Args p = base_args(E, M, F, d, 256, status);
   p.in0 = A;
   p.in1 = B;
@@ -709,7 +838,7 @@ cudaError_t tc_expert_dgrad_up(const void* dO, const void* Wd, const void* A, co
   p.out1 = dB;
   p.ld = F;
   p.bstride = (int64_t)M * F;
-  return launch<256, false, false, false, false, EPI_SWIGLU_BWD, 4>(ma, ma, mb, mb, p, st);
+  return launch<256, false, false, false, false, EPI_SWIGLU_BWD, 6, 8, true>(ma, ma, mb, mb, p, st);
 }
 
 cudaError_t tc_expert_dgrad_h(const void* dA, const void* dB, const void* Wg, const void* Wu,
@@ -717,14 +846,14 @@ cudaError_t tc_expert_dgrad_h(const void* dA, const void* dB, const void* Wg, co
   CUtensorMap ma0, ma1, mb0, mb1;
   TC_TRY(make_map(&ma0, dA, F, M, E, BM));
   TC_TRY(make_map(&ma1, dB, F, M, E, BM));
-  TC_TRY(make_map(&mb0, Wg, F, d, E, 256));  // B[n=i][k=f] = Wg[i][f]: K-major
-  TC_TRY(make_map(&mb1, Wu, F, d, E, 256));
+  TC_TRY(make_map(&mb0, Wg, F, d, E, 128));  // B[n=i][k=f] = Wg[i][f]: K-major, half per CTA
+  TC_TRY(make_map(&mb1, Wu, F, d, E, 128));
   Args p = base_args(E, M, d, 2 * F, 256, status);
   p.k_blocks0 = F / BK;
   p.out0 = dH;
   p.ld = d;
   p.bstride = (int64_t)M * d;
-  return launch<256, false, false, false, true, EPI_STORE_BF16, 4>(ma0, ma1, mb0, mb1, p, st);
+  return launch<256, false, false, false, true, EPI_STORE_BF16, 6, 8, true>(ma0, ma1, mb0, mb1, p, st);
 }
 
 cudaError_t tc_expert_wgrad(const void* H, const void* U, const void* dO, const void* dA,
@@ -739,7 +868,7 @@ cudaError_t tc_expert_wgrad(const void* H, const void* U, const void* dO, const 
     p.out0 = dWd;
     p.ld = d;
     p.bstride = (int64_t)F * d;
-    TC_TRY((launch<256, true, true, false, false, EPI_STORE_F32, 4>(ma, ma, mb, mb, p, st)));
+    TC_TRY((launch<256, true, true, false, false, EPI_STORE_F32, 6, 8, true>(ma, ma, mb, mb, p, st)));
   }
   {
     // [dWg | dWu][e] [d][F] = H[e]^T . [dA | dB][e]
@@ -752,7 +881,8 @@ cudaError_t tc_expert_wgrad(const void* H, const void* U, const void* dO, const 
     p.out1 = dWu;
     p.ld = F;
     p.bstride = (int64_t)d * F;
-    TC_TRY((launch<256, true, true, true, false, EPI_STORE_F32_SPLIT, 4>(ma, ma, mb0, mb1, p, st)));
+    TC_TRY((launch<256, true, true, true, false, EPI_STORE_F32_SPLIT, 6, 8, true>(ma, ma, mb0, mb1, p,
+                                                                                  st)));
   }
   return cudaSuccess;
 }
