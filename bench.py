@@ -210,29 +210,54 @@ def run_ours(args):
         return torch.from_numpy(t.data).to(device)
 
     X, dY = to_dev(inp.X), to_dev(inp.dY)
-    Wr, Wg, Wu, Wd = to_dev(Ld.Wr), to_dev(Ld.Wg), to_dev(Ld.Wu), to_dev(Ld.Wd)
-    br = None if Ld.br is None else torch.from_numpy(Ld.br).to(device)
-    lay = ECMoELayer(w.N, w.d, w.E, w.d_ff, inp.group_off, inp.k_g, dtype=w.dtype, device=device)
-    Y = torch.empty_like(X)
-    grads = {"dX": torch.empty_like(X),
+    stack = []          # one context per layer; several layers stack with residual adds
+    for Ld in inp.layers:
+        wts = (to_dev(Ld.Wr), None if Ld.br is None else torch.from_numpy(Ld.br).to(device),
+               to_dev(Ld.Wg), to_dev(Ld.Wu), to_dev(Ld.Wd))
+        lay_l = ECMoELayer(w.N, w.d, w.E, w.d_ff, inp.group_off, inp.k_g, dtype=w.dtype,
+                           device=device)
+        if w.layers > 1:
+            lay_l.set_residual(True)
+        g = {"dX": torch.empty_like(X),
              "dWr": torch.empty(w.d, w.E, dtype=torch.float32, device=device),
-             "dbr": None if br is None else torch.empty(w.E, dtype=torch.float32, device=device),
+             "dbr": None if Ld.br is None else torch.empty(w.E, dtype=torch.float32,
+                                                           device=device),
              "dWg": torch.empty(w.E, w.d, w.d_ff, dtype=torch.float32, device=device),
              "dWu": torch.empty(w.E, w.d, w.d_ff, dtype=torch.float32, device=device),
              "dWd": torch.empty(w.E, w.d_ff, w.d, dtype=torch.float32, device=device)}
+        stack.append((lay_l, wts, [torch.empty_like(X)], g))
+    lay, (Wr, br, Wg, Wu, Wd) = stack[0][0], stack[0][1]
+    Y = stack[-1][2][0]
+    grads = stack[0][3]
     stream = torch.cuda.current_stream(device)
 
+    def run_stack(x, dy, y_last, dx_first, st=None):
+        """Forward through every layer, then backward in reverse; returns nothing."""
+        h = x
+        for i, (l_, wts, ybuf, g) in enumerate(stack):
+            out = y_last if i == len(stack) - 1 else ybuf[0]
+            l_.forward(h, *wts, Y=out, outputs=False, stream=st)
+            h = out
+        d = dy
+        for i in range(len(stack) - 1, -1, -1):
+            l_, wts, ybuf, g = stack[i]
+            gi = dict(g)
+            if i == 0:
+                gi["dX"] = dx_first
+            l_.backward(d, grads=gi, stream=st)
+            d = gi["dX"]
+
     def step(x=X, dy=dY, y=Y, g=grads):
-        lay.forward(x, Wr, br, Wg, Wu, Wd, Y=y, outputs=False)
-        lay.backward(dy, grads=g)
+        run_stack(x, dy, y, g["dX"])
 
     for _ in range(args.warmup):
         step()
     lay.check()
 
     # ---- device-timed steps (inputs resident), per-kernel events on the same stream
-    lay.set_profiling(True)
-    launches0 = lay.launches
+    for l_ in stack:
+        l_[0].set_profiling(True)
+    launches0 = sum(l_[0].launches for l_ in stack)
     clocks = Clocks(local)
     clocks.start()
     time.sleep(0.5)       # let the sampler come up before the timed region
@@ -249,10 +274,11 @@ def run_ours(args):
     clocks.mark_end()
     _barrier(ws)
     clk = clocks.stop()
-    launches = lay.launches - launches0
-    phases = lay.profile()
-    lay.set_profiling(False)
-    lay.check()
+    launches = sum(l_[0].launches for l_ in stack) - launches0
+    phases = [ph for l_ in stack for ph in l_[0].profile()]
+    for l_ in stack:
+        l_[0].set_profiling(False)
+        l_[0].check()
     ms = e0.elapsed_time(e1) / args.steps
     ms_max = _max_over_ranks(ms, ws, device)
 
@@ -294,8 +320,7 @@ def run_ours(args):
         stream.wait_event(in_ready[b])
         if i >= 2:
             stream.wait_event(copied_out[b])         # Ye[b], dX[b] of step i-2 copied out
-        lay.forward(Xe[b], Wr, br, Wg, Wu, Wd, Y=Ye[b], outputs=False, stream=stream)
-        lay.backward(dYe[b], grads=ge[b], stream=stream)
+        run_stack(Xe[b], dYe[b], Ye[b], ge[b]["dX"], st=stream)
         computed[b].record(stream)
         with torch.cuda.stream(s_out):
             s_out.wait_event(computed[b])
@@ -306,7 +331,8 @@ def run_ours(args):
     t1.record(s_out)
     torch.cuda.synchronize(device)
     e2e_ms = _max_over_ranks(t0.elapsed_time(t1) / e_steps, ws, device)
-    lay.check()
+    for l_ in stack:
+        l_[0].check()
 
     # ---- roofline of the dominant kernel (the tcgen05 grouped GEMM)
     hbm, bf16_burst, bf16_sust, peak_src = _peaks()
@@ -317,7 +343,7 @@ def run_ours(args):
     gemm_launches = sum(len(v) for v in gemm.values()) + len(per.get("gemm_wgrad", []))
     gemm_ms_step = sum(sum(v) for v in gemm.values()) / args.steps
     P = w.E * int(inp.k_g.sum())
-    flops_step = 18.0 * P * w.d * w.d_ff
+    flops_step = 18.0 * P * w.d * w.d_ff * w.layers
     gemm_tflops = flops_step / (gemm_ms_step * 1e-3) / 1e12
     gemm_per_launch = flops_step / max(1, gemm_launches / args.steps)
     b = 2 if w.dtype == "bf16" else 4
@@ -333,7 +359,8 @@ def run_ours(args):
     }
     mem_bytes = {k: v for k, v in mem_bytes.items() if k in per}   # kernels this path launches
     mem_ms = sum(sum(per[k]) for k in mem_bytes) / args.steps
-    mem_gbs = sum(mem_bytes.values()) / (mem_ms * 1e-3) / 1e9 if mem_ms > 0 else None
+    mem_gbs = (w.layers * sum(mem_bytes.values()) / (mem_ms * 1e-3) / 1e9 if mem_ms > 0
+               else None)
     src = os.path.join(ROOT, "paper_2604_01622_gb300", "csrc", "gemm_tc.cu")
     tr = TRAFFIC.get(_src_hash(src))
     roofline = {
@@ -351,6 +378,7 @@ def run_ours(args):
         "scaling": "weak", "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
         "config": {"workload": w.name, "sequences": w.G, "seq_len": w.L, "tokens": w.N,
                    "d_model": w.d, "experts": w.E, "d_ff": w.d_ff, "k_per_seq": w.k_base,
+                   "layers": w.layers,
                    "parallelism": f"replicas{ws}" if ws > 1 else "single",
                    "l2": "inputs and activations larger than L2 (no flush)"},
     }

@@ -78,6 +78,12 @@ void ec_ctx_destroy(ec_ctx* ctx);
  * Invalidates saved forward state. */
 ec_status ec_ctx_set_capacity(ec_ctx* ctx, const int32_t* k_g);
 
+/* Residual form for stacked layers x_{l+1} = x_l + EC(x_l) (off by default): with it on,
+ * ec_moe_forward writes Y = X + EC(X) and ec_moe_backward writes dX = dY + (the input
+ * gradient of EC), both fused into the combine and scatter kernels. Tokens no expert
+ * picks then get Y_t = X_t. Invalidates saved forward state. */
+ec_status ec_ctx_set_residual(ec_ctx* ctx, int32_t on);
+
 /* Current rows per expert M = sum k_g. */
 int64_t ec_rows_per_expert(const ec_ctx* ctx);
 
@@ -131,6 +137,13 @@ int32_t ec_ctx_profile(ec_ctx* ctx, const char** names, float* ms, int32_t cap);
 
 /* Number of CUDA kernels the library has launched through this context so far. */
 int64_t ec_kernel_launches(const ec_ctx* ctx);
+
+/* Failure-path self-test (no counterpart in the paper): launches one kernel that waits on
+ * an mbarrier that nothing completes, with the same bounded wait the tensor-core kernels
+ * use but a limit of limit_ns nanoseconds (at most 10 s). The kernel gives up, records the
+ * timeout in the context's device status word and returns, so the context stays usable;
+ * ec_check_device then reports EC_ERR_TIMEOUT once. Asynchronous on `stream`. */
+ec_status ec_selftest_bounded_wait(ec_ctx* ctx, uint64_t limit_ns, void* stream);
 
 /* Expert-choice selection for callers that cannot allocate device memory (the paper has no
  * counterpart: this is a deployment variant of the selection in ec_route).

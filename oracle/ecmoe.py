@@ -279,3 +279,32 @@ def backward_expert(H, S_col, dY_rows, Wg_e, Wu_e, Wd_e):
     dA = dU * b * silu_grad(a)
     dB = dU * silu(a)
     return H.T @ dA, H.T @ dB, u.T @ dO, dgate
+
+
+# ----------------------------------------------------------------------------
+# Stacked layers with residual adds, x_{l+1} = x_l + EC_l(x_l): how the four-layer
+# wide workload composes the layer (the transformer residual stream around each MoE
+# layer). A composition of `forward`/`backward` above, nothing more.
+# ----------------------------------------------------------------------------
+def stack_forward(X, layers, group_off, k_g, forced_idx=None):
+    """layers: list of (Wr, br, Wg, Wu, Wd). Returns (xs, fwds) with xs[l+1] = xs[l] + Y_l."""
+    xs = [np.asarray(X, np.float64)]
+    fwds = []
+    for l, (Wr, br, Wg, Wu, Wd) in enumerate(layers):
+        f = forward(xs[-1], Wr, br, Wg, Wu, Wd, group_off, k_g,
+                    None if forced_idx is None else forced_idx[l])
+        fwds.append(f)
+        xs.append(xs[-1] + f["Y"])
+    return xs, fwds
+
+
+def stack_backward(fwds, layers, dOut):
+    """Gradients of <dOut, x_L>: returns (dX_0, per-layer gradient dicts)."""
+    d = np.asarray(dOut, np.float64)
+    grads = [None] * len(layers)
+    for l in range(len(layers) - 1, -1, -1):
+        Wr, br, Wg, Wu, Wd = layers[l]
+        g = backward(fwds[l], d, Wr, Wg, Wu, Wd)
+        grads[l] = g
+        d = d + g["dX"]
+    return d, grads

@@ -26,6 +26,7 @@ EXPORTS = (
     "ec_workspace_bytes", "ec_ctx_set_workspace", "ec_route", "ec_moe_forward",
     "ec_moe_backward", "ec_check_device", "ec_last_error", "ec_status_string",
     "ec_ctx_set_profiling", "ec_ctx_profile", "ec_kernel_launches", "ec_select_static",
+    "ec_selftest_bounded_wait", "ec_ctx_set_residual",
 )
 
 _lib = None
@@ -66,6 +67,8 @@ def load():
                                  ctypes.POINTER(ctypes.c_float), i32]),
         "ec_kernel_launches": (i64, [vp]),
         "ec_select_static": (i32, [vp, i32, i32, i32, P32, P32, vp, vp, vp]),
+        "ec_selftest_bounded_wait": (i32, [vp, ctypes.c_uint64, vp]),
+        "ec_ctx_set_residual": (i32, [vp, i32]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -108,6 +111,10 @@ def ec_ctx_destroy(ctx):
 def ec_ctx_set_capacity(ctx, k_g):
     k_arr, k_ptr = _i32(k_g)
     _check(ctx, load().ec_ctx_set_capacity(ctx, k_ptr))
+
+
+def ec_ctx_set_residual(ctx, on: bool):
+    _check(ctx, load().ec_ctx_set_residual(ctx, 1 if on else 0))
 
 
 def ec_rows_per_expert(ctx) -> int:
@@ -163,6 +170,10 @@ def ec_select_static(S, N, E, group_off, k_g, idx, gate, stream):
     st = load().ec_select_static(S, N, E, len(g_arr) - 1, g_ptr, k_ptr, idx, gate, stream)
     if st != EC_OK:
         raise ECError(st, "ec_select_static rejected the call")
+
+
+def ec_selftest_bounded_wait(ctx, limit_ns: int, stream):
+    _check(ctx, load().ec_selftest_bounded_wait(ctx, int(limit_ns), stream))
 
 
 def ec_last_error(ctx) -> str:

@@ -32,6 +32,7 @@ struct ec_ctx {
   int ev_n = 0;
   int64_t launches = 0;
   // state saved by the forward pass
+  bool residual = false;   // Y = X + EC(X), dX = dY + EC input gradient
   bool have_fwd = false;
   const void *X = nullptr, *Wr = nullptr, *Wg = nullptr, *Wu = nullptr, *Wd = nullptr;
   const float* br = nullptr;
@@ -289,6 +290,7 @@ ec_status run_forward(ec_ctx* c, const void* X, const void* Wg, const void* Wu, 
   }
   EC_KERNEL("combine", N > 0,
             launch_combine<T>(O, at<float>(c, c->o_gate), at<int>(c, c->o_slot),
+                              c->residual ? static_cast<const T*>(X) : nullptr,
                               static_cast<T*>(Y), N, E, M, d, st));
   return EC_OK;
 }
@@ -361,6 +363,7 @@ ec_status run_backward(ec_ctx* c, const void* dY, void* dX, float* dWr, float* d
   // router: dZ = S (dS - <dS,S>), dX = dZ Wr^T + sum dH, dWr = X^T dZ, dbr = sum dZ
   float* dXr = at<float>(c, c->o_dXr);
   float* part = at<float>(c, c->o_part);
+  const T* res = c->residual ? static_cast<const T*>(dY) : nullptr;
   if (use_tc(c)) {
     bf16* dZb = at<bf16>(c, c->o_dZb);
     EC_KERNEL("softmax_bwd", nz,
@@ -368,7 +371,7 @@ ec_status run_backward(ec_ctx* c, const void* dY, void* dX, float* dWr, float* d
     EC_KERNEL("router_dgrad_gemm", nz,
               tc_router_dgrad(dZb, at<void>(c, c->o_wrpad), dXr, N, d, c->Ep, status, st));
     EC_KERNEL("dx_combine", nz,
-              launch_dx_combine<T>(dH, slot, dXr, static_cast<T*>(dX), N, E, M, d, st));
+              launch_dx_combine<T>(dH, slot, dXr, res, static_cast<T*>(dX), N, E, M, d, st));
     EC_KERNEL("router_wgrad_gemm", nz,
               tc_router_wgrad(c->X, dZb, part, N, d, c->Ep, c->wr_splits, status, st));
     EC_KERNEL("router_wgrad_reduce", 1,
@@ -380,7 +383,7 @@ ec_status run_backward(ec_ctx* c, const void* dY, void* dX, float* dWr, float* d
               launch_simt_gemm(sg(dZ, 0, E, 1, c->Wr, 0, 1, E, dXr, 0, d, N, d, E, 1), EType::F32,
                                et(c), st));
     EC_KERNEL("dx_combine", nz,
-              launch_dx_combine<T>(dH, slot, dXr, static_cast<T*>(dX), N, E, M, d, st));
+              launch_dx_combine<T>(dH, slot, dXr, res, static_cast<T*>(dX), N, E, M, d, st));
     SimtGemmArgs a = sg(c->X, 0, 1, d, dZ, 0, E, 1, part, 0, E, d, E, N, 1);
     a.splits = c->wr_splits;
     a.c_split = (int64_t)d * E;
@@ -521,6 +524,13 @@ ec_status ec_moe_backward(ec_ctx* c, const void* dY, void* dX, float* dWr, float
   return EC_OK;
 }
 
+ec_status ec_ctx_set_residual(ec_ctx* c, int32_t on) {
+  if (!c) return EC_ERR_INVALID_ARG;
+  c->residual = on != 0;
+  c->have_fwd = false;
+  return EC_OK;
+}
+
 ec_status ec_ctx_set_profiling(ec_ctx* c, int32_t on) {
   if (!c) return EC_ERR_INVALID_ARG;
   c->prof = on != 0;
@@ -546,6 +556,15 @@ int32_t ec_ctx_profile(ec_ctx* c, const char** names, float* ms, int32_t cap) {
 }
 
 int64_t ec_kernel_launches(const ec_ctx* c) { return c ? c->launches : -1; }
+
+ec_status ec_selftest_bounded_wait(ec_ctx* c, uint64_t limit_ns, void* stream) {
+  ec_status s = check_ready(c);
+  if (s != EC_OK) return s;
+  if (limit_ns > 10000000000ull) return fail(c, EC_ERR_INVALID_ARG, "limit above 10 s");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  EC_KERNEL("wait_probe", 1, tc_wait_probe(at<int>(c, c->o_status), limit_ns, st));
+  return EC_OK;
+}
 
 ec_status ec_check_device(ec_ctx* c, void* stream) {
   ec_status s = check_ready(c);

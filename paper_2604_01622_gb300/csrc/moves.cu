@@ -66,8 +66,8 @@ __device__ __forceinline__ int token_pairs(const int* __restrict__ slot, const f
 // ------------------------------------------------------------------ combine Y_t = sum g * O
 template <typename T>
 __global__ void combine_kernel(const T* __restrict__ O, const float* __restrict__ gate,
-                               const int* __restrict__ slot, T* __restrict__ Y, int N, int E, int M,
-                               int d) {
+                               const int* __restrict__ slot, const T* __restrict__ R,
+                               T* __restrict__ Y, int N, int E, int M, int d) {
   extern __shared__ int sh[];
   int* s_e = sh;
   int* s_m = sh + E;
@@ -79,8 +79,12 @@ __global__ void combine_kernel(const T* __restrict__ O, const float* __restrict_
   const int nv = d / VN;
   for (int v = threadIdx.x; v < nv; v += blockDim.x) {
     float acc[VN];
+    if (R) {
+      unpack16(__ldg(reinterpret_cast<const uint4*>(R + (size_t)t * d) + v), acc, T());
+    } else {
 #pragma unroll
-    for (int j = 0; j < VN; ++j) acc[j] = 0.f;
+      for (int j = 0; j < VN; ++j) acc[j] = 0.f;
+    }
     for (int p = 0; p < cnt; ++p) {
       const size_t row = (size_t)s_e[p] * M + s_m[p];
       const uint4 u = __ldg(reinterpret_cast<const uint4*>(O + row * d) + v);
@@ -95,11 +99,11 @@ __global__ void combine_kernel(const T* __restrict__ O, const float* __restrict_
 }
 
 template <typename T>
-cudaError_t launch_combine(const T* O, const float* gate, const int* slot, T* Y, int N, int E,
-                           int M, int d, cudaStream_t st) {
+cudaError_t launch_combine(const T* O, const float* gate, const int* slot, const T* R, T* Y, int N,
+                           int E, int M, int d, cudaStream_t st) {
   if (N == 0) return cudaSuccess;
   const size_t smem = (size_t)3 * E * sizeof(int);
-  combine_kernel<T><<<N, 128, smem, st>>>(O, gate, slot, Y, N, E, M, d);
+  combine_kernel<T><<<N, 128, smem, st>>>(O, gate, slot, R, Y, N, E, M, d);
   return cudaGetLastError();
 }
 
@@ -214,8 +218,8 @@ cudaError_t launch_reduce_partials(const float* part, float* out, int rows, int 
 // ------------------------------------------------------------------ dX_t = dXr_t + sum dH rows
 template <typename T>
 __global__ void dx_combine_kernel(const T* __restrict__ dH, const int* __restrict__ slot,
-                                  const float* __restrict__ dXr, T* __restrict__ dX, int N, int E,
-                                  int M, int d) {
+                                  const float* __restrict__ dXr, const T* __restrict__ R,
+                                  T* __restrict__ dX, int N, int E, int M, int d) {
   extern __shared__ int sh[];
   int* s_e = sh;
   int* s_m = sh + E;
@@ -237,6 +241,12 @@ __global__ void dx_combine_kernel(const T* __restrict__ dH, const int* __restric
 #pragma unroll
       for (int j = 0; j < VN; ++j) acc[j] = 0.f;
     }
+    if (R) {
+      float r[VN];
+      unpack16(__ldg(reinterpret_cast<const uint4*>(R + (size_t)t * d) + v), r, T());
+#pragma unroll
+      for (int j = 0; j < VN; ++j) acc[j] += r[j];
+    }
     for (int p = 0; p < cnt; ++p) {
       const size_t row = (size_t)s_e[p] * M + s_m[p];
       float h[VN];
@@ -249,11 +259,11 @@ __global__ void dx_combine_kernel(const T* __restrict__ dH, const int* __restric
 }
 
 template <typename T>
-cudaError_t launch_dx_combine(const T* dH, const int* slot, const float* dXr, T* dX, int N, int E,
-                              int M, int d, cudaStream_t st) {
+cudaError_t launch_dx_combine(const T* dH, const int* slot, const float* dXr, const T* R, T* dX,
+                              int N, int E, int M, int d, cudaStream_t st) {
   if (N == 0) return cudaSuccess;
   const size_t smem = (size_t)2 * E * sizeof(int);
-  dx_combine_kernel<T><<<N, 128, smem, st>>>(dH, slot, dXr, dX, N, E, M, d);
+  dx_combine_kernel<T><<<N, 128, smem, st>>>(dH, slot, dXr, R, dX, N, E, M, d);
   return cudaGetLastError();
 }
 
@@ -359,12 +369,12 @@ cudaError_t launch_reduce_splits(const float* part, float* out, int64_t n, int s
 
 #define ECMOE_INST(T)                                                                            \
   template cudaError_t launch_gather<T>(const T*, const int*, T*, int64_t, int, cudaStream_t);    \
-  template cudaError_t launch_combine<T>(const T*, const float*, const int*, T*, int, int, int,   \
-                                         int, cudaStream_t);                                      \
+  template cudaError_t launch_combine<T>(const T*, const float*, const int*, const T*, T*, int,   \
+                                         int, int, int, cudaStream_t);                            \
   template cudaError_t launch_bwd_gather_scale<T>(const T*, const T*, const int*, const float*,   \
                                                   T*, float*, int64_t, int, cudaStream_t);        \
-  template cudaError_t launch_dx_combine<T>(const T*, const int*, const float*, T*, int, int,     \
-                                            int, int, cudaStream_t);                              \
+  template cudaError_t launch_dx_combine<T>(const T*, const int*, const float*, const T*, T*, int, \
+                                            int, int, int, cudaStream_t);                         \
   template cudaError_t launch_swiglu_fwd_ew<T>(const float*, const float*, T*, T*, T*, int64_t,   \
                                                cudaStream_t);                                     \
   template cudaError_t launch_swiglu_bwd_ew<T>(const float*, const T*, const T*, T*, T*,          \

@@ -8,7 +8,8 @@ from __future__ import annotations
 import torch
 
 from . import (EC_BF16, EC_F32, ec_check_device, ec_ctx_create, ec_ctx_destroy,
-               ec_ctx_profile, ec_ctx_set_capacity, ec_ctx_set_profiling, ec_ctx_set_workspace,
+               ec_ctx_profile, ec_ctx_set_capacity, ec_ctx_set_profiling, ec_ctx_set_residual,
+               ec_ctx_set_workspace,
                ec_kernel_launches, ec_moe_backward, ec_moe_forward, ec_route,
                ec_rows_per_expert, ec_workspace_bytes)
 
@@ -43,6 +44,10 @@ class ECMoELayer:
 
     def set_capacity(self, k_g):
         ec_ctx_set_capacity(self.ctx, k_g)
+
+    def set_residual(self, on: bool):
+        """Y = X + EC(X) and dX = dY + EC input gradient (stacked layers)."""
+        ec_ctx_set_residual(self.ctx, on)
 
     def _empty(self, *shape, dtype=None):
         return torch.empty(*shape, dtype=dtype or self.tdtype, device=self.device)

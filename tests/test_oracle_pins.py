@@ -272,3 +272,30 @@ def test_sampled_forms_match_full_layer():
         np.testing.assert_allclose(dwu, g["dWu"][e], rtol=1e-11, atol=1e-12)
         np.testing.assert_allclose(dwd, g["dWd"][e], rtol=1e-11, atol=1e-12)
         np.testing.assert_allclose(dgate, g["dgate"][e], rtol=1e-11, atol=1e-12)
+
+
+def test_residual_stack_backward_matches_finite_differences():
+    rng = np.random.default_rng(21)
+    X, *_rest, groups, k = _tiny(22, N=30, d=6, E=3, d_ff=5, groups=(0, 14, 30), k=(4, 6))
+    layers = []
+    for l in range(2):
+        _, Wr, br, Wg, Wu, Wd, _, _ = _tiny(30 + l, N=30, d=6, E=3, d_ff=5, groups=(0, 14, 30))
+        layers.append((Wr, br, Wg, Wu, Wd))
+    dOut = rng.standard_normal(X.shape)
+    xs, fwds = O.stack_forward(X, layers, groups, k)
+    # one layer of the stack is the layer plus its input
+    f0 = O.forward(X, *layers[0], groups, k)
+    np.testing.assert_allclose(xs[1], X + f0["Y"], rtol=0, atol=0)
+    dX, _ = O.stack_backward(fwds, layers, dOut)
+    idx_ref = [f["idx"] for f in fwds]
+    h = 1e-6
+    for _ in range(4):
+        V = rng.standard_normal(X.shape)
+        xp, fp = O.stack_forward(X + h * V, layers, groups, k)
+        xm, fm = O.stack_forward(X - h * V, layers, groups, k)
+        if not all(np.array_equal(a["idx"], b) and np.array_equal(c["idx"], b)
+                   for a, c, b in zip(fp, fm, idx_ref)):
+            continue
+        fd = (np.sum(dOut * xp[-1]) - np.sum(dOut * xm[-1])) / (2 * h)
+        an = float(np.sum(dX * V))
+        assert abs(fd - an) <= 1e-6 * max(1.0, abs(an))
