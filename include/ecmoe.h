@@ -138,6 +138,32 @@ int32_t ec_ctx_profile(ec_ctx* ctx, const char** names, float* ms, int32_t cap);
 /* Number of CUDA kernels the library has launched through this context so far. */
 int64_t ec_kernel_launches(const ec_ctx* ctx);
 
+/* Capacity schedulers (Sec. 4.2, Table 1): masking ratio r -> top-k equivalent
+ *   k(r) = clamp(k_min + (k_max - k_min) s(r), k_min, k_max) with
+ *   s = 1/2 (static), r, 1 - r, (1 - cos pi r)/2, (1 + cos pi r)/2, g~(r), 1 - g~(r), where
+ *   g~(r) = (g(r) - g(0)) / (1 - g(0)), g(r) = exp(-(r - 1/2)^2 / (2 sigma^2)) (appendix
+ *   "Scheduler Definitions and FLOPs Equivalence"; the paper uses sigma = 0.22). */
+typedef enum {
+  EC_SCHED_STATIC = 0,
+  EC_SCHED_LINEAR = 1,
+  EC_SCHED_LINEAR_REV = 2,
+  EC_SCHED_COSINE = 3,
+  EC_SCHED_COSINE_REV = 4,
+  EC_SCHED_GAUSSIAN = 5,
+  EC_SCHED_GAUSSIAN_REV = 6
+} ec_scheduler;
+
+/* Per-sequence capacities for one step (host only, no GPU needed): group g has masking ratio
+ * r[g] in [0, 1] and L_g = group_off[g+1] - group_off[g] tokens; expert capacity
+ * k_g[g] = floor(k(r[g]) * L_g / E + 1/2) clipped to [0, L_g] (Sec. 2.2: c = k N / E per
+ * selection pool). Host arrays: group_off [G+1], r [G], k_g [G] (written). sigma is used by
+ * the Gaussian schedulers only. EC_ERR_INVALID_ARG on an unknown scheduler, r outside
+ * [0, 1], k_min < 0 or k_max < k_min; EC_ERR_SHAPE on bad sizes. The result feeds
+ * ec_ctx_set_capacity (whose sum(k_g) limit is the caller's to respect). */
+ec_status ec_capacity_schedule(int32_t scheduler, double k_min, double k_max, double sigma,
+                               int32_t E, int32_t G, const int32_t* group_off, const double* r,
+                               int32_t* k_g);
+
 /* Failure-path self-test (no counterpart in the paper): launches one kernel that waits on
  * an mbarrier that nothing completes, with the same bounded wait the tensor-core kernels
  * use but a limit of limit_ns nanoseconds (at most 10 s). The kernel gives up, records the

@@ -26,8 +26,11 @@ EXPORTS = (
     "ec_workspace_bytes", "ec_ctx_set_workspace", "ec_route", "ec_moe_forward",
     "ec_moe_backward", "ec_check_device", "ec_last_error", "ec_status_string",
     "ec_ctx_set_profiling", "ec_ctx_profile", "ec_kernel_launches", "ec_select_static",
-    "ec_selftest_bounded_wait", "ec_ctx_set_residual",
+    "ec_selftest_bounded_wait", "ec_ctx_set_residual", "ec_capacity_schedule",
 )
+
+EC_SCHEDULERS = {"static": 0, "linear": 1, "linear_reverse": 2, "cosine": 3,
+                 "cosine_reverse": 4, "gaussian": 5, "gaussian_reverse": 6}
 
 _lib = None
 
@@ -69,6 +72,8 @@ def load():
         "ec_select_static": (i32, [vp, i32, i32, i32, P32, P32, vp, vp, vp]),
         "ec_selftest_bounded_wait": (i32, [vp, ctypes.c_uint64, vp]),
         "ec_ctx_set_residual": (i32, [vp, i32]),
+        "ec_capacity_schedule": (i32, [i32, ctypes.c_double, ctypes.c_double, ctypes.c_double,
+                                       i32, i32, P32, ctypes.POINTER(ctypes.c_double), P32]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -174,6 +179,23 @@ def ec_select_static(S, N, E, group_off, k_g, idx, gate, stream):
 
 def ec_selftest_bounded_wait(ctx, limit_ns: int, stream):
     _check(ctx, load().ec_selftest_bounded_wait(ctx, int(limit_ns), stream))
+
+
+def ec_capacity_schedule(scheduler, k_min, k_max, E, group_off, r, sigma=0.22):
+    """Per-group capacities k_g for masking ratios r (host computation in the library)."""
+    g_arr, g_ptr = _i32(group_off)
+    r_arr = np.ascontiguousarray(np.asarray(r, dtype=np.float64))
+    G = len(g_arr) - 1
+    if len(r_arr) != G:
+        raise ValueError("one masking ratio per group")
+    out = np.zeros(G, dtype=np.int32)
+    code = EC_SCHEDULERS[scheduler] if isinstance(scheduler, str) else int(scheduler)
+    st = load().ec_capacity_schedule(code, float(k_min), float(k_max), float(sigma), int(E), G,
+                                     g_ptr, r_arr.ctypes.data_as(ctypes.POINTER(ctypes.c_double)),
+                                     out.ctypes.data_as(ctypes.POINTER(ctypes.c_int32)))
+    if st != EC_OK:
+        raise ECError(st, "ec_capacity_schedule rejected its arguments")
+    return out
 
 
 def ec_last_error(ctx) -> str:

@@ -16,7 +16,7 @@ CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libecmoe.so")
 SOURCES = ["ecmoe_api.cu", "route.cu", "moves.cu", "gemm_simt.cu", "gemm_tc.cu",
-           "select_static.cu"]
+           "select_static.cu", "capacity.cpp"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr"]
 
@@ -45,7 +45,7 @@ def build(verbose: bool = False, extra_flags: list[str] | None = None) -> str:
     jobs = []
     for src in SOURCES:
         s = os.path.join(CSRC, src)
-        o = os.path.join(BUILD, src.replace(".cu", ".o"))
+        o = os.path.join(BUILD, os.path.splitext(src)[0] + ".o")
         if _stale(o, s) or extra_flags:
             jobs.append([nvcc, *ARCH, *flags, "-c", s, "-o", o])
 
@@ -58,7 +58,7 @@ def build(verbose: bool = False, extra_flags: list[str] | None = None) -> str:
 
     with cf.ThreadPoolExecutor(max_workers=len(SOURCES)) as ex:
         list(ex.map(run, jobs))
-    objs = [os.path.join(BUILD, s.replace(".cu", ".o")) for s in SOURCES]
+    objs = [os.path.join(BUILD, os.path.splitext(s)[0] + ".o") for s in SOURCES]
     if jobs or not os.path.exists(LIB):
         run([nvcc, *ARCH, "-shared", "-cudart", "static", "-o", LIB, *objs])
     return LIB
