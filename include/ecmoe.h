@@ -121,6 +121,25 @@ ec_status ec_moe_forward(ec_ctx* ctx, const void* X, const void* Wr, const float
 ec_status ec_moe_backward(ec_ctx* ctx, const void* dY, void* dX, float* dWr, float* dbr,
                           float* dWg, float* dWu, float* dWd, void* stream);
 
+/* Shared experts (the paper's MoE block also has shared experts that process every token,
+ * appendix "Token Coverage"; 2 per layer in its models, appendix "Experimental Setup").
+ * S shared SwiGLU experts of width f each sum to one SwiGLU FFN of width d_ff_shared = S*f:
+ * their weights are passed concatenated, Wg_s, Wu_s [d][d_ff_shared] (expert s in columns
+ * s*f .. s*f+f-1) and Wd_s [d_ff_shared][d] (its rows), and their gradients come back in the
+ * same layouts (float32). ec_ctx_set_shared must be called before ec_ctx_set_workspace
+ * (it changes ec_workspace_bytes); 0 removes them. On the bf16 path d_ff_shared must be a
+ * multiple of 64. With shared experts configured the layer is
+ *   Y = FFN_shared(X) + [routed expert-choice output as in ec_moe_forward] (+ X if residual)
+ * and ec_moe_forward / ec_moe_backward return EC_ERR_STATE: use the _shared calls. */
+ec_status ec_ctx_set_shared(ec_ctx* ctx, int32_t d_ff_shared);
+ec_status ec_moe_forward_shared(ec_ctx* ctx, const void* X, const void* Wr, const float* br,
+                                const void* Wg, const void* Wu, const void* Wd, const void* Wg_s,
+                                const void* Wu_s, const void* Wd_s, void* Y, int32_t* idx,
+                                float* gate, float* S_out, void* stream);
+ec_status ec_moe_backward_shared(ec_ctx* ctx, const void* dY, void* dX, float* dWr, float* dbr,
+                                 float* dWg, float* dWu, float* dWd, float* dWg_s, float* dWu_s,
+                                 float* dWd_s, void* stream);
+
 /* Synchronise `stream`, read and clear the device status word. Returns EC_ERR_TIMEOUT if a
  * kernel gave up on a bounded wait since the last check, EC_ERR_CUDA on a CUDA error. */
 ec_status ec_check_device(ec_ctx* ctx, void* stream);

@@ -120,12 +120,14 @@ def swiglu_ffn(h, Wg, Wu, Wd):
 # ----------------------------------------------------------------------------
 # Layer forward: Sec. 2.2 y_i = sum_{j: i in T_j} g_ij FFN_j(x_i)
 # ----------------------------------------------------------------------------
-def forward(X, Wr, br, Wg, Wu, Wd, group_off, k_g, forced_idx=None):
+def forward(X, Wr, br, Wg, Wu, Wd, group_off, k_g, forced_idx=None, shared=None):
     """Whole-layer forward.
 
     X [N][d]; Wr [d][E]; br [E] or None; Wg, Wu [E][d][d_ff]; Wd [E][d_ff][d].
     forced_idx [E][M] replaces the selection (used when the scores being ranked
     are another implementation's, after the selection itself was compared).
+    shared: optional list of (Wg_s, Wu_s, Wd_s), one SwiGLU expert each that every
+    token passes through (appendix "Token Coverage"); their outputs add to Y.
     Returns a dict holding S, idx, gate, Y and what the backward pass needs.
     """
     X = np.asarray(X, np.float64)
@@ -145,8 +147,14 @@ def forward(X, Wr, br, Wg, Wu, Wd, group_off, k_g, forced_idx=None):
         per_expert.append((h, a, b, u, o))
         for m in range(idx.shape[1]):                  # scatter-add, experts in ascending order
             Y[idx[e, m]] += gate[e, m] * o[m]
+    shared_cache = []
+    for (Wg_s, Wu_s, Wd_s) in (shared or []):         # shared experts: every token, no gate
+        a, b, u, o = swiglu_ffn(X, Wg_s, Wu_s, Wd_s)
+        shared_cache.append((a, b, u))
+        Y += o
     return {"S": S, "idx": idx, "gate": gate, "Y": Y, "per_expert": per_expert,
-            "X": X, "group_off": np.asarray(group_off), "k_g": np.asarray(k_g)}
+            "X": X, "group_off": np.asarray(group_off), "k_g": np.asarray(k_g),
+            "shared": list(shared or []), "shared_cache": shared_cache}
 
 
 def drop_ratio(idx, N):
@@ -201,8 +209,15 @@ def backward(fwd, dY, Wr, Wg, Wu, Wd):
     dX += dZ @ Wr64.T
     dWr = X.T @ dZ
     dbr = dZ.sum(axis=0)
+    dshared = []
+    for (Wg_s, Wu_s, Wd_s), (a, b, u) in zip(fwd.get("shared", []), fwd.get("shared_cache", [])):
+        dU = dY @ np.asarray(Wd_s, np.float64).T       # the shared output enters Y ungated
+        dA = dU * b * silu_grad(a)
+        dB = dU * silu(a)
+        dX += dA @ np.asarray(Wg_s, np.float64).T + dB @ np.asarray(Wu_s, np.float64).T
+        dshared.append((X.T @ dA, X.T @ dB, u.T @ dY))
     return {"dX": dX, "dWr": dWr, "dbr": dbr, "dWg": dWg, "dWu": dWu, "dWd": dWd,
-            "dgate": dgate, "dS": dS, "dZ": dZ}
+            "dgate": dgate, "dS": dS, "dZ": dZ, "dshared": dshared}
 
 
 # ----------------------------------------------------------------------------

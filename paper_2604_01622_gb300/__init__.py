@@ -27,6 +27,7 @@ EXPORTS = (
     "ec_moe_backward", "ec_check_device", "ec_last_error", "ec_status_string",
     "ec_ctx_set_profiling", "ec_ctx_profile", "ec_kernel_launches", "ec_select_static",
     "ec_selftest_bounded_wait", "ec_ctx_set_residual", "ec_capacity_schedule",
+    "ec_ctx_set_shared", "ec_moe_forward_shared", "ec_moe_backward_shared",
 )
 
 EC_SCHEDULERS = {"static": 0, "linear": 1, "linear_reverse": 2, "cosine": 3,
@@ -72,6 +73,9 @@ def load():
         "ec_select_static": (i32, [vp, i32, i32, i32, P32, P32, vp, vp, vp]),
         "ec_selftest_bounded_wait": (i32, [vp, ctypes.c_uint64, vp]),
         "ec_ctx_set_residual": (i32, [vp, i32]),
+        "ec_ctx_set_shared": (i32, [vp, i32]),
+        "ec_moe_forward_shared": (i32, [vp] * 15),
+        "ec_moe_backward_shared": (i32, [vp] * 12),
         "ec_capacity_schedule": (i32, [i32, ctypes.c_double, ctypes.c_double, ctypes.c_double,
                                        i32, i32, P32, ctypes.POINTER(ctypes.c_double), P32]),
     }
@@ -144,6 +148,21 @@ def ec_moe_forward(ctx, X, Wr, br, Wg, Wu, Wd, Y, idx, gate, S_out, stream):
 
 def ec_moe_backward(ctx, dY, dX, dWr, dbr, dWg, dWu, dWd, stream):
     _check(ctx, load().ec_moe_backward(ctx, dY, dX, dWr, dbr, dWg, dWu, dWd, stream))
+
+
+def ec_ctx_set_shared(ctx, d_ff_shared: int):
+    _check(ctx, load().ec_ctx_set_shared(ctx, int(d_ff_shared)))
+
+
+def ec_moe_forward_shared(ctx, X, Wr, br, Wg, Wu, Wd, Wg_s, Wu_s, Wd_s, Y, idx, gate, S_out,
+                          stream):
+    _check(ctx, load().ec_moe_forward_shared(ctx, X, Wr, br, Wg, Wu, Wd, Wg_s, Wu_s, Wd_s, Y, idx,
+                                             gate, S_out, stream))
+
+
+def ec_moe_backward_shared(ctx, dY, dX, dWr, dbr, dWg, dWu, dWd, dWg_s, dWu_s, dWd_s, stream):
+    _check(ctx, load().ec_moe_backward_shared(ctx, dY, dX, dWr, dbr, dWg, dWu, dWd, dWg_s, dWu_s,
+                                              dWd_s, stream))
 
 
 def ec_check_device(ctx, stream):

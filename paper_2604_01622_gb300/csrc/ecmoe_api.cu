@@ -33,6 +33,10 @@ struct ec_ctx {
   int64_t launches = 0;
   // state saved by the forward pass
   bool residual = false;   // Y = X + EC(X), dX = dY + EC input gradient
+  int Fs = 0;              // shared experts: total hidden width (0 = none)
+  size_t o_Ash = 0, o_Bsh = 0, o_Ush = 0, o_Osh = 0, o_dAsh = 0, o_dBsh = 0;
+  const void *Wgs = nullptr, *Wus = nullptr, *Wds = nullptr;
+  float *dWgs = nullptr, *dWus = nullptr, *dWds = nullptr;
   bool have_fwd = false;
   const void *X = nullptr, *Wr = nullptr, *Wg = nullptr, *Wu = nullptr, *Wd = nullptr;
   const float* br = nullptr;
@@ -124,10 +128,19 @@ void layout(ec_ctx* c) {
   c->Ep = (c->E + 63) / 64 * 64;
   c->o_dZb = take(use_tc(c) ? 2 * N * c->Ep * 2 : 0);
   c->o_wrpad = take(d * c->Ep * 2);
+  // shared experts: one SwiGLU FFN of width Fs over all N tokens (Osh also holds its dH)
+  const size_t Fs = c->Fs;
+  c->o_Ash = take(N * Fs * es);
+  c->o_Bsh = take(N * Fs * es);
+  c->o_Ush = take(N * Fs * es);
+  c->o_Osh = take(Fs ? N * d * es : 0);
+  c->o_dAsh = take(N * Fs * es);
+  c->o_dBsh = take(N * Fs * es);
   // fp32 scratch: SIMT GEMM outputs (fp32 path) and router logits / router dX part
-  const size_t f32n = use_tc(c) ? N * E : std::max(std::max(P * F, P * d), N * E);
+  const size_t big = std::max(std::max(P * F, P * d), std::max(N * Fs, Fs ? N * d : 0));
+  const size_t f32n = use_tc(c) ? N * E : std::max(big, N * E);
   c->o_f32a = take(f32n * 4);
-  c->o_f32b = take((use_tc(c) ? 0 : std::max(P * F, P * d)) * 4);
+  c->o_f32b = take((use_tc(c) ? 0 : big) * 4);
   c->o_dXr = take(N * d * 4);
   // split-K partials of dWr = X^T dZ (tensor cores: equal token blocks, so N % splits == 0)
   if (use_tc(c)) {
@@ -253,117 +266,174 @@ ec_status copy_out(ec_ctx* c, int32_t* idx, float* gate, float* S_out, cudaStrea
   return EC_OK;
 }
 
+// ---------------------------------------------------------------- SwiGLU FFN building blocks
+// One batch of E SwiGLU FFNs over M rows each: [A | B] = H.[Wg | Wu], U = silu(A) * B,
+// O = U.Wd. Used for the routed experts (E experts, M selected rows each) and for the
+// shared experts (one FFN of the concatenated width over all N tokens).
+struct FfnNames {
+  const char *up, *down, *dgrad_up, *dgrad_h, *wgrad;
+};
+const FfnNames kRouted = {"gemm_gate_up_swiglu", "gemm_down", "gemm_dgrad_up_swiglu",
+                          "gemm_dgrad_h", "gemm_wgrad"};
+const FfnNames kShared = {"shared_gate_up_swiglu", "shared_down", "shared_dgrad_up_swiglu",
+                          "shared_dgrad_h", "shared_wgrad"};
+
+template <typename T>
+ec_status ffn_forward(ec_ctx* c, const FfnNames& nm, const T* H, const void* Wg, const void* Wu,
+                      const void* Wd, T* A, T* B, T* U, T* O, int E, int M, int F,
+                      cudaStream_t st) {
+  const int d = c->d;
+  const int64_t P = (int64_t)E * M;
+  if (P == 0) return EC_OK;
+  int* status = at<int>(c, c->o_status);
+  if (use_tc(c)) {
+    EC_KERNEL(nm.up, 1, tc_expert_up(H, Wg, Wu, A, B, U, E, M, d, F, status, st));
+    EC_KERNEL(nm.down, 1, tc_expert_down(U, Wd, O, E, M, d, F, status, st));
+  } else {
+    float* Ag = at<float>(c, c->o_f32a);
+    float* Bu = at<float>(c, c->o_f32b);
+    const int64_t hs = (int64_t)M * d, ws = (int64_t)d * F, os = (int64_t)M * F;
+    EC_KERNEL(nm.up, 1,
+              launch_simt_gemm(sg(H, hs, d, 1, Wg, ws, F, 1, Ag, os, F, M, F, d, E), et(c), et(c), st));
+    EC_KERNEL(nm.up, 1,
+              launch_simt_gemm(sg(H, hs, d, 1, Wu, ws, F, 1, Bu, os, F, M, F, d, E), et(c), et(c), st));
+    EC_KERNEL("swiglu", 1, launch_swiglu_fwd_ew<T>(Ag, Bu, A, B, U, P * F, st));
+    float* O32 = at<float>(c, c->o_f32a);
+    EC_KERNEL(nm.down, 1,
+              launch_simt_gemm(sg(U, os, F, 1, Wd, (int64_t)F * d, d, 1, O32, hs, d, M, d, F, E),
+                               et(c), et(c), st));
+    EC_KERNEL("convert_o", 1, launch_convert<T>(O32, O, P * d, st));
+  }
+  return EC_OK;
+}
+
+// Backward of ffn_forward given dO: dU = dO.Wd^T, dA = dU*B*silu'(A), dB = dU*silu(A),
+// dH = dA.Wg^T + dB.Wu^T, dWd = U^T.dO, dWg = H^T.dA, dWu = H^T.dB (fp32, overwritten).
+template <typename T>
+ec_status ffn_backward(ec_ctx* c, const FfnNames& nm, const T* dO, const T* H, const T* A,
+                       const T* B, const T* U, const void* Wg, const void* Wu, const void* Wd,
+                       T* dA, T* dB, T* dH, float* dWg, float* dWu, float* dWd, int E, int M, int F,
+                       cudaStream_t st) {
+  const int d = c->d;
+  const int64_t P = (int64_t)E * M;
+  if (P == 0) {
+    EC_CUDA(cudaMemsetAsync(dWg, 0, (size_t)E * d * F * 4, st), "zero dWg");
+    EC_CUDA(cudaMemsetAsync(dWu, 0, (size_t)E * d * F * 4, st), "zero dWu");
+    EC_CUDA(cudaMemsetAsync(dWd, 0, (size_t)E * d * F * 4, st), "zero dWd");
+    return EC_OK;
+  }
+  int* status = at<int>(c, c->o_status);
+  if (use_tc(c)) {
+    EC_KERNEL(nm.dgrad_up, 1, tc_expert_dgrad_up(dO, Wd, A, B, dA, dB, E, M, d, F, status, st));
+    EC_KERNEL(nm.dgrad_h, 1, tc_expert_dgrad_h(dA, dB, Wg, Wu, dH, E, M, d, F, status, st));
+    EC_KERNEL(nm.wgrad, 2,
+              tc_expert_wgrad(H, U, dO, dA, dB, dWg, dWu, dWd, E, M, d, F, status, st));
+  } else {
+    float* dU32 = at<float>(c, c->o_f32a);
+    float* dH32 = at<float>(c, c->o_f32b);
+    const int64_t hs = (int64_t)M * d, fs = (int64_t)M * F, wgs = (int64_t)d * F;
+    // dU = dO . Wd^T : B[k=i][n=j] = Wd[j][i]
+    EC_KERNEL(nm.dgrad_up, 1,
+              launch_simt_gemm(sg(dO, hs, d, 1, Wd, (int64_t)F * d, 1, d, dU32, fs, F, M, F, d, E),
+                               et(c), et(c), st));
+    EC_KERNEL("swiglu_bwd", 1, launch_swiglu_bwd_ew<T>(dU32, A, B, dA, dB, P * F, st));
+    // dH = dA . Wg^T + dB . Wu^T
+    EC_KERNEL(nm.dgrad_h, 1,
+              launch_simt_gemm(sg(dA, fs, F, 1, Wg, wgs, 1, F, dH32, hs, d, M, d, F, E),
+                               et(c), et(c), st));
+    EC_KERNEL(nm.dgrad_h, 1,
+              launch_simt_gemm(sg(dB, fs, F, 1, Wu, wgs, 1, F, dH32, hs, d, M, d, F, E, 1.f),
+                               et(c), et(c), st));
+    EC_KERNEL("convert_dh", 1, launch_convert<T>(dH32, dH, P * d, st));
+    // dWd = U^T dO ; dWg = H^T dA ; dWu = H^T dB   (A[m][k] = U[k][m])
+    EC_KERNEL(nm.wgrad, 1,
+              launch_simt_gemm(sg(U, fs, 1, F, dO, hs, d, 1, dWd, (int64_t)F * d, d, F, d, M, E),
+                               et(c), et(c), st));
+    EC_KERNEL(nm.wgrad, 1,
+              launch_simt_gemm(sg(H, hs, 1, d, dA, fs, F, 1, dWg, wgs, F, d, F, M, E),
+                               et(c), et(c), st));
+    EC_KERNEL(nm.wgrad, 1,
+              launch_simt_gemm(sg(H, hs, 1, d, dB, fs, F, 1, dWu, wgs, F, d, F, M, E),
+                               et(c), et(c), st));
+  }
+  return EC_OK;
+}
+
+#define EC_TRY(call)                  \
+  do {                                \
+    ec_status _s = (call);            \
+    if (_s != EC_OK) return _s;       \
+  } while (0)
+
 // ---------------------------------------------------------------- forward
+// Shared experts (appendix "Token Coverage": they process every token) are one SwiGLU FFN
+// of width Fs over all N tokens; their output is added in the combine.
 template <typename T>
 ec_status run_forward(ec_ctx* c, const void* X, const void* Wg, const void* Wu, const void* Wd,
-                      void* Y, cudaStream_t st) {
-  const int N = c->N, d = c->d, E = c->E, F = c->F, M = c->M;
+                      const void* Wgs, const void* Wus, const void* Wds, void* Y,
+                      cudaStream_t st) {
+  const int N = c->N, d = c->d, E = c->E, F = c->F, M = c->M, Fs = c->Fs;
   const int64_t P = (int64_t)E * M;
   const int pz = P > 0;
+  const T* Xt = static_cast<const T*>(X);
   T* H = at<T>(c, c->o_H);
-  T* A = at<T>(c, c->o_A);
-  T* B = at<T>(c, c->o_B);
-  T* U = at<T>(c, c->o_U);
   T* O = at<T>(c, c->o_O);
-  int* status = at<int>(c, c->o_status);
-  const int* idx = at<int>(c, c->o_idx);
-  EC_KERNEL("gather", pz, launch_gather<T>(static_cast<const T*>(X), idx, H, P, d, st));
-  if (P > 0) {
-    if (use_tc(c)) {
-      EC_KERNEL("gemm_gate_up_swiglu", 1, tc_expert_up(H, Wg, Wu, A, B, U, E, M, d, F, status, st));
-      EC_KERNEL("gemm_down", 1, tc_expert_down(U, Wd, O, E, M, d, F, status, st));
-    } else {
-      float* Ag = at<float>(c, c->o_f32a);
-      float* Bu = at<float>(c, c->o_f32b);
-      const int64_t hs = (int64_t)M * d, ws = (int64_t)d * F, os = (int64_t)M * F;
-      EC_KERNEL("gemm_gate", 1,
-                launch_simt_gemm(sg(H, hs, d, 1, Wg, ws, F, 1, Ag, os, F, M, F, d, E), et(c), et(c), st));
-      EC_KERNEL("gemm_up", 1,
-                launch_simt_gemm(sg(H, hs, d, 1, Wu, ws, F, 1, Bu, os, F, M, F, d, E), et(c), et(c), st));
-      EC_KERNEL("swiglu", 1, launch_swiglu_fwd_ew<T>(Ag, Bu, A, B, U, P * F, st));
-      float* O32 = at<float>(c, c->o_f32a);
-      EC_KERNEL("gemm_down", 1,
-                launch_simt_gemm(sg(U, os, F, 1, Wd, (int64_t)F * d, d, 1, O32, hs, d, M, d, F, E),
-                                 et(c), et(c), st));
-      EC_KERNEL("convert_o", 1, launch_convert<T>(O32, O, P * d, st));
-    }
+  const T* Osh = nullptr;
+  if (Fs > 0) {
+    T* o = at<T>(c, c->o_Osh);
+    EC_TRY(ffn_forward<T>(c, kShared, Xt, Wgs, Wus, Wds, at<T>(c, c->o_Ash), at<T>(c, c->o_Bsh),
+                          at<T>(c, c->o_Ush), o, 1, N, Fs, st));
+    Osh = o;
   }
+  const int* idx = at<int>(c, c->o_idx);
+  EC_KERNEL("gather", pz, launch_gather<T>(Xt, idx, H, P, d, st));
+  EC_TRY(ffn_forward<T>(c, kRouted, H, Wg, Wu, Wd, at<T>(c, c->o_A), at<T>(c, c->o_B),
+                        at<T>(c, c->o_U), O, E, M, F, st));
   EC_KERNEL("combine", N > 0,
             launch_combine<T>(O, at<float>(c, c->o_gate), at<int>(c, c->o_slot),
-                              c->residual ? static_cast<const T*>(X) : nullptr,
-                              static_cast<T*>(Y), N, E, M, d, st));
+                              c->residual ? Xt : nullptr, Osh, static_cast<T*>(Y), N, E, M, d,
+                              st));
   return EC_OK;
 }
 
 // ---------------------------------------------------------------- backward
 template <typename T>
 ec_status run_backward(ec_ctx* c, const void* dY, void* dX, float* dWr, float* dbr, float* dWg,
-                       float* dWu, float* dWd, cudaStream_t st) {
-  const int N = c->N, d = c->d, E = c->E, F = c->F, M = c->M;
+                       float* dWu, float* dWd, float* dWgs, float* dWus, float* dWds,
+                       cudaStream_t st) {
+  const int N = c->N, d = c->d, E = c->E, F = c->F, M = c->M, Fs = c->Fs;
   const int64_t P = (int64_t)E * M;
   const int pz = P > 0, nz = N > 0;
-  T* H = at<T>(c, c->o_H);
-  T* A = at<T>(c, c->o_A);
-  T* B = at<T>(c, c->o_B);
-  T* U = at<T>(c, c->o_U);
+  const T* dYt = static_cast<const T*>(dY);
   T* O = at<T>(c, c->o_O);
   T* dH = O;  // O is dead once dgate is formed
   T* dO = at<T>(c, c->o_dO);
-  T* dA = at<T>(c, c->o_dA);
-  T* dB = at<T>(c, c->o_dB);
   float* dgate = at<float>(c, c->o_dgate);
   float* dZ = at<float>(c, c->o_dZ);
   int* status = at<int>(c, c->o_status);
   const int* idx = at<int>(c, c->o_idx);
   const float* gate = at<float>(c, c->o_gate);
   const int* slot = at<int>(c, c->o_slot);
-  const int64_t hs = (int64_t)M * d, fs = (int64_t)M * F, wgs = (int64_t)d * F;
 
   EC_KERNEL("bwd_gather_scale", pz,
-            launch_bwd_gather_scale<T>(static_cast<const T*>(dY), O, idx, gate, dO, dgate, P, d, st));
-  if (P > 0) {
-    if (use_tc(c)) {
-      EC_KERNEL("gemm_dgrad_up_swiglu", 1,
-                tc_expert_dgrad_up(dO, c->Wd, A, B, dA, dB, E, M, d, F, status, st));
-      EC_KERNEL("gemm_dgrad_h", 1, tc_expert_dgrad_h(dA, dB, c->Wg, c->Wu, dH, E, M, d, F, status, st));
-      EC_KERNEL("gemm_wgrad", 2,
-                tc_expert_wgrad(H, U, dO, dA, dB, dWg, dWu, dWd, E, M, d, F, status, st));
-    } else {
-      float* dU32 = at<float>(c, c->o_f32a);
-      float* dH32 = at<float>(c, c->o_f32b);
-      // dU = dO . Wd^T : B[k=i][n=j] = Wd[j][i]
-      EC_KERNEL("gemm_dgrad_u", 1,
-                launch_simt_gemm(sg(dO, hs, d, 1, c->Wd, (int64_t)F * d, 1, d, dU32, fs, F, M, F, d, E),
-                                 et(c), et(c), st));
-      EC_KERNEL("swiglu_bwd", 1, launch_swiglu_bwd_ew<T>(dU32, A, B, dA, dB, P * F, st));
-      // dH = dA . Wg^T + dB . Wu^T
-      EC_KERNEL("gemm_dgrad_h_gate", 1,
-                launch_simt_gemm(sg(dA, fs, F, 1, c->Wg, wgs, 1, F, dH32, hs, d, M, d, F, E),
-                                 et(c), et(c), st));
-      EC_KERNEL("gemm_dgrad_h_up", 1,
-                launch_simt_gemm(sg(dB, fs, F, 1, c->Wu, wgs, 1, F, dH32, hs, d, M, d, F, E, 1.f),
-                                 et(c), et(c), st));
-      EC_KERNEL("convert_dh", 1, launch_convert<T>(dH32, dH, P * d, st));
-      // dWd = U^T dO ; dWg = H^T dA ; dWu = H^T dB   (A[m][k] = U[k][m])
-      EC_KERNEL("gemm_wgrad_down", 1,
-                launch_simt_gemm(sg(U, fs, 1, F, dO, hs, d, 1, dWd, (int64_t)F * d, d, F, d, M, E),
-                                 et(c), et(c), st));
-      EC_KERNEL("gemm_wgrad_gate", 1,
-                launch_simt_gemm(sg(H, hs, 1, d, dA, fs, F, 1, dWg, wgs, F, d, F, M, E),
-                                 et(c), et(c), st));
-      EC_KERNEL("gemm_wgrad_up", 1,
-                launch_simt_gemm(sg(H, hs, 1, d, dB, fs, F, 1, dWu, wgs, F, d, F, M, E),
-                                 et(c), et(c), st));
-    }
-  } else {
-    EC_CUDA(cudaMemsetAsync(dWg, 0, (size_t)E * d * F * 4, st), "zero dWg");
-    EC_CUDA(cudaMemsetAsync(dWu, 0, (size_t)E * d * F * 4, st), "zero dWu");
-    EC_CUDA(cudaMemsetAsync(dWd, 0, (size_t)E * d * F * 4, st), "zero dWd");
+            launch_bwd_gather_scale<T>(dYt, O, idx, gate, dO, dgate, P, d, st));
+  EC_TRY(ffn_backward<T>(c, kRouted, dO, at<T>(c, c->o_H), at<T>(c, c->o_A), at<T>(c, c->o_B),
+                         at<T>(c, c->o_U), c->Wg, c->Wu, c->Wd, at<T>(c, c->o_dA),
+                         at<T>(c, c->o_dB), dH, dWg, dWu, dWd, E, M, F, st));
+  const T* dHsh = nullptr;
+  if (Fs > 0) {
+    // shared experts: dO is dY itself (no gate), the input gradient goes into the dX scatter
+    T* dh = at<T>(c, c->o_Osh);
+    EC_TRY(ffn_backward<T>(c, kShared, dYt, static_cast<const T*>(c->X), at<T>(c, c->o_Ash),
+                           at<T>(c, c->o_Bsh), at<T>(c, c->o_Ush), c->Wgs, c->Wus, c->Wds,
+                           at<T>(c, c->o_dAsh), at<T>(c, c->o_dBsh), dh, dWgs, dWus, dWds, 1, N,
+                           Fs, st));
+    dHsh = dh;
   }
   // router: dZ = S (dS - <dS,S>), dX = dZ Wr^T + sum dH, dWr = X^T dZ, dbr = sum dZ
   float* dXr = at<float>(c, c->o_dXr);
   float* part = at<float>(c, c->o_part);
-  const T* res = c->residual ? static_cast<const T*>(dY) : nullptr;
+  const T* res = c->residual ? dYt : nullptr;
   if (use_tc(c)) {
     bf16* dZb = at<bf16>(c, c->o_dZb);
     EC_KERNEL("softmax_bwd", nz,
@@ -371,7 +441,7 @@ ec_status run_backward(ec_ctx* c, const void* dY, void* dX, float* dWr, float* d
     EC_KERNEL("router_dgrad_gemm", nz,
               tc_router_dgrad(dZb, at<void>(c, c->o_wrpad), dXr, N, d, c->Ep, status, st));
     EC_KERNEL("dx_combine", nz,
-              launch_dx_combine<T>(dH, slot, dXr, res, static_cast<T*>(dX), N, E, M, d, st));
+              launch_dx_combine<T>(dH, slot, dXr, res, dHsh, static_cast<T*>(dX), N, E, M, d, st));
     EC_KERNEL("router_wgrad_gemm", nz,
               tc_router_wgrad(c->X, dZb, part, N, d, c->Ep, c->wr_splits, status, st));
     EC_KERNEL("router_wgrad_reduce", 1,
@@ -383,7 +453,7 @@ ec_status run_backward(ec_ctx* c, const void* dY, void* dX, float* dWr, float* d
               launch_simt_gemm(sg(dZ, 0, E, 1, c->Wr, 0, 1, E, dXr, 0, d, N, d, E, 1), EType::F32,
                                et(c), st));
     EC_KERNEL("dx_combine", nz,
-              launch_dx_combine<T>(dH, slot, dXr, res, static_cast<T*>(dX), N, E, M, d, st));
+              launch_dx_combine<T>(dH, slot, dXr, res, dHsh, static_cast<T*>(dX), N, E, M, d, st));
     SimtGemmArgs a = sg(c->X, 0, 1, d, dZ, 0, E, 1, part, 0, E, d, E, N, 1);
     a.splits = c->wr_splits;
     a.c_split = (int64_t)d * E;
@@ -481,22 +551,26 @@ ec_status ec_route(ec_ctx* c, const void* X, const void* Wr, const float* br, co
   return copy_out(c, idx, gate, S_out, st);
 }
 
-ec_status ec_moe_forward(ec_ctx* c, const void* X, const void* Wr, const float* br, const void* Wg,
-                         const void* Wu, const void* Wd, void* Y, int32_t* idx, float* gate,
-                         float* S_out, void* stream) {
+static ec_status forward_impl(ec_ctx* c, const void* X, const void* Wr, const float* br,
+                              const void* Wg, const void* Wu, const void* Wd, const void* Wgs,
+                              const void* Wus, const void* Wds, void* Y, int32_t* idx,
+                              float* gate, float* S_out, void* stream) {
   ec_status s = check_ready(c);
   if (s != EC_OK) return s;
   if (!X || !Wr || !Wg || !Wu || !Wd || !Y)
     return fail(c, EC_ERR_INVALID_ARG, "X, Wr, Wg, Wu, Wd and Y are required");
   for (const void* p : {X, Wr, Wg, Wu, Wd, (const void*)Y})
     if (!aligned16(p)) return fail(c, EC_ERR_INVALID_ARG, "tensors must be 16-byte aligned");
+  if (c->Fs > 0 && (!Wgs || !Wus || !Wds || !aligned16(Wgs) || !aligned16(Wus) || !aligned16(Wds)))
+    return fail(c, EC_ERR_INVALID_ARG, "shared-expert weights are required and 16-byte aligned");
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   c->have_fwd = false;
+  c->Wgs = Wgs; c->Wus = Wus; c->Wds = Wds;
   s = c->dtype == EC_BF16 ? run_route<bf16>(c, X, Wr, br, nullptr, st)
                           : run_route<float>(c, X, Wr, br, nullptr, st);
   if (s != EC_OK) return s;
-  s = c->dtype == EC_BF16 ? run_forward<bf16>(c, X, Wg, Wu, Wd, Y, st)
-                          : run_forward<float>(c, X, Wg, Wu, Wd, Y, st);
+  s = c->dtype == EC_BF16 ? run_forward<bf16>(c, X, Wg, Wu, Wd, Wgs, Wus, Wds, Y, st)
+                          : run_forward<float>(c, X, Wg, Wu, Wd, Wgs, Wus, Wds, Y, st);
   if (s != EC_OK) return s;
   mark(c, "end", st);
   s = copy_out(c, idx, gate, S_out, st);
@@ -506,22 +580,75 @@ ec_status ec_moe_forward(ec_ctx* c, const void* X, const void* Wr, const float* 
   return EC_OK;
 }
 
-ec_status ec_moe_backward(ec_ctx* c, const void* dY, void* dX, float* dWr, float* dbr, float* dWg,
-                          float* dWu, float* dWd, void* stream) {
+static ec_status backward_impl(ec_ctx* c, const void* dY, void* dX, float* dWr, float* dbr,
+                               float* dWg, float* dWu, float* dWd, float* dWgs, float* dWus,
+                               float* dWds, void* stream) {
   ec_status s = check_ready(c);
   if (s != EC_OK) return s;
-  if (!c->have_fwd) return fail(c, EC_ERR_STATE, "ec_moe_backward needs a preceding ec_moe_forward");
+  if (!c->have_fwd) return fail(c, EC_ERR_STATE, "the backward call needs a preceding forward");
   if (!dY || !dX || !dWr || !dWg || !dWu || !dWd)
     return fail(c, EC_ERR_INVALID_ARG, "dY, dX, dWr, dWg, dWu and dWd are required");
   for (const void* p : {dY, (const void*)dX, (const void*)dWr, (const void*)dWg, (const void*)dWu,
                         (const void*)dWd})
     if (!aligned16(p)) return fail(c, EC_ERR_INVALID_ARG, "tensors must be 16-byte aligned");
+  if (c->Fs > 0 && (!dWgs || !dWus || !dWds || !aligned16(dWgs) || !aligned16(dWus) ||
+                    !aligned16(dWds)))
+    return fail(c, EC_ERR_INVALID_ARG, "shared-expert gradients are required and 16-byte aligned");
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  s = c->dtype == EC_BF16 ? run_backward<bf16>(c, dY, dX, dWr, dbr, dWg, dWu, dWd, st)
-                          : run_backward<float>(c, dY, dX, dWr, dbr, dWg, dWu, dWd, st);
+  c->dWgs = dWgs; c->dWus = dWus; c->dWds = dWds;
+  s = c->dtype == EC_BF16
+          ? run_backward<bf16>(c, dY, dX, dWr, dbr, dWg, dWu, dWd, dWgs, dWus, dWds, st)
+          : run_backward<float>(c, dY, dX, dWr, dbr, dWg, dWu, dWd, dWgs, dWus, dWds, st);
   if (s != EC_OK) return s;
   mark(c, "end", st);
   return EC_OK;
+}
+
+ec_status ec_moe_forward(ec_ctx* c, const void* X, const void* Wr, const float* br, const void* Wg,
+                         const void* Wu, const void* Wd, void* Y, int32_t* idx, float* gate,
+                         float* S_out, void* stream) {
+  if (c && c->Fs > 0)
+    return fail(c, EC_ERR_STATE, "the context has shared experts: use ec_moe_forward_shared");
+  return forward_impl(c, X, Wr, br, Wg, Wu, Wd, nullptr, nullptr, nullptr, Y, idx, gate, S_out,
+                      stream);
+}
+
+ec_status ec_moe_backward(ec_ctx* c, const void* dY, void* dX, float* dWr, float* dbr, float* dWg,
+                          float* dWu, float* dWd, void* stream) {
+  if (c && c->Fs > 0)
+    return fail(c, EC_ERR_STATE, "the context has shared experts: use ec_moe_backward_shared");
+  return backward_impl(c, dY, dX, dWr, dbr, dWg, dWu, dWd, nullptr, nullptr, nullptr, stream);
+}
+
+ec_status ec_ctx_set_shared(ec_ctx* c, int32_t d_ff_shared) {
+  if (!c) return EC_ERR_INVALID_ARG;
+  if (c->ws) return fail(c, EC_ERR_STATE, "set shared experts before attaching the workspace");
+  if (d_ff_shared < 0) return fail(c, EC_ERR_SHAPE, "negative shared width");
+  if (c->dtype == EC_BF16 && d_ff_shared % 64)
+    return fail(c, EC_ERR_UNSUPPORTED, "bf16 shared width must be a multiple of 64");
+  if (c->dtype == EC_F32 && d_ff_shared % 4)
+    return fail(c, EC_ERR_UNSUPPORTED, "fp32 shared width must be a multiple of 4");
+  c->Fs = d_ff_shared;
+  c->have_fwd = false;
+  layout(c);
+  return EC_OK;
+}
+
+ec_status ec_moe_forward_shared(ec_ctx* c, const void* X, const void* Wr, const float* br,
+                                const void* Wg, const void* Wu, const void* Wd, const void* Wg_s,
+                                const void* Wu_s, const void* Wd_s, void* Y, int32_t* idx,
+                                float* gate, float* S_out, void* stream) {
+  if (c && c->Fs == 0)
+    return fail(c, EC_ERR_STATE, "no shared experts configured (ec_ctx_set_shared)");
+  return forward_impl(c, X, Wr, br, Wg, Wu, Wd, Wg_s, Wu_s, Wd_s, Y, idx, gate, S_out, stream);
+}
+
+ec_status ec_moe_backward_shared(ec_ctx* c, const void* dY, void* dX, float* dWr, float* dbr,
+                                 float* dWg, float* dWu, float* dWd, float* dWg_s, float* dWu_s,
+                                 float* dWd_s, void* stream) {
+  if (c && c->Fs == 0)
+    return fail(c, EC_ERR_STATE, "no shared experts configured (ec_ctx_set_shared)");
+  return backward_impl(c, dY, dX, dWr, dbr, dWg, dWu, dWd, dWg_s, dWu_s, dWd_s, stream);
 }
 
 ec_status ec_ctx_set_residual(ec_ctx* c, int32_t on) {

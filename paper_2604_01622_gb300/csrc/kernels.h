@@ -21,10 +21,10 @@ cudaError_t launch_topk(const float* ST, int N, int E, int G, const int* group_o
 // ---------------------------------------------------------------- data movement
 template <typename T>
 cudaError_t launch_gather(const T* X, const int* idx, T* H, int64_t P, int d, cudaStream_t st);
-// Y_t = R_t (if R) + sum over the experts that chose t of gate * O row.
+// Y_t = R_t + R2_t (each if given) + sum over the experts that chose t of gate * O row.
 template <typename T>
-cudaError_t launch_combine(const T* O, const float* gate, const int* slot, const T* R, T* Y, int N,
-                           int E, int M, int d, cudaStream_t st);
+cudaError_t launch_combine(const T* O, const float* gate, const int* slot, const T* R, const T* R2,
+                           T* Y, int N, int E, int M, int d, cudaStream_t st);
 template <typename T>
 cudaError_t launch_bwd_gather_scale(const T* dY, const T* O, const int* idx, const float* gate,
                                     T* dO, float* dgate, int64_t P, int d, cudaStream_t st);
@@ -32,10 +32,10 @@ cudaError_t launch_softmax_bwd(const float* S, const int* slot, const float* dga
                                __nv_bfloat16* dZb, int N, int E, int Ep, int M, cudaStream_t st);
 cudaError_t launch_reduce_partials(const float* part, float* out, int rows, int cols, int ld,
                                    int splits, cudaStream_t st);
-// dX_t = dXr_t + R_t (each if given) + sum of the token's dH rows.
+// dX_t = dXr_t + R_t + R2_t (each if given) + sum of the token's dH rows.
 template <typename T>
-cudaError_t launch_dx_combine(const T* dH, const int* slot, const float* dXr, const T* R, T* dX,
-                              int N, int E, int M, int d, cudaStream_t st);
+cudaError_t launch_dx_combine(const T* dH, const int* slot, const float* dXr, const T* R,
+                              const T* R2, T* dX, int N, int E, int M, int d, cudaStream_t st);
 cudaError_t launch_colsum(const float* Z, float* out, int N, int E, cudaStream_t st);
 template <typename T>
 cudaError_t launch_swiglu_fwd_ew(const float* Ag, const float* Bu, T* A, T* B, T* U, int64_t n,

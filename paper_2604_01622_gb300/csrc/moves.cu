@@ -67,7 +67,8 @@ __device__ __forceinline__ int token_pairs(const int* __restrict__ slot, const f
 template <typename T>
 __global__ void combine_kernel(const T* __restrict__ O, const float* __restrict__ gate,
                                const int* __restrict__ slot, const T* __restrict__ R,
-                               T* __restrict__ Y, int N, int E, int M, int d) {
+                               const T* __restrict__ R2, T* __restrict__ Y, int N, int E, int M,
+                               int d) {
   extern __shared__ int sh[];
   int* s_e = sh;
   int* s_m = sh + E;
@@ -85,6 +86,12 @@ __global__ void combine_kernel(const T* __restrict__ O, const float* __restrict_
 #pragma unroll
       for (int j = 0; j < VN; ++j) acc[j] = 0.f;
     }
+    if (R2) {
+      float r[VN];
+      unpack16(__ldg(reinterpret_cast<const uint4*>(R2 + (size_t)t * d) + v), r, T());
+#pragma unroll
+      for (int j = 0; j < VN; ++j) acc[j] += r[j];
+    }
     for (int p = 0; p < cnt; ++p) {
       const size_t row = (size_t)s_e[p] * M + s_m[p];
       const uint4 u = __ldg(reinterpret_cast<const uint4*>(O + row * d) + v);
@@ -99,11 +106,11 @@ __global__ void combine_kernel(const T* __restrict__ O, const float* __restrict_
 }
 
 template <typename T>
-cudaError_t launch_combine(const T* O, const float* gate, const int* slot, const T* R, T* Y, int N,
-                           int E, int M, int d, cudaStream_t st) {
+cudaError_t launch_combine(const T* O, const float* gate, const int* slot, const T* R, const T* R2,
+                           T* Y, int N, int E, int M, int d, cudaStream_t st) {
   if (N == 0) return cudaSuccess;
   const size_t smem = (size_t)3 * E * sizeof(int);
-  combine_kernel<T><<<N, 128, smem, st>>>(O, gate, slot, R, Y, N, E, M, d);
+  combine_kernel<T><<<N, 128, smem, st>>>(O, gate, slot, R, R2, Y, N, E, M, d);
   return cudaGetLastError();
 }
 
@@ -219,7 +226,8 @@ cudaError_t launch_reduce_partials(const float* part, float* out, int rows, int 
 template <typename T>
 __global__ void dx_combine_kernel(const T* __restrict__ dH, const int* __restrict__ slot,
                                   const float* __restrict__ dXr, const T* __restrict__ R,
-                                  T* __restrict__ dX, int N, int E, int M, int d) {
+                                  const T* __restrict__ R2, T* __restrict__ dX, int N, int E,
+                                  int M, int d) {
   extern __shared__ int sh[];
   int* s_e = sh;
   int* s_m = sh + E;
@@ -247,6 +255,12 @@ __global__ void dx_combine_kernel(const T* __restrict__ dH, const int* __restric
 #pragma unroll
       for (int j = 0; j < VN; ++j) acc[j] += r[j];
     }
+    if (R2) {
+      float r[VN];
+      unpack16(__ldg(reinterpret_cast<const uint4*>(R2 + (size_t)t * d) + v), r, T());
+#pragma unroll
+      for (int j = 0; j < VN; ++j) acc[j] += r[j];
+    }
     for (int p = 0; p < cnt; ++p) {
       const size_t row = (size_t)s_e[p] * M + s_m[p];
       float h[VN];
@@ -259,11 +273,11 @@ __global__ void dx_combine_kernel(const T* __restrict__ dH, const int* __restric
 }
 
 template <typename T>
-cudaError_t launch_dx_combine(const T* dH, const int* slot, const float* dXr, const T* R, T* dX,
-                              int N, int E, int M, int d, cudaStream_t st) {
+cudaError_t launch_dx_combine(const T* dH, const int* slot, const float* dXr, const T* R,
+                              const T* R2, T* dX, int N, int E, int M, int d, cudaStream_t st) {
   if (N == 0) return cudaSuccess;
   const size_t smem = (size_t)2 * E * sizeof(int);
-  dx_combine_kernel<T><<<N, 128, smem, st>>>(dH, slot, dXr, R, dX, N, E, M, d);
+  dx_combine_kernel<T><<<N, 128, smem, st>>>(dH, slot, dXr, R, R2, dX, N, E, M, d);
   return cudaGetLastError();
 }
 
@@ -369,12 +383,12 @@ cudaError_t launch_reduce_splits(const float* part, float* out, int64_t n, int s
 
 #define ECMOE_INST(T)                                                                            \
   template cudaError_t launch_gather<T>(const T*, const int*, T*, int64_t, int, cudaStream_t);    \
-  template cudaError_t launch_combine<T>(const T*, const float*, const int*, const T*, T*, int,   \
-                                         int, int, int, cudaStream_t);                            \
+  template cudaError_t launch_combine<T>(const T*, const float*, const int*, const T*, const T*,  \
+                                         T*, int, int, int, int, cudaStream_t);                   \
   template cudaError_t launch_bwd_gather_scale<T>(const T*, const T*, const int*, const float*,   \
                                                   T*, float*, int64_t, int, cudaStream_t);        \
-  template cudaError_t launch_dx_combine<T>(const T*, const int*, const float*, const T*, T*, int, \
-                                            int, int, int, cudaStream_t);                         \
+  template cudaError_t launch_dx_combine<T>(const T*, const int*, const float*, const T*,         \
+                                            const T*, T*, int, int, int, int, cudaStream_t);      \
   template cudaError_t launch_swiglu_fwd_ew<T>(const float*, const float*, T*, T*, T*, int64_t,   \
                                                cudaStream_t);                                     \
   template cudaError_t launch_swiglu_bwd_ew<T>(const float*, const T*, const T*, T*, T*,          \

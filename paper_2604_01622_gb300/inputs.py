@@ -7,7 +7,8 @@ layer takes k_g as an input array). Both the CUDA path (tests, bench) and the
 float64 oracle's tests consume the arrays made here.
 
 Workloads stand in for one MoE layer of the paper's EC-vs-TC model (d=2048,
-64 fine-grained experts, App. B); the paper's training data is not used.
+64 fine-grained experts; appendix "Experimental Setup"); the paper's training data
+is not used.
 
 Random numbers come from numpy's counter-based Philox bit generator with a
 fixed 128-bit key per (workload seed, layer, tensor), so every machine
@@ -231,6 +232,42 @@ def make_layer(w: Workload, layer: int, experts: slice | None = None) -> LayerIn
     Wu = per_expert(_T_WU, (d, d_ff), s_in)
     Wd = per_expert(_T_WD, (d_ff, d), s_ff)
     return LayerInputs(Wr, br, Wg, Wu, Wd)
+
+
+@dataclass
+class SharedInputs:
+    """Shared experts in concatenated form: expert s owns columns s*f .. s*f+f-1 of Wg, Wu
+    ([d][S*f]) and the same rows of Wd ([S*f][d])."""
+    n: int
+    f: int
+    Wg: Tensor
+    Wu: Tensor
+    Wd: Tensor
+
+    def expert(self, s: int):
+        """float64 (Wg_s, Wu_s, Wd_s) of shared expert s."""
+        c = slice(s * self.f, (s + 1) * self.f)
+        return self.Wg.f64()[:, c], self.Wu.f64()[:, c], self.Wd.f64()[c, :]
+
+
+_T_SHARED = 3000
+
+
+def make_shared(w: Workload, layer: int, n: int, f: int) -> SharedInputs:
+    """n shared experts of width f, drawn like the routed experts' weights."""
+    d = w.d
+    if w.init == "fan_in":
+        s_in, s_ff = 1.0 / math.sqrt(d), 1.0 / math.sqrt(f)
+    else:
+        s_in = s_ff = 0.02
+    g, u, dn = [], [], []
+    for s in range(n):
+        g.append(_normal(_rng(w.seed, layer, _T_SHARED + 3 * s), (d, f), s_in))
+        u.append(_normal(_rng(w.seed, layer, _T_SHARED + 3 * s + 1), (d, f), s_in))
+        dn.append(_normal(_rng(w.seed, layer, _T_SHARED + 3 * s + 2), (f, d), s_ff))
+    return SharedInputs(n, f, _store(np.concatenate(g, axis=1), w.dtype),
+                        _store(np.concatenate(u, axis=1), w.dtype),
+                        _store(np.concatenate(dn, axis=0), w.dtype))
 
 
 def make_inputs(w: Workload, with_layers: bool = True) -> Inputs:

@@ -9,7 +9,8 @@ import torch
 
 from . import (EC_BF16, EC_F32, ec_check_device, ec_ctx_create, ec_ctx_destroy,
                ec_ctx_profile, ec_ctx_set_capacity, ec_ctx_set_profiling, ec_ctx_set_residual,
-               ec_ctx_set_workspace,
+               ec_ctx_set_shared, ec_ctx_set_workspace, ec_moe_backward_shared,
+               ec_moe_forward_shared,
                ec_kernel_launches, ec_moe_backward, ec_moe_forward, ec_route,
                ec_rows_per_expert, ec_workspace_bytes)
 
@@ -27,13 +28,17 @@ def _stream(stream):
 class ECMoELayer:
     """One layer shape: N tokens in groups `group_off`, E experts, capacities k_g."""
 
-    def __init__(self, N, d, E, d_ff, group_off, k_g, dtype="bf16", device="cuda"):
+    def __init__(self, N, d, E, d_ff, group_off, k_g, dtype="bf16", device="cuda",
+                 d_ff_shared=0):
         self.N, self.d, self.E, self.d_ff = int(N), int(d), int(E), int(d_ff)
         self.G = len(group_off) - 1
         self.code, self.tdtype = _DT[dtype]
         self.device = torch.device(device)
+        self.d_ff_shared = int(d_ff_shared)
         self.ctx = ec_ctx_create(self.N, self.d, self.E, self.d_ff, self.G, group_off, k_g,
                                  self.code)
+        if self.d_ff_shared:
+            ec_ctx_set_shared(self.ctx, self.d_ff_shared)
         self.ws_bytes = ec_workspace_bytes(self.ctx)
         self.ws = torch.empty(self.ws_bytes, dtype=torch.uint8, device=self.device)
         ec_ctx_set_workspace(self.ctx, self.ws.data_ptr(), self.ws_bytes)
@@ -61,18 +66,25 @@ class ECMoELayer:
                  _stream(stream))
         return idx, gate, S
 
-    def forward(self, X, Wr, br, Wg, Wu, Wd, Y=None, stream=None, outputs=True):
-        """Y = EC-MoE(X). Returns (Y, idx, gate, S) (idx/gate/S None if outputs=False)."""
+    def forward(self, X, Wr, br, Wg, Wu, Wd, Y=None, stream=None, outputs=True, shared=None):
+        """Y = EC-MoE(X) (+ shared experts). Returns (Y, idx, gate, S); idx/gate/S are None if
+        outputs=False. shared = (Wg_s, Wu_s, Wd_s) in concatenated form when configured."""
         Y = self._empty(self.N, self.d) if Y is None else Y
         idx = gate = S = None
         if outputs:
             idx = self._empty(self.E, self.M, dtype=torch.int32)
             gate = self._empty(self.E, self.M, dtype=torch.float32)
             S = self._empty(self.E, self.N, dtype=torch.float32)
-        ec_moe_forward(self.ctx, _p(X), _p(Wr), _p(br), _p(Wg), _p(Wu), _p(Wd), _p(Y),
-                       _p(idx), _p(gate), _p(S), _stream(stream))
+        if self.d_ff_shared:
+            Wgs, Wus, Wds = shared
+            ec_moe_forward_shared(self.ctx, _p(X), _p(Wr), _p(br), _p(Wg), _p(Wu), _p(Wd),
+                                  _p(Wgs), _p(Wus), _p(Wds), _p(Y), _p(idx), _p(gate), _p(S),
+                                  _stream(stream))
+        else:
+            ec_moe_forward(self.ctx, _p(X), _p(Wr), _p(br), _p(Wg), _p(Wu), _p(Wd), _p(Y),
+                           _p(idx), _p(gate), _p(S), _stream(stream))
         # the backward pass reads these through the pointers the context remembered
-        self._keep = (X, Wr, br, Wg, Wu, Wd)
+        self._keep = (X, Wr, br, Wg, Wu, Wd, shared)
         return Y, idx, gate, S
 
     def backward(self, dY, grads=None, stream=None, with_bias=False):
@@ -85,8 +97,18 @@ class ECMoELayer:
             "dWu": self._empty(self.E, self.d, self.d_ff, dtype=torch.float32),
             "dWd": self._empty(self.E, self.d_ff, self.d, dtype=torch.float32),
         }
-        ec_moe_backward(self.ctx, _p(dY), _p(g["dX"]), _p(g["dWr"]), _p(g.get("dbr")),
-                        _p(g["dWg"]), _p(g["dWu"]), _p(g["dWd"]), _stream(stream))
+        if self.d_ff_shared:
+            for k, shape in (("dWg_s", (self.d, self.d_ff_shared)),
+                             ("dWu_s", (self.d, self.d_ff_shared)),
+                             ("dWd_s", (self.d_ff_shared, self.d))):
+                if g.get(k) is None:
+                    g[k] = self._empty(*shape, dtype=torch.float32)
+            ec_moe_backward_shared(self.ctx, _p(dY), _p(g["dX"]), _p(g["dWr"]), _p(g.get("dbr")),
+                                   _p(g["dWg"]), _p(g["dWu"]), _p(g["dWd"]), _p(g["dWg_s"]),
+                                   _p(g["dWu_s"]), _p(g["dWd_s"]), _stream(stream))
+        else:
+            ec_moe_backward(self.ctx, _p(dY), _p(g["dX"]), _p(g["dWr"]), _p(g.get("dbr")),
+                            _p(g["dWg"]), _p(g["dWu"]), _p(g["dWd"]), _stream(stream))
         return g
 
     def set_profiling(self, on: bool):

@@ -299,3 +299,63 @@ def test_residual_stack_backward_matches_finite_differences():
         fd = (np.sum(dOut * xp[-1]) - np.sum(dOut * xm[-1])) / (2 * h)
         an = float(np.sum(dX * V))
         assert abs(fd - an) <= 1e-6 * max(1.0, abs(an))
+
+
+# --------------------------------------------------------------- shared experts (appendix "Token Coverage")
+def _shared(seed, d, f, S=2):
+    rng = np.random.default_rng(seed)
+    return [(rng.standard_normal((d, f)) / np.sqrt(d), rng.standard_normal((d, f)) / np.sqrt(d),
+             rng.standard_normal((f, d)) / np.sqrt(f)) for _ in range(S)]
+
+
+def test_shared_experts_sum_equals_one_concatenated_swiglu():
+    """Two shared experts of width f act like one SwiGLU FFN of width 2f (hidden units are
+    independent), computed here with torch on concatenated weights."""
+    X, Wr, br, Wg, Wu, Wd, groups, k = _tiny(40)
+    sh = _shared(41, X.shape[1], 7)
+    with_sh = O.forward(X, Wr, br, Wg, Wu, Wd, groups, k, shared=sh)
+    without = O.forward(X, Wr, br, Wg, Wu, Wd, groups, k)
+    tx = torch.tensor(X)
+    Wgc = torch.tensor(np.concatenate([s[0] for s in sh], axis=1))
+    Wuc = torch.tensor(np.concatenate([s[1] for s in sh], axis=1))
+    Wdc = torch.tensor(np.concatenate([s[2] for s in sh], axis=0))
+    ffn = (torch.nn.functional.silu(tx @ Wgc) * (tx @ Wuc)) @ Wdc
+    np.testing.assert_allclose(with_sh["Y"] - without["Y"], ffn.numpy(), rtol=1e-11, atol=1e-12)
+    # unpicked tokens now carry only the shared output
+    picked = np.zeros(X.shape[0], bool)
+    picked[with_sh["idx"].ravel()] = True
+    np.testing.assert_allclose(with_sh["Y"][~picked], ffn.numpy()[~picked], rtol=1e-11, atol=1e-12)
+
+
+def test_shared_experts_backward_matches_finite_differences():
+    X, Wr, br, Wg, Wu, Wd, groups, k = _tiny(42)
+    sh = _shared(43, X.shape[1], 6)
+    rng = np.random.default_rng(44)
+    dY = rng.standard_normal(X.shape)
+    out = O.forward(X, Wr, br, Wg, Wu, Wd, groups, k, shared=sh)
+    g = O.backward(out, dY, Wr, Wg, Wu, Wd)
+    h = 1e-6
+
+    def f(X_, sh_):
+        o = O.forward(X_, Wr, br, Wg, Wu, Wd, groups, k, shared=sh_)
+        return float(np.sum(dY * o["Y"])), np.array_equal(o["idx"], out["idx"])
+    checked = 0
+    for trial in range(3):
+        V = rng.standard_normal(X.shape)
+        (fp, okp), (fm, okm) = f(X + h * V, sh), f(X - h * V, sh)
+        if okp and okm:
+            an = float(np.sum(g["dX"] * V))
+            assert abs((fp - fm) / (2 * h) - an) <= 1e-6 * max(1.0, abs(an))
+            checked += 1
+        for s_i in range(2):
+            for w_i in range(3):
+                Vw = rng.standard_normal(sh[s_i][w_i].shape)
+                shp = [list(t) for t in sh]
+                shm = [list(t) for t in sh]
+                shp[s_i][w_i] = sh[s_i][w_i] + h * Vw
+                shm[s_i][w_i] = sh[s_i][w_i] - h * Vw
+                fd = (f(X, shp)[0] - f(X, shm)[0]) / (2 * h)
+                an = float(np.sum(g["dshared"][s_i][w_i] * Vw))
+                assert abs(fd - an) <= 1e-6 * max(1.0, abs(an)), (s_i, w_i)
+                checked += 1
+    assert checked >= 12
