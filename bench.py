@@ -211,11 +211,16 @@ def run_ours(args):
 
     X, dY = to_dev(inp.X), to_dev(inp.dY)
     stack = []          # one context per layer; several layers stack with residual adds
-    for Ld in inp.layers:
+    Fs = args.shared_experts * args.shared_dff
+    for li, Ld in enumerate(inp.layers):
         wts = (to_dev(Ld.Wr), None if Ld.br is None else torch.from_numpy(Ld.br).to(device),
                to_dev(Ld.Wg), to_dev(Ld.Wu), to_dev(Ld.Wd))
+        shared = None
+        if Fs:
+            sh = I.make_shared(w, li, args.shared_experts, args.shared_dff)
+            shared = (to_dev(sh.Wg), to_dev(sh.Wu), to_dev(sh.Wd))
         lay_l = ECMoELayer(w.N, w.d, w.E, w.d_ff, inp.group_off, inp.k_g, dtype=w.dtype,
-                           device=device)
+                           device=device, d_ff_shared=Fs)
         if w.layers > 1:
             lay_l.set_residual(True)
         g = {"dX": torch.empty_like(X),
@@ -225,7 +230,11 @@ def run_ours(args):
              "dWg": torch.empty(w.E, w.d, w.d_ff, dtype=torch.float32, device=device),
              "dWu": torch.empty(w.E, w.d, w.d_ff, dtype=torch.float32, device=device),
              "dWd": torch.empty(w.E, w.d_ff, w.d, dtype=torch.float32, device=device)}
-        stack.append((lay_l, wts, [torch.empty_like(X)], g))
+        if Fs:
+            g.update(dWg_s=torch.empty(w.d, Fs, dtype=torch.float32, device=device),
+                     dWu_s=torch.empty(w.d, Fs, dtype=torch.float32, device=device),
+                     dWd_s=torch.empty(Fs, w.d, dtype=torch.float32, device=device))
+        stack.append((lay_l, wts, [torch.empty_like(X)], g, shared))
     lay, (Wr, br, Wg, Wu, Wd) = stack[0][0], stack[0][1]
     Y = stack[-1][2][0]
     grads = stack[0][3]
@@ -234,13 +243,13 @@ def run_ours(args):
     def run_stack(x, dy, y_last, dx_first, st=None):
         """Forward through every layer, then backward in reverse; returns nothing."""
         h = x
-        for i, (l_, wts, ybuf, g) in enumerate(stack):
+        for i, (l_, wts, ybuf, g, shared) in enumerate(stack):
             out = y_last if i == len(stack) - 1 else ybuf[0]
-            l_.forward(h, *wts, Y=out, outputs=False, stream=st)
+            l_.forward(h, *wts, Y=out, outputs=False, stream=st, shared=shared)
             h = out
         d = dy
         for i in range(len(stack) - 1, -1, -1):
-            l_, wts, ybuf, g = stack[i]
+            l_, wts, ybuf, g, _sh = stack[i]
             gi = dict(g)
             if i == 0:
                 gi["dX"] = dx_first
@@ -340,6 +349,7 @@ def run_ours(args):
     for name, t in phases:
         per.setdefault(name, []).append(t)
     gemm = {k: v for k, v in per.items() if k.startswith("gemm_")}
+    shared_ms = sum(sum(v) for k, v in per.items() if k.startswith("shared_")) / args.steps
     gemm_launches = sum(len(v) for v in gemm.values()) + len(per.get("gemm_wgrad", []))
     gemm_ms_step = sum(sum(v) for v in gemm.values()) / args.steps
     P = w.E * int(inp.k_g.sum())
@@ -378,7 +388,7 @@ def run_ours(args):
         "scaling": "weak", "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
         "config": {"workload": w.name, "sequences": w.G, "seq_len": w.L, "tokens": w.N,
                    "d_model": w.d, "experts": w.E, "d_ff": w.d_ff, "k_per_seq": w.k_base,
-                   "layers": w.layers,
+                   "layers": w.layers, "shared_experts": args.shared_experts,
                    "parallelism": f"replicas{ws}" if ws > 1 else "single",
                    "l2": "inputs and activations larger than L2 (no flush)"},
     }
@@ -390,6 +400,11 @@ def run_ours(args):
                   "h2d_bytes_per_step": int(X.numel() * X.element_size() * 2),
                   "d2h_bytes_per_step": int(X.numel() * X.element_size() * 2)}
     out["roofline"] = roofline
+    if Fs:
+        sh_flops = 18.0 * w.N * w.d * Fs * w.layers
+        out["shared_experts"] = {"experts": args.shared_experts, "d_ff_each": args.shared_dff,
+                                 "gemm_ms_per_step": round(shared_ms, 4),
+                                 "tflops": round(sh_flops / (shared_ms * 1e-3) / 1e12, 1)}
     out["gpu_launches"] = int(launches)
     out["kernel_ms_per_step"] = {k: round(sum(v) / args.steps, 4) for k, v in per.items()}
     out["clocks"] = clk
@@ -443,6 +458,9 @@ def main():
     ap.add_argument("--workload", default="ec_d2048_e64")
     ap.add_argument("--seqs", type=int, default=0,
                     help="run only this many sequences of the workload (small profiling cases)")
+    ap.add_argument("--shared-experts", type=int, default=0,
+                    help="add this many shared SwiGLU experts per layer (the paper's block has 2)")
+    ap.add_argument("--shared-dff", type=int, default=1024, help="width of each shared expert")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-tokens", type=int, default=8192,
                     help="tokens of the oracle's CPU baseline sample")
