@@ -140,6 +140,38 @@ ec_status ec_moe_backward_shared(ec_ctx* ctx, const void* dY, void* dX, float* d
                                  float* dWg, float* dWu, float* dWd, float* dWg_s, float* dWu_s,
                                  float* dWd_s, void* stream);
 
+/* Token choice (TC), the routing the paper compares expert choice against (Sec. 2.2,
+ * "Token-choice"): every token t takes its k best experts E_t = TopK_e(S[t,e], k) and
+ *   Y_t = sum_{e in E_t, pair kept} g[t,e] FFN_e(x_t),  g[t,e] = S[t,e] / sum_{e' in E_t} S[t,e']
+ * (gates renormalised over the k chosen experts). With capacity >= 0 each expert keeps at
+ * most `capacity` tokens, the first ones in ascending token order, and drops the rest (a
+ * dropped pair contributes nothing; the token's other gates are unchanged); the paper's
+ * capacity is ceil(CF k N / E) for a capacity factor CF. capacity < 0: dropless (no cap).
+ * Ties in TopK go to the lower expert index; each token's choices are listed best first.
+ * The backward pass holds the choices and drops fixed and differentiates through the gate
+ * normalisation and the softmax.
+ *
+ * ec_tc_ctx_create makes a token-choice context (bf16 only: dtype must be EC_BF16, else
+ * EC_ERR_UNSUPPORTED; 1 <= k <= min(E, 32)). Its workspace holds every expert's rows in one
+ * tensor, each expert's region padded to a multiple of 256 rows (at most N k + 255 E rows).
+ * On such a context ec_route, ec_moe_forward(_shared), ec_moe_backward(_shared),
+ * ec_ctx_set_capacity and ec_ctx_set_shared return EC_ERR_STATE; ec_ctx_set_residual,
+ * profiling, ec_check_device and the workspace calls work as for expert choice.
+ *
+ * ec_tc_forward: X, Wr, br, Wg, Wu, Wd, Y as in ec_moe_forward. Optional outputs (device,
+ * NULL to skip): choice [N][k] int32 expert ids best first, gate [N][k] float normalised
+ * gates, kept [N][k] int32 (1 kept, 0 dropped), load [E] int32 tokens kept per expert,
+ * S_out [N][E] float router scores (token-major, unlike the expert-choice calls).
+ * ec_tc_backward: arguments as in ec_moe_backward; needs a preceding ec_tc_forward on the
+ * same context whose inputs are still alive. */
+ec_status ec_tc_ctx_create(ec_ctx** out, int32_t N, int32_t d, int32_t E, int32_t d_ff,
+                           int32_t k, int32_t capacity, int32_t dtype);
+ec_status ec_tc_forward(ec_ctx* ctx, const void* X, const void* Wr, const float* br,
+                        const void* Wg, const void* Wu, const void* Wd, void* Y, int32_t* choice,
+                        float* gate, int32_t* kept, int32_t* load, float* S_out, void* stream);
+ec_status ec_tc_backward(ec_ctx* ctx, const void* dY, void* dX, float* dWr, float* dbr,
+                         float* dWg, float* dWu, float* dWd, void* stream);
+
 /* Synchronise `stream`, read and clear the device status word. Returns EC_ERR_TIMEOUT if a
  * kernel gave up on a bounded wait since the last check, EC_ERR_CUDA on a CUDA error. */
 ec_status ec_check_device(ec_ctx* ctx, void* stream);

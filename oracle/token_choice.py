@@ -29,6 +29,12 @@ def tc_capacity(cf: float | None, k: int, N: int, E: int):
     return int(math.ceil(cf * k * N / E))
 
 
+def tc_gates(S, choices):
+    """Normalised gates g_tj = S_tj / sum_{j' in E_t} S_tj' of the given choices [N][k]."""
+    sel = np.take_along_axis(np.asarray(S, np.float64), np.asarray(choices), axis=1)
+    return sel / sel.sum(axis=1, keepdims=True)
+
+
 def tc_select(S, k, capacity=None):
     """Returns (choices [N][k] expert ids best first, gates [N][k], kept [N][k] bool)."""
     S = np.asarray(S, np.float64)
@@ -37,8 +43,7 @@ def tc_select(S, k, capacity=None):
     for t in range(N):
         order = np.lexsort((np.arange(E), -(S[t] + 0.0)))     # score desc, expert index asc
         choices[t] = order[:k]
-    sel = np.take_along_axis(S, choices, axis=1)
-    gates = sel / sel.sum(axis=1, keepdims=True)
+    gates = tc_gates(S, choices)
     kept = np.ones((N, k), dtype=bool)
     if capacity is not None:
         load = np.zeros(E, dtype=np.int64)
@@ -59,8 +64,7 @@ def tc_forward(X, Wr, br, Wg, Wu, Wd, k, capacity=None, forced=None):
         choices, gates, kept = tc_select(S, k, capacity)
     else:
         choices, kept = (np.asarray(a) for a in forced)
-        sel = np.take_along_axis(S, choices, axis=1)
-        gates = sel / sel.sum(axis=1, keepdims=True)
+        gates = tc_gates(S, choices)
     Y = np.zeros((N, d))
     cache = {}
     for t in range(N):

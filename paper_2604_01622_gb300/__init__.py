@@ -28,6 +28,7 @@ EXPORTS = (
     "ec_ctx_set_profiling", "ec_ctx_profile", "ec_kernel_launches", "ec_select_static",
     "ec_selftest_bounded_wait", "ec_ctx_set_residual", "ec_capacity_schedule",
     "ec_ctx_set_shared", "ec_moe_forward_shared", "ec_moe_backward_shared",
+    "ec_tc_ctx_create", "ec_tc_forward", "ec_tc_backward",
 )
 
 EC_SCHEDULERS = {"static": 0, "linear": 1, "linear_reverse": 2, "cosine": 3,
@@ -76,6 +77,9 @@ def load():
         "ec_ctx_set_shared": (i32, [vp, i32]),
         "ec_moe_forward_shared": (i32, [vp] * 15),
         "ec_moe_backward_shared": (i32, [vp] * 12),
+        "ec_tc_ctx_create": (i32, [ctypes.POINTER(vp), i32, i32, i32, i32, i32, i32, i32]),
+        "ec_tc_forward": (i32, [vp] * 14),
+        "ec_tc_backward": (i32, [vp] * 9),
         "ec_capacity_schedule": (i32, [i32, ctypes.c_double, ctypes.c_double, ctypes.c_double,
                                        i32, i32, P32, ctypes.POINTER(ctypes.c_double), P32]),
     }
@@ -163,6 +167,25 @@ def ec_moe_forward_shared(ctx, X, Wr, br, Wg, Wu, Wd, Wg_s, Wu_s, Wd_s, Y, idx, 
 def ec_moe_backward_shared(ctx, dY, dX, dWr, dbr, dWg, dWu, dWd, dWg_s, dWu_s, dWd_s, stream):
     _check(ctx, load().ec_moe_backward_shared(ctx, dY, dX, dWr, dbr, dWg, dWu, dWd, dWg_s, dWu_s,
                                               dWd_s, stream))
+
+
+def ec_tc_ctx_create(N, d, E, d_ff, k, capacity, dtype):
+    """Token-choice context: k experts per token, `capacity` tokens per expert (< 0: none)."""
+    lib = load()
+    ctx = ctypes.c_void_p()
+    st = lib.ec_tc_ctx_create(ctypes.byref(ctx), N, d, E, d_ff, k, int(capacity), dtype)
+    if st != EC_OK:
+        raise ECError(st, "ec_tc_ctx_create rejected the sizes")
+    return ctx
+
+
+def ec_tc_forward(ctx, X, Wr, br, Wg, Wu, Wd, Y, choice, gate, kept, load_out, S_out, stream):
+    _check(ctx, load().ec_tc_forward(ctx, X, Wr, br, Wg, Wu, Wd, Y, choice, gate, kept, load_out,
+                                     S_out, stream))
+
+
+def ec_tc_backward(ctx, dY, dX, dWr, dbr, dWg, dWu, dWd, stream):
+    _check(ctx, load().ec_tc_backward(ctx, dY, dX, dWr, dbr, dWg, dWu, dWd, stream))
 
 
 def ec_check_device(ctx, stream):

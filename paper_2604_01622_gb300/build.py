@@ -15,7 +15,7 @@ PKG = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libecmoe.so")
-SOURCES = ["ecmoe_api.cu", "route.cu", "moves.cu", "gemm_simt.cu", "gemm_tc.cu",
+SOURCES = ["ecmoe_api.cu", "route.cu", "route_tc.cu", "moves.cu", "gemm_simt.cu", "gemm_tc.cu",
            "select_static.cu", "capacity.cpp"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr"]

@@ -40,6 +40,10 @@ struct ec_ctx {
   bool have_fwd = false;
   const void *X = nullptr, *Wr = nullptr, *Wg = nullptr, *Wu = nullptr, *Wd = nullptr;
   const float* br = nullptr;
+  // token choice (k > 0): k experts per token, per-expert cap (< 0: none), padded rows
+  int tc_k = 0, tc_cap = -1;
+  int64_t P_tc = 0;
+  size_t o_choice = 0, o_tgate = 0, o_Zs = 0, o_count = 0, o_tiles = 0, o_kept = 0;
   std::string err;
 };
 
@@ -103,10 +107,19 @@ bool use_tc(const ec_ctx* c) { return c->dtype == EC_BF16; }
 
 void layout(ec_ctx* c) {
   const size_t N = c->N, d = c->d, E = c->E, F = c->F, M = c->M_cap, G = c->G, es = esize(c);
-  const size_t P = E * M;
+  // expert rows: E x M for expert choice; token choice keeps each expert's rows in a region
+  // padded to 256 rows, at most N k + 255 E rows in all
+  const size_t P = c->tc_k ? (size_t)c->P_tc : E * M;
   size_t o = 0;
   auto take = [&](size_t bytes) { size_t r = o; o = up256(o + bytes); return r; };
   c->o_status = take(256);
+  const size_t NK = c->tc_k ? N * c->tc_k : 0;
+  c->o_choice = take(NK * 4);
+  c->o_tgate = take(NK * 4);
+  c->o_kept = take(NK * 4);
+  c->o_Zs = take(c->tc_k ? N * 4 : 0);
+  c->o_count = take(c->tc_k ? (E + 1) * 4 : 0);
+  c->o_tiles = take(c->tc_k ? (E + 1) * 4 : 0);
   c->o_goff = take((G + 1) * 4);
   c->o_kg = take(G * 4);
   c->o_koff = take((G + 1) * 4);
@@ -465,6 +478,100 @@ ec_status run_backward(ec_ctx* c, const void* dY, void* dX, float* dWr, float* d
   return EC_OK;
 }
 
+// ---------------------------------------------------------------- token choice (bf16)
+// Sec. 2.2 "Token-choice": router -> per-token top-k with renormalised gates and the
+// per-expert cap -> gather into padded expert regions -> variable-row expert GEMMs ->
+// gated combine through the token->row map.
+ec_status run_tc_forward(ec_ctx* c, const void* X, const void* Wr, const float* br, const void* Wg,
+                         const void* Wu, const void* Wd, void* Y, cudaStream_t st) {
+  const int N = c->N, d = c->d, E = c->E, F = c->F, k = c->tc_k;
+  const int nz = N > 0;
+  int* status = at<int>(c, c->o_status);
+  float* S = at<float>(c, c->o_S);
+  int* count = at<int>(c, c->o_count);
+  int* tiles = at<int>(c, c->o_tiles);
+  int* row_token = at<int>(c, c->o_idx);
+  float* row_gate = at<float>(c, c->o_gate);
+  int* slot = at<int>(c, c->o_slot);
+  const bf16* Xt = static_cast<const bf16*>(X);
+  bf16* H = at<bf16>(c, c->o_H);
+  bf16* U = at<bf16>(c, c->o_U);
+  bf16* O = at<bf16>(c, c->o_O);
+  if (!nz) return EC_OK;
+  EC_KERNEL("router_gemm_softmax", 2,
+            tc_router_softmax(X, Wr, at<void>(c, c->o_wrpad), br, S, at<float>(c, c->o_ST), N, d,
+                              E, status, st));
+  EC_KERNEL("tc_route", 4,
+            launch_tc_route(S, N, E, k, c->tc_cap, at<int>(c, c->o_choice),
+                            at<float>(c, c->o_tgate), at<float>(c, c->o_Zs), count, tiles,
+                            row_token, row_gate, slot, at<int>(c, c->o_kept), st));
+  const VarRows vr{tiles, count, (int)c->P_tc};
+  EC_KERNEL("gather", 1, launch_gather<bf16>(Xt, row_token, H, c->P_tc, d, st, count + E));
+  EC_KERNEL("gemm_gate_up_swiglu", 1,
+            tc_expert_up(H, Wg, Wu, at<bf16>(c, c->o_A), at<bf16>(c, c->o_B), U, E, 0, d, F,
+                         status, st, &vr));
+  EC_KERNEL("gemm_down", 1, tc_expert_down(U, Wd, O, E, 0, d, F, status, st, &vr));
+  EC_KERNEL("combine", 1,
+            launch_combine<bf16>(O, row_gate, slot, c->residual ? Xt : nullptr, nullptr,
+                                 static_cast<bf16*>(Y), N, E, 0, d, st));
+  return EC_OK;
+}
+
+ec_status run_tc_backward(ec_ctx* c, const void* dY, void* dX, float* dWr, float* dbr, float* dWg,
+                          float* dWu, float* dWd, cudaStream_t st) {
+  const int N = c->N, d = c->d, E = c->E, F = c->F, k = c->tc_k;
+  if (N == 0) {
+    const size_t w = (size_t)E * d * F * 4;
+    EC_CUDA(cudaMemsetAsync(dWg, 0, w, st), "zero dWg");
+    EC_CUDA(cudaMemsetAsync(dWu, 0, w, st), "zero dWu");
+    EC_CUDA(cudaMemsetAsync(dWd, 0, w, st), "zero dWd");
+    EC_CUDA(cudaMemsetAsync(dWr, 0, (size_t)d * E * 4, st), "zero dWr");
+    if (dbr) EC_CUDA(cudaMemsetAsync(dbr, 0, (size_t)E * 4, st), "zero dbr");
+    return EC_OK;
+  }
+  int* status = at<int>(c, c->o_status);
+  const int* count = at<int>(c, c->o_count);
+  const VarRows vr{at<int>(c, c->o_tiles), count, (int)c->P_tc};
+  const bf16* dYt = static_cast<const bf16*>(dY);
+  bf16* O = at<bf16>(c, c->o_O);
+  bf16* dH = O;   // O is dead once the gate gradients are formed
+  bf16* dO = at<bf16>(c, c->o_dO);
+  bf16* dA = at<bf16>(c, c->o_dA);
+  bf16* dB = at<bf16>(c, c->o_dB);
+  float* row_dgate = at<float>(c, c->o_dgate);
+  const int* slot = at<int>(c, c->o_slot);
+  EC_KERNEL("bwd_gather_scale", 1,
+            launch_bwd_gather_scale<bf16>(dYt, O, at<int>(c, c->o_idx), at<float>(c, c->o_gate), dO,
+                                          row_dgate, c->P_tc, d, st, count + E));
+  EC_KERNEL("gemm_dgrad_up_swiglu", 1,
+            tc_expert_dgrad_up(dO, c->Wd, at<bf16>(c, c->o_A), at<bf16>(c, c->o_B), dA, dB, E, 0,
+                               d, F, status, st, &vr));
+  EC_KERNEL("gemm_dgrad_h", 1,
+            tc_expert_dgrad_h(dA, dB, c->Wg, c->Wu, dH, E, 0, d, F, status, st, &vr));
+  EC_KERNEL("gemm_wgrad", 2,
+            tc_expert_wgrad(at<bf16>(c, c->o_H), at<bf16>(c, c->o_U), dO, dA, dB, dWg, dWu, dWd, E,
+                            0, d, F, status, st, &vr));
+  float* dZ = at<float>(c, c->o_dZ);
+  bf16* dZb = at<bf16>(c, c->o_dZb);
+  float* dXr = at<float>(c, c->o_dXr);
+  float* part = at<float>(c, c->o_part);
+  EC_KERNEL("softmax_bwd", 1,
+            launch_tc_softmax_bwd(at<float>(c, c->o_S), at<int>(c, c->o_choice),
+                                  at<float>(c, c->o_tgate), at<float>(c, c->o_Zs), slot, row_dgate,
+                                  dZ, dZb, N, E, c->Ep, k, st));
+  EC_KERNEL("router_dgrad_gemm", 1,
+            tc_router_dgrad(dZb, at<void>(c, c->o_wrpad), dXr, N, d, c->Ep, status, st));
+  EC_KERNEL("dx_combine", 1,
+            launch_dx_combine<bf16>(dH, slot, dXr, c->residual ? dYt : nullptr, nullptr,
+                                    static_cast<bf16*>(dX), N, E, 0, d, st));
+  EC_KERNEL("router_wgrad_gemm", 1,
+            tc_router_wgrad(c->X, dZb, part, N, d, c->Ep, c->wr_splits, status, st));
+  EC_KERNEL("router_wgrad_reduce", 1,
+            launch_reduce_partials(part, dWr, d, E, c->Ep, 2 * c->wr_splits, st));
+  if (dbr) EC_KERNEL("router_dbias", 1, launch_colsum(dZ, dbr, N, E, st));
+  return EC_OK;
+}
+
 }  // namespace
 
 // ====================================================================== C ABI
@@ -511,6 +618,7 @@ void ec_ctx_destroy(ec_ctx* c) {
 
 ec_status ec_ctx_set_capacity(ec_ctx* c, const int32_t* k_g) {
   if (!c) return EC_ERR_INVALID_ARG;
+  if (c && c->tc_k) return fail(c, EC_ERR_STATE, "token-choice context: use ec_tc_forward / ec_tc_backward");
   ec_status s = set_groups(c, nullptr, k_g, false);
   if (s != EC_OK) return s;
   return upload_groups(c);
@@ -538,6 +646,7 @@ ec_status ec_route(ec_ctx* c, const void* X, const void* Wr, const float* br, co
                    float* S_out, int32_t* idx, float* gate, void* stream) {
   ec_status s = check_ready(c);
   if (s != EC_OK) return s;
+  if (c && c->tc_k) return fail(c, EC_ERR_STATE, "token-choice context: use ec_tc_forward / ec_tc_backward");
   if (!S_in && (!X || !Wr)) return fail(c, EC_ERR_INVALID_ARG, "X and Wr are required without S_in");
   if (!idx || !gate) return fail(c, EC_ERR_INVALID_ARG, "idx and gate are required");
   if ((X && !aligned16(X)) || (Wr && !aligned16(Wr)) || (S_in && !aligned16(S_in)))
@@ -557,6 +666,7 @@ static ec_status forward_impl(ec_ctx* c, const void* X, const void* Wr, const fl
                               float* gate, float* S_out, void* stream) {
   ec_status s = check_ready(c);
   if (s != EC_OK) return s;
+  if (c && c->tc_k) return fail(c, EC_ERR_STATE, "token-choice context: use ec_tc_forward / ec_tc_backward");
   if (!X || !Wr || !Wg || !Wu || !Wd || !Y)
     return fail(c, EC_ERR_INVALID_ARG, "X, Wr, Wg, Wu, Wd and Y are required");
   for (const void* p : {X, Wr, Wg, Wu, Wd, (const void*)Y})
@@ -585,6 +695,7 @@ static ec_status backward_impl(ec_ctx* c, const void* dY, void* dX, float* dWr, 
                                float* dWds, void* stream) {
   ec_status s = check_ready(c);
   if (s != EC_OK) return s;
+  if (c && c->tc_k) return fail(c, EC_ERR_STATE, "token-choice context: use ec_tc_forward / ec_tc_backward");
   if (!c->have_fwd) return fail(c, EC_ERR_STATE, "the backward call needs a preceding forward");
   if (!dY || !dX || !dWr || !dWg || !dWu || !dWd)
     return fail(c, EC_ERR_INVALID_ARG, "dY, dX, dWr, dWg, dWu and dWd are required");
@@ -622,6 +733,7 @@ ec_status ec_moe_backward(ec_ctx* c, const void* dY, void* dX, float* dWr, float
 
 ec_status ec_ctx_set_shared(ec_ctx* c, int32_t d_ff_shared) {
   if (!c) return EC_ERR_INVALID_ARG;
+  if (c && c->tc_k) return fail(c, EC_ERR_STATE, "token-choice context: use ec_tc_forward / ec_tc_backward");
   if (c->ws) return fail(c, EC_ERR_STATE, "set shared experts before attaching the workspace");
   if (d_ff_shared < 0) return fail(c, EC_ERR_SHAPE, "negative shared width");
   if (c->dtype == EC_BF16 && d_ff_shared % 64)
@@ -649,6 +761,87 @@ ec_status ec_moe_backward_shared(ec_ctx* c, const void* dY, void* dX, float* dWr
   if (c && c->Fs == 0)
     return fail(c, EC_ERR_STATE, "no shared experts configured (ec_ctx_set_shared)");
   return backward_impl(c, dY, dX, dWr, dbr, dWg, dWu, dWd, dWg_s, dWu_s, dWd_s, stream);
+}
+
+ec_status ec_tc_ctx_create(ec_ctx** out, int32_t N, int32_t d, int32_t E, int32_t d_ff,
+                           int32_t k, int32_t capacity, int32_t dtype) {
+  if (!out) return EC_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (dtype != EC_F32 && dtype != EC_BF16) return EC_ERR_INVALID_ARG;
+  if (dtype != EC_BF16) return EC_ERR_UNSUPPORTED;
+  if (N < 0 || d <= 0 || E <= 0 || d_ff <= 0) return EC_ERR_SHAPE;
+  if (k < 1 || k > E || k > 32) return EC_ERR_SHAPE;
+  if (E > 256 || d % 64 || d_ff % 64) return EC_ERR_UNSUPPORTED;
+  const int64_t P = ((int64_t)N * k + 255 * (int64_t)E + 255) / 256 * 256;
+  if (P > ((int64_t)1 << 30)) return EC_ERR_UNSUPPORTED;
+  const int32_t off[2] = {0, N};
+  const int32_t kg[1] = {0};
+  ec_status s = ec_ctx_create(out, N, d, E, d_ff, 1, off, kg, dtype);
+  if (s != EC_OK) return s;
+  ec_ctx* c = *out;
+  c->tc_k = k;
+  c->tc_cap = capacity < 0 ? -1 : capacity;
+  c->P_tc = P;
+  layout(c);
+  return EC_OK;
+}
+
+ec_status ec_tc_forward(ec_ctx* c, const void* X, const void* Wr, const float* br,
+                        const void* Wg, const void* Wu, const void* Wd, void* Y, int32_t* choice,
+                        float* gate, int32_t* kept, int32_t* load, float* S_out, void* stream) {
+  ec_status s = check_ready(c);
+  if (s != EC_OK) return s;
+  if (!c->tc_k) return fail(c, EC_ERR_STATE, "not a token-choice context (ec_tc_ctx_create)");
+  if (!X || !Wr || !Wg || !Wu || !Wd || !Y)
+    return fail(c, EC_ERR_INVALID_ARG, "X, Wr, Wg, Wu, Wd and Y are required");
+  for (const void* p : {X, Wr, Wg, Wu, Wd, (const void*)Y})
+    if (!aligned16(p)) return fail(c, EC_ERR_INVALID_ARG, "tensors must be 16-byte aligned");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  c->have_fwd = false;
+  s = run_tc_forward(c, X, Wr, br, Wg, Wu, Wd, Y, st);
+  if (s != EC_OK) return s;
+  mark(c, "end", st);
+  const size_t NK = (size_t)c->N * c->tc_k;
+  if (NK) {
+    if (choice)
+      EC_CUDA(cudaMemcpyAsync(choice, at<int>(c, c->o_choice), NK * 4, cudaMemcpyDeviceToDevice, st),
+              "choice out");
+    if (gate)
+      EC_CUDA(cudaMemcpyAsync(gate, at<float>(c, c->o_tgate), NK * 4, cudaMemcpyDeviceToDevice, st),
+              "gate out");
+    if (kept)
+      EC_CUDA(cudaMemcpyAsync(kept, at<int>(c, c->o_kept), NK * 4, cudaMemcpyDeviceToDevice, st),
+              "kept out");
+    if (load)
+      EC_CUDA(cudaMemcpyAsync(load, at<int>(c, c->o_count), (size_t)c->E * 4,
+                              cudaMemcpyDeviceToDevice, st), "load out");
+    if (S_out)
+      EC_CUDA(cudaMemcpyAsync(S_out, at<float>(c, c->o_S), (size_t)c->N * c->E * 4,
+                              cudaMemcpyDeviceToDevice, st), "S out");
+  } else if (load) {
+    EC_CUDA(cudaMemsetAsync(load, 0, (size_t)c->E * 4, st), "load out");
+  }
+  c->X = X; c->Wr = Wr; c->br = br; c->Wg = Wg; c->Wu = Wu; c->Wd = Wd;
+  c->have_fwd = true;
+  return EC_OK;
+}
+
+ec_status ec_tc_backward(ec_ctx* c, const void* dY, void* dX, float* dWr, float* dbr,
+                         float* dWg, float* dWu, float* dWd, void* stream) {
+  ec_status s = check_ready(c);
+  if (s != EC_OK) return s;
+  if (!c->tc_k) return fail(c, EC_ERR_STATE, "not a token-choice context (ec_tc_ctx_create)");
+  if (!c->have_fwd) return fail(c, EC_ERR_STATE, "the backward call needs a preceding forward");
+  if (!dY || !dX || !dWr || !dWg || !dWu || !dWd)
+    return fail(c, EC_ERR_INVALID_ARG, "dY, dX, dWr, dWg, dWu and dWd are required");
+  for (const void* p : {dY, (const void*)dX, (const void*)dWr, (const void*)dWg, (const void*)dWu,
+                        (const void*)dWd})
+    if (!aligned16(p)) return fail(c, EC_ERR_INVALID_ARG, "tensors must be 16-byte aligned");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  s = run_tc_backward(c, dY, dX, dWr, dbr, dWg, dWu, dWd, st);
+  if (s != EC_OK) return s;
+  mark(c, "end", st);
+  return EC_OK;
 }
 
 ec_status ec_ctx_set_residual(ec_ctx* c, int32_t on) {

@@ -48,7 +48,15 @@ struct Args {
   int64_t bstride;              // output batch stride (elements)
   int n_valid;                  // router: number of experts
   int* status;
+  // Variable rows per expert (token-choice routing): expert e owns padded rows
+  // vm_tiles[e]*PADR .. vm_tiles[e+1]*PADR of the row-major activations, of which the first
+  // vm_count[e] are real (the rest are zero). Device arrays, read by the kernel.
+  const int* vm_tiles;          // [vm_E + 1] cumulative PADR-row blocks
+  const int* vm_count;          // [vm_E] rows per expert
+  int vm_E;
 };
+
+constexpr int PADR = 256;       // row padding unit of variable-row expert regions
 
 // ------------------------------------------------------------------ PTX wrappers
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
@@ -272,13 +280,61 @@ __device__ __forceinline__ void store_bf16x32(void* dst, const float* v) {
                       pack_bf16x2(v[8 * i + 6], v[8 * i + 7]));
 }
 
+// ------------------------------------------------------------------ tile decode
+// VARM: 0 uniform batch of equal-M problems; 1 variable rows per expert (the M dimension,
+// rows are global padded rows, B is the expert's weights); 2 variable K per expert (weight
+// gradients: K runs over the expert's padded rows).
+struct Tile {
+  int b, mt, nt;
+  int row0;      // first row of this CTA in the A / output row space
+  int valid;     // rows from row0 that are real (the rest are masked)
+  int kbl;       // k-blocks of this tile
+  int krow0;     // first K row (variable K)
+};
+
+template <int VARM, int TM>
+__device__ __forceinline__ Tile tile_at(const Args& p, int tile, int tiles_per_b, uint32_t rank) {
+  static_assert(VARM != 1 || TM == PADR, "variable-row tiles are one padding unit high");
+  Tile t;
+  if constexpr (VARM == 1) {
+    const int mtile = tile / p.n_tiles;
+    t.nt = tile - mtile * p.n_tiles;
+    int lo = 0, hi = p.vm_E;   // last expert whose first block is at or before mtile
+    while (hi - lo > 1) {
+      const int mid = (lo + hi) >> 1;
+      if (__ldg(p.vm_tiles + mid) <= mtile) lo = mid; else hi = mid;
+    }
+    t.b = lo;
+    t.mt = mtile - __ldg(p.vm_tiles + lo);
+    t.row0 = mtile * TM + (int)rank * BM;
+    t.valid = __ldg(p.vm_count + lo) - (t.mt * TM + (int)rank * BM);
+    t.kbl = p.k_blocks;
+    t.krow0 = 0;
+  } else {
+    t.b = tile / tiles_per_b;
+    const int rem = tile - t.b * tiles_per_b;
+    t.mt = rem / p.n_tiles;
+    t.nt = rem - t.mt * p.n_tiles;
+    t.row0 = t.mt * TM + (int)rank * BM;
+    t.valid = p.M - t.row0;
+    if constexpr (VARM == 2) {
+      t.kbl = (__ldg(p.vm_count + t.b) + BK - 1) / BK;
+      t.krow0 = __ldg(p.vm_tiles + t.b) * PADR;
+    } else {
+      t.kbl = p.k_blocks;
+      t.krow0 = 0;
+    }
+  }
+  return t;
+}
+
 // ------------------------------------------------------------------ the kernel
 // PAIR: the CTAs of a 2-CTA cluster share each 256 x BN tile. Each CTA loads its own 128 rows
 // of A and half (BN/2 columns) of B; the leader CTA (rank 0) issues M = 256 MMAs that read
 // both CTAs' shared memory and write each CTA's 128 rows into that CTA's TMEM. Per SM this
 // halves the B traffic into shared memory.
 template <int BN, bool A_MN, bool B_MN, bool B_SPLIT, bool K_SPLIT, int EPI, int STAGES, int EPW,
-          bool PAIR>
+          bool PAIR, int VARM>
 __global__ void __launch_bounds__(64 + 32 * EPW, 1)
 tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ CUtensorMap mA1,
                const __grid_constant__ CUtensorMap mB0, const __grid_constant__ CUtensorMap mB1,
@@ -343,7 +399,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
   const uint32_t tmem_base = *tmem_holder;
 
   const int tiles_per_b = p.m_tiles * p.n_tiles;
-  const int total = p.batch * tiles_per_b;
+  const int total = VARM == 1 ? __ldg(p.vm_tiles + p.vm_E) * p.n_tiles : p.batch * tiles_per_b;
 
   if (warp == 0) {
     // ------------------------------------------------------------ TMA producer
@@ -352,30 +408,34 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
       uint32_t ph = 0;
       bool ok = true;
       for (int tile = cid; tile < total && ok; tile += nwalk) {
-        const int b = tile / tiles_per_b;
-        const int rem = tile - b * tiles_per_b;
-        const int mt = rem / p.n_tiles, nt = rem - mt * p.n_tiles;
-        const int m0 = mt * TM + (int)rank * BM;
-        for (int kb = 0; kb < p.k_blocks; ++kb) {
+        const Tile T = tile_at<VARM, TM>(p, tile, tiles_per_b, rank);
+        const int nt = T.nt;
+        const int m0 = T.row0;
+        const int ab = VARM ? 0 : T.b;          // batch coordinate of A
+        const int bb = VARM == 2 ? 0 : T.b;     // batch coordinate of B
+        for (int kb = 0; kb < T.kbl; ++kb) {
           if (!mbar_wait(&empty[s], ph ^ 1u, abort_flag, p.status)) { ok = false; break; }
           if (!PAIR || leader) mbar_arrive_expect_tx(&full[s], (A_BYTES + B_BYTES) * (PAIR ? 2 : 1));
           // completion goes to the leader's barrier: it gates the pair's MMAs
           const uint32_t fb = PAIR ? mapa_shared(smem_u32(&full[s]), 0) : smem_u32(&full[s]);
+          auto load_b = [&](void* dst, const CUtensorMap* m, int c0, int c1, int bc) {
+            if constexpr (PAIR) tma_load_3d_pair(dst, m, fb, c0, c1, bc);
+            else tma_load_3d(dst, m, &full[s], c0, c1, bc);
+          };
           auto load = [&](void* dst, const CUtensorMap* m, int c0, int c1) {
-            if constexpr (PAIR) tma_load_3d_pair(dst, m, fb, c0, c1, b);
-            else tma_load_3d(dst, m, &full[s], c0, c1, b);
+            load_b(dst, m, c0, c1, bb);
           };
           const bool second = K_SPLIT && kb >= p.k_blocks0;
           const CUtensorMap* mA = second ? &mA1 : &mA0;
           const CUtensorMap* mB = second ? &mB1 : &mB0;
-          const int k0 = (second ? kb - p.k_blocks0 : kb) * BK;
+          const int k0 = (second ? kb - p.k_blocks0 : kb) * BK + T.krow0;
           uint8_t* a_dst = sA + s * A_BYTES;
           uint8_t* b_dst = sB + s * B_BYTES;
           if (!A_MN) {
-            load(a_dst, mA, k0, m0);
+            load_b(a_dst, mA, k0, m0, ab);
           } else {
 #pragma unroll
-            for (int j = 0; j < BM / 64; ++j) load(a_dst + j * 8192, mA, m0 + 64 * j, k0);
+            for (int j = 0; j < BM / 64; ++j) load_b(a_dst + j * 8192, mA, m0 + 64 * j, k0, ab);
           }
           if constexpr (PAIR) {
             // this CTA's half of the B tile: for split tiles the gate (rank 0) or up half
@@ -428,10 +488,11 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
       for (int tile = cid; tile < total && ok; tile += nwalk, ++it) {
         const int a = it & 1;
         const uint32_t use = (uint32_t)(it >> 1);
+        const int kbl = tile_at<VARM, TM>(p, tile, tiles_per_b, 0).kbl;
         if (!mbar_wait(&tempty[a], (use & 1u) ^ 1u, abort_flag, p.status)) { ok = false; break; }
         tc_fence_after();
         const uint32_t tacc = tmem_base + (uint32_t)(a * BN);
-        for (int kb = 0; kb < p.k_blocks; ++kb) {
+        for (int kb = 0; kb < kbl; ++kb) {
           if (!mbar_wait(&full[s], ph, abort_flag, p.status)) { ok = false; break; }
           tc_fence_after();
           const uint32_t sa = smem_u32(sA + s * A_BYTES);
@@ -474,13 +535,19 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
       const uint32_t use = (uint32_t)(it >> 1);
       if (!mbar_wait(&tfull[a], use & 1u, abort_flag, p.status)) break;
       tc_fence_after();
-      const int b = tile / tiles_per_b;
-      const int rem = tile - b * tiles_per_b;
-      const int mt = rem / p.n_tiles, nt = rem - mt * p.n_tiles;
-      const int gm = mt * TM + (int)rank * BM + r;
-      const bool row_ok = gm < p.M;
+      const Tile T = tile_at<VARM, TM>(p, tile, tiles_per_b, rank);
+      const int nt = T.nt;
+      const int gm = T.row0 + r;
+      const bool row_ok = r < T.valid;
+      // Variable rows: a 256-row tile never leaves its expert's padded region, and the
+      // region's unused rows are written as zeros (the weight gradients run their K loop
+      // over them). Uniform batches store only the valid rows.
+      const bool row_st = VARM == 1 ? true : row_ok;
       const uint32_t tacc = tmem_base + (uint32_t)(a * BN) + ((uint32_t)(q * 32) << 16);
-      const int64_t row_off = (int64_t)b * p.bstride + (int64_t)gm * p.ld;
+      const int64_t row_off =
+          VARM == 1 ? (int64_t)gm * p.ld : (int64_t)T.b * p.bstride + (int64_t)gm * p.ld;
+      // zero output: an empty expert's weight gradient, or a padding row
+      const bool no_k = (VARM == 2 && T.kbl == 0) || (VARM == 1 && !row_ok);
       uint32_t v[32];
       float f[32];
 
@@ -491,8 +558,11 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
         for (int c = c32; c < c32 + NC32; ++c) {
           tmem_ld32(tacc + c * 32, v);
           tmem_wait_ld();
+          if (no_k)
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] = 0u;
           const int n = nt * BN + c * 32;
-          if (row_ok && n < p.N) {
+          if (row_st && n < p.N) {
 #pragma unroll
             for (int i = 0; i < 32; ++i) f[i] = f32(v[i]);
             if constexpr (EPI == EPI_STORE_BF16) {
@@ -509,9 +579,12 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
         for (int c = c32; c < c32 + NC32; ++c) {
           tmem_ld32(tacc + c * 32, v);
           tmem_wait_ld();
+          if (no_k)
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] = 0u;
           const int half = c >= BN / 64;
           const int n = nt * (BN / 2) + (c % (BN / 64)) * 32;
-          if (row_ok && n < p.N) {
+          if (row_st && n < p.N) {
             float* out = reinterpret_cast<float*>(half ? p.out1 : p.out0) + row_off + n;
             float4* d4 = reinterpret_cast<float4*>(out);
 #pragma unroll
@@ -528,13 +601,13 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
           tmem_ld32(tacc + BN / 2 + c * 32, w);
           tmem_wait_ld();
           const int n = nt * (BN / 2) + c * 32;
-          if (row_ok && n < p.N) {
+          if (row_st && n < p.N) {
             float g[32];
 #pragma unroll
             for (int i = 0; i < 32; ++i) {
               const float av = f32(v[i]), bv = f32(w[i]);
-              f[i] = av;
-              g[i] = bv;
+              f[i] = no_k ? 0.f : av;
+              g[i] = no_k ? 0.f : bv;
             }
             store_bf16x32(reinterpret_cast<bf16*>(p.out0) + row_off + n, f);
             store_bf16x32(reinterpret_cast<bf16*>(p.out1) + row_off + n, g);
@@ -565,7 +638,12 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
           tmem_ld32(tacc + c * 32, v);
           tmem_wait_ld();
           const int n = nt * BN + c * 32;
-          if (row_ok && n < p.N) {
+          if (no_k && row_st && n < p.N) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) f[i] = 0.f;
+            store_bf16x32(reinterpret_cast<bf16*>(p.out0) + row_off + n, f);
+            store_bf16x32(reinterpret_cast<bf16*>(p.out1) + row_off + n, f);
+          } else if (row_ok && n < p.N) {
             float av[32], bv[32], db[32];
 #pragma unroll
             for (int i = 0; i < 4; ++i) {
@@ -693,10 +771,10 @@ int sm_count() {
 }
 
 template <int BN, bool A_MN, bool B_MN, bool B_SPLIT, bool K_SPLIT, int EPI, int STAGES,
-          int EPW = 8, bool PAIR = false>
+          int EPW = 8, bool PAIR = false, int VARM = 0>
 cudaError_t launch(const CUtensorMap& a0, const CUtensorMap& a1, const CUtensorMap& b0,
                    const CUtensorMap& b1, Args p, cudaStream_t st) {
-  auto kern = tc_gemm_kernel<BN, A_MN, B_MN, B_SPLIT, K_SPLIT, EPI, STAGES, EPW, PAIR>;
+  auto kern = tc_gemm_kernel<BN, A_MN, B_MN, B_SPLIT, K_SPLIT, EPI, STAGES, EPW, PAIR, VARM>;
   constexpr uint32_t smem = smem_bytes<BN, STAGES, PAIR>();
   constexpr int threads = 64 + 32 * EPW;
   static bool attr = false;
@@ -725,9 +803,10 @@ cudaError_t launch(const CUtensorMap& a0, const CUtensorMap& a1, const CUtensorM
     }
     attr = true;
   }
+  // variable rows: p.M carries an upper bound of the padded rows, so `total` bounds the tiles
   if (PAIR) p.m_tiles = (p.M + 2 * BM - 1) / (2 * BM);
   const int total = p.batch * p.m_tiles * p.n_tiles;
-  if (total == 0 || p.k_blocks == 0) return cudaSuccess;
+  if (total == 0 || (VARM != 2 && p.k_blocks == 0)) return cudaSuccess;
   if (PAIR) {
     const int clusters = total < max_clusters ? total : max_clusters;
     cfg.gridDim = dim3(2 * clusters);
@@ -808,90 +887,136 @@ cudaError_t tc_router_softmax(const void* X, const void* Wr, void* Wr_pad, const
   return cudaErrorInvalidValue;
 }
 
+// Activation maps and Args for the expert GEMMs: a uniform batch [E][M][cols], or with `vr`
+// one [1][P][cols] tensor of padded variable-row expert regions (the tile decode finds the
+// expert of each 256-row tile from vr->tiles).
+static cudaError_t act_map(CUtensorMap* m, const void* base, int cols, int E, int M,
+                           const VarRows* vr, uint32_t box_rows) {
+  return vr ? make_map(m, base, cols, vr->P, 1, box_rows) : make_map(m, base, cols, M, E, box_rows);
+}
+
+static Args row_args(int E, int M, int N, int K, int BN_tile, int* status, const VarRows* vr) {
+  Args p = vr ? base_args(1, vr->P, N, K, BN_tile, status) : base_args(E, M, N, K, BN_tile, status);
+  if (vr) {
+    p.vm_tiles = vr->tiles;
+    p.vm_count = vr->count;
+    p.vm_E = E;
+  }
+  return p;
+}
+
+template <int BN, bool A_MN, bool B_MN, bool B_SPLIT, bool K_SPLIT, int EPI>
+static cudaError_t launch_rows(const CUtensorMap& a0, const CUtensorMap& a1, const CUtensorMap& b0,
+                               const CUtensorMap& b1, const Args& p, const VarRows* vr,
+                               cudaStream_t st) {
+  if (vr) return launch<BN, A_MN, B_MN, B_SPLIT, K_SPLIT, EPI, 6, 8, true, 1>(a0, a1, b0, b1, p, st);
+  return launch<BN, A_MN, B_MN, B_SPLIT, K_SPLIT, EPI, 6, 8, true, 0>(a0, a1, b0, b1, p, st);
+}
+
 cudaError_t tc_expert_up(const void* H, const void* Wg, const void* Wu, void* A, void* B, void* U,
-                         int E, int M, int d, int F, int* status, cudaStream_t st) {
+                         int E, int M, int d, int F, int* status, cudaStream_t st,
+                         const VarRows* vr) {
   CUtensorMap ma, mg, mu;
-  TC_TRY(make_map(&ma, H, d, M, E, BM));
+  TC_TRY(act_map(&ma, H, d, E, M, vr, BM));
   TC_TRY(make_map(&mg, Wg, F, d, E, 64));
   TC_TRY(make_map(&mu, Wu, F, d, E, 64));
-  Args p = base_args(E, M, F, d, 128, status);
+  Args p = row_args(E, M, F, d, 128, status, vr);
   p.out0 = A;
   p.out1 = B;
   p.out2 = U;
   p.ld = F;
   p.bstride = (int64_t)M * F;
-  return launch<256, false, true, true, false, EPI_SWIGLU_FWD, 6, 8, true>(ma, ma, mg, mu, p, st);
+  return launch_rows<256, false, true, true, false, EPI_SWIGLU_FWD>(ma, ma, mg, mu, p, vr, st);
 }
 
 cudaError_t tc_expert_down(const void* U, const void* Wd, void* O, int E, int M, int d, int F,
-                           int* status, cudaStream_t st) {
+                           int* status, cudaStream_t st, const VarRows* vr) {
   CUtensorMap ma, mb;
-  TC_TRY(make_map(&ma, U, F, M, E, BM));
+  TC_TRY(act_map(&ma, U, F, E, M, vr, BM));
   TC_TRY(make_map(&mb, Wd, d, F, E, 64));
-  Args p = base_args(E, M, d, F, 256, status);
+  Args p = row_args(E, M, d, F, 256, status, vr);
   p.out0 = O;
   p.ld = d;
   p.bstride = (int64_t)M * d;
-  return launch<256, false, true, false, false, EPI_STORE_BF16, 6, 8, true>(ma, ma, mb, mb, p, st);
+  return launch_rows<256, false, true, false, false, EPI_STORE_BF16>(ma, ma, mb, mb, p, vr, st);
 }
 
 cudaError_t tc_expert_dgrad_up(const void* dO, const void* Wd, const void* A, const void* B,
                                void* dA, void* dB, int E, int M, int d, int F, int* status,
-                               cudaStream_t st) {
+                               cudaStream_t st, const VarRows* vr) {
   CUtensorMap ma, mb;
-  TC_TRY(make_map(&ma, dO, d, M, E, BM));
+  TC_TRY(act_map(&ma, dO, d, E, M, vr, BM));
   TC_TRY(make_map(&mb, Wd, d, F, E, 128));   // B[n=f][k=i] = Wd[f][i]: K-major, half per CTA
-  Args p = base_args(E, M, F, d, 256, status);
+  Args p = row_args(E, M, F, d, 256, status, vr);
   p.in0 = A;
   p.in1 = B;
   p.out0 = dA;
   p.out1 = dB;
   p.ld = F;
   p.bstride = (int64_t)M * F;
-  return launch<256, false, false, false, false, EPI_SWIGLU_BWD, 6, 8, true>(ma, ma, mb, mb, p, st);
+  return launch_rows<256, false, false, false, false, EPI_SWIGLU_BWD>(ma, ma, mb, mb, p, vr, st);
 }
 
 cudaError_t tc_expert_dgrad_h(const void* dA, const void* dB, const void* Wg, const void* Wu,
-                              void* dH, int E, int M, int d, int F, int* status, cudaStream_t st) {
+                              void* dH, int E, int M, int d, int F, int* status, cudaStream_t st,
+                              const VarRows* vr) {
   CUtensorMap ma0, ma1, mb0, mb1;
-  TC_TRY(make_map(&ma0, dA, F, M, E, BM));
-  TC_TRY(make_map(&ma1, dB, F, M, E, BM));
+  TC_TRY(act_map(&ma0, dA, F, E, M, vr, BM));
+  TC_TRY(act_map(&ma1, dB, F, E, M, vr, BM));
   TC_TRY(make_map(&mb0, Wg, F, d, E, 128));  // B[n=i][k=f] = Wg[i][f]: K-major, half per CTA
   TC_TRY(make_map(&mb1, Wu, F, d, E, 128));
-  Args p = base_args(E, M, d, 2 * F, 256, status);
+  Args p = row_args(E, M, d, 2 * F, 256, status, vr);
   p.k_blocks0 = F / BK;
   p.out0 = dH;
   p.ld = d;
   p.bstride = (int64_t)M * d;
-  return launch<256, false, false, false, true, EPI_STORE_BF16, 6, 8, true>(ma0, ma1, mb0, mb1, p, st);
+  return launch_rows<256, false, false, false, true, EPI_STORE_BF16>(ma0, ma1, mb0, mb1, p, vr, st);
 }
 
 cudaError_t tc_expert_wgrad(const void* H, const void* U, const void* dO, const void* dA,
                             const void* dB, float* dWg, float* dWu, float* dWd, int E, int M,
-                            int d, int F, int* status, cudaStream_t st) {
+                            int d, int F, int* status, cudaStream_t st, const VarRows* vr) {
+  // Variable rows: the K loop of expert e runs over its own padded region (count rows,
+  // rounded up to the 64-row k-step, the rest of which is zero in both operands).
+  auto wg_args = [&](int Mo, int No, int BNt) {
+    Args p = base_args(E, Mo, No, vr ? vr->P : M, BNt, status);
+    if (vr) {
+      p.vm_tiles = vr->tiles;
+      p.vm_count = vr->count;
+      p.vm_E = E;
+    }
+    return p;
+  };
   {
     // dWd[e] [F][d] = U[e]^T . dO[e]: A[m=f][k=t] = U[t][f] (MN-major), B[k=t][n=i] = dO[t][i]
     CUtensorMap ma, mb;
-    TC_TRY(make_map(&ma, U, F, M, E, 64));
-    TC_TRY(make_map(&mb, dO, d, M, E, 64));
-    Args p = base_args(E, F, d, M, 256, status);
+    TC_TRY(act_map(&ma, U, F, E, M, vr, 64));
+    TC_TRY(act_map(&mb, dO, d, E, M, vr, 64));
+    Args p = wg_args(F, d, 256);
     p.out0 = dWd;
     p.ld = d;
     p.bstride = (int64_t)F * d;
-    TC_TRY((launch<256, true, true, false, false, EPI_STORE_F32, 6, 8, true>(ma, ma, mb, mb, p, st)));
+    if (vr)
+      TC_TRY((launch<256, true, true, false, false, EPI_STORE_F32, 6, 8, true, 2>(ma, ma, mb, mb, p, st)));
+    else
+      TC_TRY((launch<256, true, true, false, false, EPI_STORE_F32, 6, 8, true>(ma, ma, mb, mb, p, st)));
   }
   {
     // [dWg | dWu][e] [d][F] = H[e]^T . [dA | dB][e]
     CUtensorMap ma, mb0, mb1;
-    TC_TRY(make_map(&ma, H, d, M, E, 64));
-    TC_TRY(make_map(&mb0, dA, F, M, E, 64));
-    TC_TRY(make_map(&mb1, dB, F, M, E, 64));
-    Args p = base_args(E, d, F, M, 128, status);
+    TC_TRY(act_map(&ma, H, d, E, M, vr, 64));
+    TC_TRY(act_map(&mb0, dA, F, E, M, vr, 64));
+    TC_TRY(act_map(&mb1, dB, F, E, M, vr, 64));
+    Args p = wg_args(d, F, 128);
     p.out0 = dWg;
     p.out1 = dWu;
     p.ld = F;
     p.bstride = (int64_t)d * F;
-    TC_TRY((launch<256, true, true, true, false, EPI_STORE_F32_SPLIT, 6, 8, true>(ma, ma, mb0, mb1, p,
+    if (vr)
+      TC_TRY((launch<256, true, true, true, false, EPI_STORE_F32_SPLIT, 6, 8, true, 2>(ma, ma, mb0, mb1,
+                                                                                     p, st)));
+    else
+      TC_TRY((launch<256, true, true, true, false, EPI_STORE_F32_SPLIT, 6, 8, true>(ma, ma, mb0, mb1, p,
                                                                                   st)));
   }
   return cudaSuccess;

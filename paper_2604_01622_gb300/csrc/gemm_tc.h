@@ -9,6 +9,16 @@
 
 namespace ecmoe {
 
+// Variable rows per expert (token-choice routing): expert e owns the padded rows
+// [256*tiles[e], 256*tiles[e+1]) of [P][cols] activation tensors, the first count[e] of them
+// real. tiles [E+1] and count [E] are device arrays; P bounds the padded rows. The GEMMs
+// write the unused rows of each region as zeros.
+struct VarRows {
+  const int* tiles;
+  const int* count;
+  int P;
+};
+
 // Router: Z = X.Wr (+br), S = row softmax over the E experts, written as S [N][E] and
 // S^T [E][N]. X [N][d] bf16, Wr [d][E] bf16. Wr_pad: device scratch of d*round_up(E,64)
 // bf16 (zero-padded copy of Wr made on the stream).
@@ -19,25 +29,29 @@ cudaError_t tc_router_softmax(const void* X, const void* Wr, void* Wr_pad, const
 // [A | B] = H.[Wg | Wu] per expert; U = silu(A) * B. H [E][M][d]; Wg, Wu [E][d][F];
 // A, B, U [E][M][F] bf16.
 cudaError_t tc_expert_up(const void* H, const void* Wg, const void* Wu, void* A, void* B, void* U,
-                         int E, int M, int d, int F, int* status, cudaStream_t st);
+                         int E, int M, int d, int F, int* status, cudaStream_t st,
+                         const VarRows* vr = nullptr);
 
 // O = U.Wd per expert. U [E][M][F]; Wd [E][F][d]; O [E][M][d] bf16.
 cudaError_t tc_expert_down(const void* U, const void* Wd, void* O, int E, int M, int d, int F,
-                           int* status, cudaStream_t st);
+                           int* status, cudaStream_t st, const VarRows* vr = nullptr);
 
 // dU = dO.Wd^T per expert, then dA = dU * B * silu'(A), dB = dU * silu(A) (bf16 out).
 cudaError_t tc_expert_dgrad_up(const void* dO, const void* Wd, const void* A, const void* B,
                                void* dA, void* dB, int E, int M, int d, int F, int* status,
-                               cudaStream_t st);
+                               cudaStream_t st, const VarRows* vr = nullptr);
 
 // dH = dA.Wg^T + dB.Wu^T per expert (one K loop over both halves). dH [E][M][d] bf16.
 cudaError_t tc_expert_dgrad_h(const void* dA, const void* dB, const void* Wg, const void* Wu,
-                              void* dH, int E, int M, int d, int F, int* status, cudaStream_t st);
+                              void* dH, int E, int M, int d, int F, int* status, cudaStream_t st,
+                              const VarRows* vr = nullptr);
 
 // Weight gradients per expert, fp32: dWd = U^T.dO, dWg = H^T.dA, dWu = H^T.dB.
+// With `vr`, each expert sums over its own rows (an expert with none gets zeros).
 cudaError_t tc_expert_wgrad(const void* H, const void* U, const void* dO, const void* dA,
                             const void* dB, float* dWg, float* dWu, float* dWd, int E, int M,
-                            int d, int F, int* status, cudaStream_t st);
+                            int d, int F, int* status, cudaStream_t st,
+                            const VarRows* vr = nullptr);
 
 // Router backward on the tensor cores. dZb [2][N][Ep] bf16: hi and lo planes of the
 // zero-padded softmax gradient (dZ ~ hi + lo); Wr_pad [d][Ep] bf16 (the padded router

@@ -18,16 +18,41 @@ cudaError_t launch_topk(const float* ST, int N, int E, int G, const int* group_o
                         const int* k_off, int M, int max_group, int* idx, float* gate, int* slot,
                         cudaStream_t st);
 
+// ---------------------------------------------------------------- token-choice routing
+// Row top-k of S [N][E] (k <= 32, E <= 512), per-expert counts capped at cap (cap < 0:
+// dropless), padded expert regions (tiles[e] in 256-row blocks), row->token map (-1 in
+// padding), row gates, slot map [N][E] (absolute row or -1) and kept flags [N][k].
+// Token-choice routing of the scores S [N][E] (k <= 32, E <= 512; cap < 0: no cap):
+// choice/tgate/kept [N][k] (experts best first, normalised gates, kept flags), Z [N] (sum of
+// the k chosen scores), count [E+1] (kept rows per expert; count[E] = padded rows in use),
+// tiles [E+1] (cumulative 256-row blocks), row_token/row_gate [P] per padded row (-1 / 0 in
+// padding), slot [N][E] absolute padded row of each kept pair, else -1.
+cudaError_t launch_tc_route(const float* S, int N, int E, int k, int cap, int* choice,
+                            float* tgate, float* Z, int* count, int* tiles, int* row_token,
+                            float* row_gate, int* slot, int* kept, cudaStream_t st);
+// Router gradient of token choice: dZ [N][E] (and optionally the bf16 hi/lo planes
+// dZb [2][N][Ep]) from the per-row gate gradients row_dgate [P].
+cudaError_t launch_tc_softmax_bwd(const float* S, const int* choice, const float* tgate,
+                                  const float* Z, const int* slot, const float* row_dgate,
+                                  float* dZ, __nv_bfloat16* dZb, int N, int E, int Ep, int k,
+                                  cudaStream_t st);
+
 // ---------------------------------------------------------------- data movement
+// H row r = X row idx[r] (zeros where idx[r] < 0), rows r < P and, if p_used is given,
+// r < *p_used (a device count).
 template <typename T>
-cudaError_t launch_gather(const T* X, const int* idx, T* H, int64_t P, int d, cudaStream_t st);
+cudaError_t launch_gather(const T* X, const int* idx, T* H, int64_t P, int d, cudaStream_t st,
+                          const int* p_used = nullptr);
 // Y_t = R_t + R2_t (each if given) + sum over the experts that chose t of gate * O row.
 template <typename T>
 cudaError_t launch_combine(const T* O, const float* gate, const int* slot, const T* R, const T* R2,
                            T* Y, int N, int E, int M, int d, cudaStream_t st);
+// dO row r = gate[r] dY row idx[r], dgate[r] = <dY row idx[r], O row r> (zero rows where
+// idx[r] < 0); rows as in launch_gather.
 template <typename T>
 cudaError_t launch_bwd_gather_scale(const T* dY, const T* O, const int* idx, const float* gate,
-                                    T* dO, float* dgate, int64_t P, int d, cudaStream_t st);
+                                    T* dO, float* dgate, int64_t P, int d, cudaStream_t st,
+                                    const int* p_used = nullptr);
 cudaError_t launch_softmax_bwd(const float* S, const int* slot, const float* dgate, float* dZ,
                                __nv_bfloat16* dZb, int N, int E, int Ep, int M, cudaStream_t st);
 cudaError_t launch_reduce_partials(const float* part, float* out, int rows, int cols, int ld,

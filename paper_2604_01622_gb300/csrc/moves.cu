@@ -18,22 +18,28 @@ static unsigned grid_for(int64_t n, int64_t cap) {
 // ------------------------------------------------------------------ gather H[e][m] = X[idx[e][m]]
 template <typename T>
 __global__ void gather_kernel(const T* __restrict__ X, const int* __restrict__ idx,
-                              T* __restrict__ H, int64_t P, int d) {
+                              T* __restrict__ H, int64_t P, int d, const int* __restrict__ p_used) {
   const int64_t row = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
-  if (row >= P) return;
-  const int t = idx[row];
+  if (row >= P || (p_used && row >= *p_used)) return;
+  const int t = idx[row];     // -1: a padding row of a variable-row expert region
   const int nv = d * (int)sizeof(T) / 16;
-  const uint4* src = reinterpret_cast<const uint4*>(X + (size_t)t * d);
   uint4* dst = reinterpret_cast<uint4*>(H + (size_t)row * d);
+  if (t < 0) {
+    for (int v = lane; v < nv; v += 32) dst[v] = make_uint4(0, 0, 0, 0);
+    return;
+  }
+  const uint4* src = reinterpret_cast<const uint4*>(X + (size_t)t * d);
   for (int v = lane; v < nv; v += 32) dst[v] = __ldg(src + v);
 }
 
 template <typename T>
-cudaError_t launch_gather(const T* X, const int* idx, T* H, int64_t P, int d, cudaStream_t st) {
+cudaError_t launch_gather(const T* X, const int* idx, T* H, int64_t P, int d, cudaStream_t st,
+                          const int* p_used) {
   if (P == 0) return cudaSuccess;
   const int warps = 8;
-  gather_kernel<T><<<(unsigned)((P + warps - 1) / warps), warps * 32, 0, st>>>(X, idx, H, P, d);
+  gather_kernel<T><<<(unsigned)((P + warps - 1) / warps), warps * 32, 0, st>>>(X, idx, H, P, d,
+                                                                                p_used);
   return cudaGetLastError();
 }
 
@@ -119,14 +125,20 @@ template <typename T>
 __global__ void bwd_gather_scale_kernel(const T* __restrict__ dY, const T* __restrict__ O,
                                         const int* __restrict__ idx, const float* __restrict__ gate,
                                         T* __restrict__ dO, float* __restrict__ dgate, int64_t P,
-                                        int d) {
+                                        int d, const int* __restrict__ p_used) {
   const int64_t row = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
-  if (row >= P) return;
+  if (row >= P || (p_used && row >= *p_used)) return;
   const int t = idx[row];
   const float g = gate[row];
   constexpr int VN = 16 / sizeof(T);
   const int nv = d / VN;
+  if (t < 0) {   // padding row: zero gradient row, zero gate gradient
+    uint4* out = reinterpret_cast<uint4*>(dO + (size_t)row * d);
+    for (int v = lane; v < nv; v += 32) out[v] = make_uint4(0, 0, 0, 0);
+    if (lane == 0) dgate[row] = 0.f;
+    return;
+  }
   const uint4* dy = reinterpret_cast<const uint4*>(dY + (size_t)t * d);
   const uint4* o = reinterpret_cast<const uint4*>(O + (size_t)row * d);
   uint4* out = reinterpret_cast<uint4*>(dO + (size_t)row * d);
@@ -148,11 +160,12 @@ __global__ void bwd_gather_scale_kernel(const T* __restrict__ dY, const T* __res
 
 template <typename T>
 cudaError_t launch_bwd_gather_scale(const T* dY, const T* O, const int* idx, const float* gate,
-                                    T* dO, float* dgate, int64_t P, int d, cudaStream_t st) {
+                                    T* dO, float* dgate, int64_t P, int d, cudaStream_t st,
+                                    const int* p_used) {
   if (P == 0) return cudaSuccess;
   const int warps = 8;
   bwd_gather_scale_kernel<T><<<(unsigned)((P + warps - 1) / warps), warps * 32, 0, st>>>(
-      dY, O, idx, gate, dO, dgate, P, d);
+      dY, O, idx, gate, dO, dgate, P, d, p_used);
   return cudaGetLastError();
 }
 
@@ -382,11 +395,13 @@ cudaError_t launch_reduce_splits(const float* part, float* out, int64_t n, int s
 }
 
 #define ECMOE_INST(T)                                                                            \
-  template cudaError_t launch_gather<T>(const T*, const int*, T*, int64_t, int, cudaStream_t);    \
+  template cudaError_t launch_gather<T>(const T*, const int*, T*, int64_t, int, cudaStream_t,     \
+                                        const int*);                                              \
   template cudaError_t launch_combine<T>(const T*, const float*, const int*, const T*, const T*,  \
                                          T*, int, int, int, int, cudaStream_t);                   \
   template cudaError_t launch_bwd_gather_scale<T>(const T*, const T*, const int*, const float*,   \
-                                                  T*, float*, int64_t, int, cudaStream_t);        \
+                                                  T*, float*, int64_t, int, cudaStream_t,         \
+                                                  const int*);                                    \
   template cudaError_t launch_dx_combine<T>(const T*, const int*, const float*, const T*,         \
                                             const T*, T*, int, int, int, int, cudaStream_t);      \
   template cudaError_t launch_swiglu_fwd_ew<T>(const float*, const float*, T*, T*, T*, int64_t,   \

@@ -7,12 +7,14 @@ from __future__ import annotations
 
 import torch
 
+import math
+
 from . import (EC_BF16, EC_F32, ec_check_device, ec_ctx_create, ec_ctx_destroy,
                ec_ctx_profile, ec_ctx_set_capacity, ec_ctx_set_profiling, ec_ctx_set_residual,
-               ec_ctx_set_shared, ec_ctx_set_workspace, ec_moe_backward_shared,
-               ec_moe_forward_shared,
-               ec_kernel_launches, ec_moe_backward, ec_moe_forward, ec_route,
-               ec_rows_per_expert, ec_workspace_bytes)
+               ec_ctx_set_shared, ec_ctx_set_workspace, ec_kernel_launches,
+               ec_moe_backward, ec_moe_backward_shared, ec_moe_forward, ec_moe_forward_shared,
+               ec_route, ec_rows_per_expert, ec_tc_backward, ec_tc_ctx_create, ec_tc_forward,
+               ec_workspace_bytes)
 
 _DT = {"f32": (EC_F32, torch.float32), "bf16": (EC_BF16, torch.bfloat16)}
 
@@ -136,3 +138,64 @@ class ECMoELayer:
             self.close()
         except Exception:
             pass
+
+
+def tc_capacity(cf, k, N, E) -> int:
+    """Token-choice expert capacity ceil(CF k N / E) (arXiv 2604.01622, Sec. 2.2); -1 (no cap,
+    dropless) when cf is None or <= 0."""
+    if cf is None or cf <= 0:
+        return -1
+    return int(math.ceil(cf * k * N / E))
+
+
+class TCMoELayer(ECMoELayer):
+    """Token-choice layer of the same shape (bf16): every token takes its k best experts,
+    each expert keeps at most `capacity` tokens (-1: dropless)."""
+
+    def __init__(self, N, d, E, d_ff, k, capacity=-1, dtype="bf16", device="cuda"):
+        self.N, self.d, self.E, self.d_ff = int(N), int(d), int(E), int(d_ff)
+        self.k, self.capacity = int(k), int(capacity)
+        self.G = 1
+        self.code, self.tdtype = _DT[dtype]
+        self.device = torch.device(device)
+        self.d_ff_shared = 0
+        self.ctx = None
+        self.ctx = ec_tc_ctx_create(self.N, self.d, self.E, self.d_ff, self.k, self.capacity,
+                                    self.code)
+        self.ws_bytes = ec_workspace_bytes(self.ctx)
+        self.ws = torch.empty(self.ws_bytes, dtype=torch.uint8, device=self.device)
+        ec_ctx_set_workspace(self.ctx, self.ws.data_ptr(), self.ws_bytes)
+
+    def route(self, *a, **kw):
+        raise NotImplementedError("token choice routes inside forward()")
+
+    def forward(self, X, Wr, br, Wg, Wu, Wd, Y=None, stream=None, outputs=True, shared=None):
+        """Y = TC-MoE(X). Returns (Y, choice [N][k], gate [N][k], kept [N][k], load [E],
+        S [N][E]); all but Y are None if outputs=False."""
+        if shared is not None:
+            raise ValueError("token-choice layers have no shared experts")
+        Y = self._empty(self.N, self.d) if Y is None else Y
+        outs = [None] * 5
+        if outputs:
+            outs = [self._empty(self.N, self.k, dtype=torch.int32),
+                    self._empty(self.N, self.k, dtype=torch.float32),
+                    self._empty(self.N, self.k, dtype=torch.int32),
+                    self._empty(self.E, dtype=torch.int32),
+                    self._empty(self.N, self.E, dtype=torch.float32)]
+        ec_tc_forward(self.ctx, _p(X), _p(Wr), _p(br), _p(Wg), _p(Wu), _p(Wd), _p(Y),
+                      *[_p(t) for t in outs], _stream(stream))
+        self._keep = (X, Wr, br, Wg, Wu, Wd)
+        return (Y, *outs)
+
+    def backward(self, dY, grads=None, stream=None, with_bias=False):
+        g = grads or {
+            "dX": self._empty(self.N, self.d),
+            "dWr": self._empty(self.d, self.E, dtype=torch.float32),
+            "dbr": self._empty(self.E, dtype=torch.float32) if with_bias else None,
+            "dWg": self._empty(self.E, self.d, self.d_ff, dtype=torch.float32),
+            "dWu": self._empty(self.E, self.d, self.d_ff, dtype=torch.float32),
+            "dWd": self._empty(self.E, self.d_ff, self.d, dtype=torch.float32),
+        }
+        ec_tc_backward(self.ctx, _p(dY), _p(g["dX"]), _p(g["dWr"]), _p(g.get("dbr")),
+                       _p(g["dWg"]), _p(g["dWu"]), _p(g["dWd"]), _stream(stream))
+        return g
