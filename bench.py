@@ -13,6 +13,9 @@ With N > 1 (torchrun) every rank runs its own replica of the workload on its own
 (the layer needs no exchange in the forward pass and this benchmark does not all-reduce
 weight gradients); value = tokens of all ranks / max over ranks of the step time.
 `--impl reference` times the float64 CPU oracle on the host cores instead.
+`--routing tc --tc-k K [--tc-cf CF]` runs the same shape under token-choice routing (each
+token takes its K best experts, capacity ceil(CF K N / E) per expert, dropless without
+--tc-cf), the comparison baseline of the paper's Sec. 2.2.
 """
 from __future__ import annotations
 
@@ -30,6 +33,7 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 METRIC = "EC-MoE layer fwd+bwd tokens/sec on 1 GB300; expert-GEMM % BF16 peak; routing HBM GB/s"
+METRIC_TC = "TC-MoE layer fwd+bwd tokens/sec on 1 GB300 (token-choice comparison routing)"
 UNIT = "tokens/s"
 
 # DRAM traffic per launch of the grouped-GEMM kernels, from one ncu capture of this
@@ -157,6 +161,34 @@ class OracleSample:
         return self.tokens / dt, dt
 
 
+class TCOracleSample:
+    """A bounded sample for the token-choice oracle: `tokens` tokens of the workload's
+    first sequence under the same k and capacity factor."""
+
+    def __init__(self, tokens: int, w, k: int, cf):
+        from paper_2604_01622_gb300 import inputs as I
+        L = min(tokens, w.L)
+        ws = I.scaled(w, G=1, L=L, timestep_capacity=False, layers=1)
+        inp = I.make_inputs(ws)
+        Ld = inp.layers[0]
+        self.tokens, self.k = L, k
+        self.cap = None if cf is None else int(math.ceil(cf * k * L / w.E))
+        self.args = (inp.X.f64(), Ld.Wr.f64(), Ld.br, Ld.Wg.f64(), Ld.Wu.f64(), Ld.Wd.f64())
+        self.dY = inp.dY.f64()
+        self.desc = (f"{L} tokens of one sequence of the workload, token choice k={k}, "
+                     f"capacity {'none' if cf is None else self.cap}, E={w.E}, d={w.d}, "
+                     f"d_ff={w.d_ff}, oracle fwd+bwd")
+
+    def run(self):
+        from oracle import token_choice as TC
+        X, Wr, br, Wg, Wu, Wd = self.args
+        t0 = time.perf_counter()
+        f = TC.tc_forward(X, Wr, br, Wg, Wu, Wd, self.k, self.cap)
+        TC.tc_backward(f, self.dY, Wr, Wg, Wu, Wd)
+        dt = time.perf_counter() - t0
+        return self.tokens / dt, dt
+
+
 # ------------------------------------------------------------------ distributed
 def _dist():
     ws = int(os.environ.get("WORLD_SIZE", "1"))
@@ -197,8 +229,11 @@ def run_ours(args):
         B.build()
     _barrier(ws)
     from paper_2604_01622_gb300 import inputs as I
-    from paper_2604_01622_gb300.layer import ECMoELayer
+    from paper_2604_01622_gb300.layer import ECMoELayer, TCMoELayer, tc_capacity
     w = I.WORKLOADS[args.workload]
+    tc = args.routing == "tc"
+    if tc and args.shared_experts:
+        raise SystemExit("--routing tc has no shared experts")
     if args.seqs:
         w = I.scaled(w, G=args.seqs)
     inp = I.make_inputs(w)
@@ -219,8 +254,13 @@ def run_ours(args):
         if Fs:
             sh = I.make_shared(w, li, args.shared_experts, args.shared_dff)
             shared = (to_dev(sh.Wg), to_dev(sh.Wu), to_dev(sh.Wd))
-        lay_l = ECMoELayer(w.N, w.d, w.E, w.d_ff, inp.group_off, inp.k_g, dtype=w.dtype,
-                           device=device, d_ff_shared=Fs)
+        if tc:
+            tc_cap = tc_capacity(args.tc_cf, args.tc_k, w.N, w.E)
+            lay_l = TCMoELayer(w.N, w.d, w.E, w.d_ff, args.tc_k, tc_cap, dtype=w.dtype,
+                               device=device)
+        else:
+            lay_l = ECMoELayer(w.N, w.d, w.E, w.d_ff, inp.group_off, inp.k_g, dtype=w.dtype,
+                               device=device, d_ff_shared=Fs)
         if w.layers > 1:
             lay_l.set_residual(True)
         g = {"dX": torch.empty_like(X),
@@ -262,6 +302,17 @@ def run_ours(args):
     for _ in range(args.warmup):
         step()
     lay.check()
+    # expert rows per layer: E x sum(k_g) under expert choice; the kept (token, expert)
+    # pairs under token choice (read once from a forward with outputs)
+    if tc:
+        rows = []
+        h = X
+        for l_, wts, ybuf, g, _sh in stack:
+            o = l_.forward(h, *wts, Y=ybuf[0], outputs=True)
+            rows.append(int(o[4].sum().item()))
+            h = ybuf[0]
+    else:
+        rows = [w.E * int(inp.k_g.sum())] * w.layers
 
     # ---- device-timed steps (inputs resident), per-kernel events on the same stream
     for l_ in stack:
@@ -352,8 +403,8 @@ def run_ours(args):
     shared_ms = sum(sum(v) for k, v in per.items() if k.startswith("shared_")) / args.steps
     gemm_launches = sum(len(v) for v in gemm.values()) + len(per.get("gemm_wgrad", []))
     gemm_ms_step = sum(sum(v) for v in gemm.values()) / args.steps
-    P = w.E * int(inp.k_g.sum())
-    flops_step = 18.0 * P * w.d * w.d_ff * w.layers
+    P = sum(rows) / len(rows)
+    flops_step = 18.0 * sum(rows) * w.d * w.d_ff
     gemm_tflops = flops_step / (gemm_ms_step * 1e-3) / 1e12
     gemm_per_launch = flops_step / max(1, gemm_launches / args.steps)
     b = 2 if w.dtype == "bf16" else 4
@@ -361,6 +412,7 @@ def run_ours(args):
     mem_bytes = {
         "router_gemm_softmax": N * d * b + 2 * N * E * 4,
         "topk": 2 * N * E * 4 + 2 * P * 4,
+        "tc_route": 2 * N * E * 4 + 3 * P * 4,
         "gather": 2 * P * d * b,
         "combine": P * d * b + N * d * b,
         "bwd_gather_scale": 3 * P * d * b,
@@ -383,7 +435,7 @@ def run_ours(args):
         "traffic": tr,
     }
     out = {
-        "metric": METRIC, "value": None, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
+        "metric": METRIC_TC if tc else METRIC, "value": None, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": round(ms_max, 4), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
         "config": {"workload": w.name, "sequences": w.G, "seq_len": w.L, "tokens": w.N,
@@ -392,6 +444,9 @@ def run_ours(args):
                    "parallelism": f"replicas{ws}" if ws > 1 else "single",
                    "l2": "inputs and activations larger than L2 (no flush)"},
     }
+    if tc:
+        out["config"].update(routing="token_choice", k=args.tc_k, capacity=tc_cap,
+                             capacity_factor=args.tc_cf, expert_rows=rows)
     out["value"] = round(ws * w.N / (ms_max * 1e-3), 1)
     out["expert_gemm_pct_bf16_peak"] = round(100 * gemm_tflops / bf16_burst, 2)
     out["routing_hbm_gbs"] = None if mem_gbs is None else round(mem_gbs, 1)
@@ -409,7 +464,8 @@ def run_ours(args):
     out["kernel_ms_per_step"] = {k: round(sum(v) / args.steps, 4) for k, v in per.items()}
     out["clocks"] = clk
     if rank == 0 and not args.no_cpu_baseline:
-        smp = OracleSample(args.cpu_tokens, w)
+        smp = (TCOracleSample(args.tc_cpu_tokens, w, args.tc_k, args.tc_cf) if tc
+               else OracleSample(args.cpu_tokens, w))
         v, dt = smp.run()
         out["cpu_baseline"] = {"value": round(v, 2), "unit": UNIT, "cores": _cores(),
                                "kind": "oracle", "sample": smp.desc, "seconds": round(dt, 2)}
@@ -427,7 +483,9 @@ def run_reference(args):
         return
     from paper_2604_01622_gb300 import inputs as I
     w = I.WORKLOADS[args.workload]
-    smp = OracleSample(args.ref_tokens, w)
+    tc = args.routing == "tc"
+    smp = (TCOracleSample(args.tc_cpu_tokens, w, args.tc_k, args.tc_cf) if tc
+           else OracleSample(args.ref_tokens, w))
     for _ in range(args.warmup):
         smp.run()
     total_t = 0.0
@@ -435,13 +493,16 @@ def run_reference(args):
         total_t += smp.run()[1]
     desc = smp.desc
     v = args.steps * smp.tokens / total_t
-    out = {"impl": "reference", "metric": METRIC, "value": round(v, 2), "unit": UNIT,
+    out = {"impl": "reference", "metric": METRIC_TC if tc else METRIC, "value": round(v, 2),
+           "unit": UNIT,
            "n_gpus": 1, "steps": args.steps, "warmup": args.warmup,
            "ms_per_step": round(1e3 * total_t / args.steps, 2), "higher_is_better": True,
            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
            "config": {"workload": w.name, "sequences": w.G, "seq_len": w.L, "tokens": w.N,
                       "d_model": w.d, "experts": w.E, "d_ff": w.d_ff, "k_per_seq": w.k_base,
-                      "parallelism": "host cores"},
+                      "parallelism": "host cores",
+                      **({"routing": "token_choice", "k": args.tc_k,
+                          "capacity_factor": args.tc_cf} if tc else {})},
            "cpu_baseline": {"value": round(v, 2), "unit": UNIT, "cores": _cores(),
                             "kind": "oracle", "sample": desc + " per step"},
            "e2e": {"value": round(v, 2), "unit": UNIT, "h2d_bytes_per_step": 0,
@@ -461,6 +522,13 @@ def main():
     ap.add_argument("--shared-experts", type=int, default=0,
                     help="add this many shared SwiGLU experts per layer (the paper's block has 2)")
     ap.add_argument("--shared-dff", type=int, default=1024, help="width of each shared expert")
+    ap.add_argument("--routing", choices=["ec", "tc"], default="ec",
+                    help="expert choice (the paper's method) or token choice (its baseline)")
+    ap.add_argument("--tc-k", type=int, default=8, help="experts per token under --routing tc")
+    ap.add_argument("--tc-cf", type=float, default=None,
+                    help="token-choice capacity factor (default: dropless)")
+    ap.add_argument("--tc-cpu-tokens", type=int, default=32,
+                    help="tokens of the token-choice oracle's CPU sample (both arms)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-tokens", type=int, default=8192,
                     help="tokens of the oracle's CPU baseline sample")
