@@ -416,7 +416,9 @@ def run_ours(args):
         "gather": 2 * P * d * b,
         "combine": P * d * b + N * d * b,
         "bwd_gather_scale": 3 * P * d * b,
+        "gather_dy": 2 * P * d * b,
         "softmax_bwd": 3 * N * E * 4,
+        "dgate_reduce": (2 * math.ceil(w.d_ff / 256) + 1) * P * 4,
         "dx_combine": P * d * b + N * d * 4 + N * d * b,
     }
     mem_bytes = {k: v for k, v in mem_bytes.items() if k in per}   # kernels this path launches

@@ -24,6 +24,8 @@ struct ec_ctx {
   size_t o_status, o_goff, o_kg, o_koff, o_ST, o_S, o_idx, o_gate, o_slot, o_H, o_A, o_B, o_U,
       o_O, o_dO, o_dA, o_dB, o_dgate, o_dZ, o_dZb, o_wrpad, o_f32a, o_f32b, o_dXr, o_part, total;
   int wr_splits = 1;   // split-K factor of dWr = X^T dZ
+  int dg_parts = 1;    // partial sums per gate gradient (tensor-core dU epilogue)
+  size_t o_dgsum = 0;  // the gate gradients summed over their partials
   int Ep = 64;         // experts rounded up to 64 (tensor-core router operands)
   // per-kernel event timing (off by default) and kernel launch counter
   bool prof = false;
@@ -136,7 +138,10 @@ void layout(ec_ctx* c) {
   c->o_dO = take(P * d * es);
   c->o_dA = take(P * F * es);
   c->o_dB = take(P * F * es);
-  c->o_dgate = take(P * 4);
+  // bf16: the dU GEMM's epilogue leaves 2 partial gate gradients per 256-column tile
+  c->dg_parts = use_tc(c) ? 2 * ((c->F + 255) / 256) : 1;
+  c->o_dgate = take(c->dg_parts * P * 4);
+  c->o_dgsum = use_tc(c) ? take(P * 4) : c->o_dgate;
   c->o_dZ = take(N * E * 4);
   c->Ep = (c->E + 63) / 64 * 64;
   c->o_dZb = take(use_tc(c) ? 2 * N * c->Ep * 2 : 0);
@@ -291,16 +296,17 @@ const FfnNames kRouted = {"gemm_gate_up_swiglu", "gemm_down", "gemm_dgrad_up_swi
 const FfnNames kShared = {"shared_gate_up_swiglu", "shared_down", "shared_dgrad_up_swiglu",
                           "shared_dgrad_h", "shared_wgrad"};
 
+// On the tensor-core path `gate` (per row, or NULL) scales U, so O rows come out gated.
 template <typename T>
 ec_status ffn_forward(ec_ctx* c, const FfnNames& nm, const T* H, const void* Wg, const void* Wu,
                       const void* Wd, T* A, T* B, T* U, T* O, int E, int M, int F,
-                      cudaStream_t st) {
+                      cudaStream_t st, const float* gate = nullptr) {
   const int d = c->d;
   const int64_t P = (int64_t)E * M;
   if (P == 0) return EC_OK;
   int* status = at<int>(c, c->o_status);
   if (use_tc(c)) {
-    EC_KERNEL(nm.up, 1, tc_expert_up(H, Wg, Wu, A, B, U, E, M, d, F, status, st));
+    EC_KERNEL(nm.up, 1, tc_expert_up(H, Wg, Wu, A, B, U, E, M, d, F, status, st, nullptr, gate));
     EC_KERNEL(nm.down, 1, tc_expert_down(U, Wd, O, E, M, d, F, status, st));
   } else {
     float* Ag = at<float>(c, c->o_f32a);
@@ -322,11 +328,14 @@ ec_status ffn_forward(ec_ctx* c, const FfnNames& nm, const T* H, const void* Wg,
 
 // Backward of ffn_forward given dO: dU = dO.Wd^T, dA = dU*B*silu'(A), dB = dU*silu(A),
 // dH = dA.Wg^T + dB.Wu^T, dWd = U^T.dO, dWg = H^T.dA, dWu = H^T.dB (fp32, overwritten).
+// On the tensor-core path with `gate`, dO holds the ungated rows dY[idx] and U the gated
+// ones (as ffn_forward wrote them): dU = gate * dO.Wd^T, dWd = U^T.dO, and the gate
+// gradients <dO.Wd^T, silu(A) B> land in dgate_part (c->dg_parts partials, stride E*M).
 template <typename T>
 ec_status ffn_backward(ec_ctx* c, const FfnNames& nm, const T* dO, const T* H, const T* A,
                        const T* B, const T* U, const void* Wg, const void* Wu, const void* Wd,
                        T* dA, T* dB, T* dH, float* dWg, float* dWu, float* dWd, int E, int M, int F,
-                       cudaStream_t st) {
+                       cudaStream_t st, const float* gate = nullptr, float* dgate_part = nullptr) {
   const int d = c->d;
   const int64_t P = (int64_t)E * M;
   if (P == 0) {
@@ -337,7 +346,9 @@ ec_status ffn_backward(ec_ctx* c, const FfnNames& nm, const T* dO, const T* H, c
   }
   int* status = at<int>(c, c->o_status);
   if (use_tc(c)) {
-    EC_KERNEL(nm.dgrad_up, 1, tc_expert_dgrad_up(dO, Wd, A, B, dA, dB, E, M, d, F, status, st));
+    EC_KERNEL(nm.dgrad_up, 1,
+              tc_expert_dgrad_up(dO, Wd, A, B, dA, dB, E, M, d, F, status, st, nullptr, gate,
+                                 dgate_part, P));
     EC_KERNEL(nm.dgrad_h, 1, tc_expert_dgrad_h(dA, dB, Wg, Wu, dH, E, M, d, F, status, st));
     EC_KERNEL(nm.wgrad, 2,
               tc_expert_wgrad(H, U, dO, dA, dB, dWg, dWu, dWd, E, M, d, F, status, st));
@@ -399,11 +410,14 @@ ec_status run_forward(ec_ctx* c, const void* X, const void* Wg, const void* Wu, 
     Osh = o;
   }
   const int* idx = at<int>(c, c->o_idx);
+  const float* gate = at<float>(c, c->o_gate);
+  // tensor cores: the gate is applied in the gate/up epilogue (O rows come out gated)
+  const bool fused_gate = use_tc(c);
   EC_KERNEL("gather", pz, launch_gather<T>(Xt, idx, H, P, d, st));
   EC_TRY(ffn_forward<T>(c, kRouted, H, Wg, Wu, Wd, at<T>(c, c->o_A), at<T>(c, c->o_B),
-                        at<T>(c, c->o_U), O, E, M, F, st));
+                        at<T>(c, c->o_U), O, E, M, F, st, fused_gate ? gate : nullptr));
   EC_KERNEL("combine", N > 0,
-            launch_combine<T>(O, at<float>(c, c->o_gate), at<int>(c, c->o_slot),
+            launch_combine<T>(O, fused_gate ? nullptr : gate, at<int>(c, c->o_slot),
                               c->residual ? Xt : nullptr, Osh, static_cast<T*>(Y), N, E, M, d,
                               st));
   return EC_OK;
@@ -428,11 +442,19 @@ ec_status run_backward(ec_ctx* c, const void* dY, void* dX, float* dWr, float* d
   const float* gate = at<float>(c, c->o_gate);
   const int* slot = at<int>(c, c->o_slot);
 
-  EC_KERNEL("bwd_gather_scale", pz,
-            launch_bwd_gather_scale<T>(dYt, O, idx, gate, dO, dgate, P, d, st));
-  EC_TRY(ffn_backward<T>(c, kRouted, dO, at<T>(c, c->o_H), at<T>(c, c->o_A), at<T>(c, c->o_B),
-                         at<T>(c, c->o_U), c->Wg, c->Wu, c->Wd, at<T>(c, c->o_dA),
-                         at<T>(c, c->o_dB), dH, dWg, dWu, dWd, E, M, F, st));
+  if (use_tc(c)) {
+    // dO holds dY[idx] ungated; the dU epilogue applies the gate and forms dgate
+    EC_KERNEL("gather_dy", pz, launch_gather<T>(dYt, idx, dO, P, d, st));
+    EC_TRY(ffn_backward<T>(c, kRouted, dO, at<T>(c, c->o_H), at<T>(c, c->o_A), at<T>(c, c->o_B),
+                           at<T>(c, c->o_U), c->Wg, c->Wu, c->Wd, at<T>(c, c->o_dA),
+                           at<T>(c, c->o_dB), dH, dWg, dWu, dWd, E, M, F, st, gate, dgate));
+  } else {
+    EC_KERNEL("bwd_gather_scale", pz,
+              launch_bwd_gather_scale<T>(dYt, O, idx, gate, dO, dgate, P, d, st));
+    EC_TRY(ffn_backward<T>(c, kRouted, dO, at<T>(c, c->o_H), at<T>(c, c->o_A), at<T>(c, c->o_B),
+                           at<T>(c, c->o_U), c->Wg, c->Wu, c->Wd, at<T>(c, c->o_dA),
+                           at<T>(c, c->o_dB), dH, dWg, dWu, dWd, E, M, F, st));
+  }
   const T* dHsh = nullptr;
   if (Fs > 0) {
     // shared experts: dO is dY itself (no gate), the input gradient goes into the dX scatter
@@ -449,8 +471,10 @@ ec_status run_backward(ec_ctx* c, const void* dY, void* dX, float* dWr, float* d
   const T* res = c->residual ? dYt : nullptr;
   if (use_tc(c)) {
     bf16* dZb = at<bf16>(c, c->o_dZb);
+    float* dgsum = at<float>(c, c->o_dgsum);
+    EC_KERNEL("dgate_reduce", pz, launch_reduce_splits(dgate, dgsum, P, c->dg_parts, st));
     EC_KERNEL("softmax_bwd", nz,
-              launch_softmax_bwd(at<float>(c, c->o_S), slot, dgate, dZ, dZb, N, E, c->Ep, M, st));
+              launch_softmax_bwd(at<float>(c, c->o_S), slot, dgsum, dZ, dZb, N, E, c->Ep, M, st));
     EC_KERNEL("router_dgrad_gemm", nz,
               tc_router_dgrad(dZb, at<void>(c, c->o_wrpad), dXr, N, d, c->Ep, status, st));
     EC_KERNEL("dx_combine", nz,
@@ -509,10 +533,10 @@ ec_status run_tc_forward(ec_ctx* c, const void* X, const void* Wr, const float* 
   EC_KERNEL("gather", 1, launch_gather<bf16>(Xt, row_token, H, c->P_tc, d, st, count + E));
   EC_KERNEL("gemm_gate_up_swiglu", 1,
             tc_expert_up(H, Wg, Wu, at<bf16>(c, c->o_A), at<bf16>(c, c->o_B), U, E, 0, d, F,
-                         status, st, &vr));
+                         status, st, &vr, row_gate));
   EC_KERNEL("gemm_down", 1, tc_expert_down(U, Wd, O, E, 0, d, F, status, st, &vr));
   EC_KERNEL("combine", 1,
-            launch_combine<bf16>(O, row_gate, slot, c->residual ? Xt : nullptr, nullptr,
+            launch_combine<bf16>(O, nullptr, slot, c->residual ? Xt : nullptr, nullptr,
                                  static_cast<bf16*>(Y), N, E, 0, d, st));
   return EC_OK;
 }
@@ -540,12 +564,13 @@ ec_status run_tc_backward(ec_ctx* c, const void* dY, void* dX, float* dWr, float
   bf16* dB = at<bf16>(c, c->o_dB);
   float* row_dgate = at<float>(c, c->o_dgate);
   const int* slot = at<int>(c, c->o_slot);
-  EC_KERNEL("bwd_gather_scale", 1,
-            launch_bwd_gather_scale<bf16>(dYt, O, at<int>(c, c->o_idx), at<float>(c, c->o_gate), dO,
-                                          row_dgate, c->P_tc, d, st, count + E));
+  // dO = dY rows ungated; the dU epilogue applies the row gates and forms their gradients
+  EC_KERNEL("gather_dy", 1,
+            launch_gather<bf16>(dYt, at<int>(c, c->o_idx), dO, c->P_tc, d, st, count + E));
   EC_KERNEL("gemm_dgrad_up_swiglu", 1,
             tc_expert_dgrad_up(dO, c->Wd, at<bf16>(c, c->o_A), at<bf16>(c, c->o_B), dA, dB, E, 0,
-                               d, F, status, st, &vr));
+                               d, F, status, st, &vr, at<float>(c, c->o_gate), row_dgate,
+                               c->P_tc));
   EC_KERNEL("gemm_dgrad_h", 1,
             tc_expert_dgrad_h(dA, dB, c->Wg, c->Wu, dH, E, 0, d, F, status, st, &vr));
   EC_KERNEL("gemm_wgrad", 2,
@@ -555,10 +580,12 @@ ec_status run_tc_backward(ec_ctx* c, const void* dY, void* dX, float* dWr, float
   bf16* dZb = at<bf16>(c, c->o_dZb);
   float* dXr = at<float>(c, c->o_dXr);
   float* part = at<float>(c, c->o_part);
+  float* dgsum = at<float>(c, c->o_dgsum);
+  EC_KERNEL("dgate_reduce", 1, launch_reduce_splits(row_dgate, dgsum, c->P_tc, c->dg_parts, st));
   EC_KERNEL("softmax_bwd", 1,
             launch_tc_softmax_bwd(at<float>(c, c->o_S), at<int>(c, c->o_choice),
-                                  at<float>(c, c->o_tgate), at<float>(c, c->o_Zs), slot, row_dgate,
-                                  dZ, dZb, N, E, c->Ep, k, st));
+                                  at<float>(c, c->o_tgate), at<float>(c, c->o_Zs), slot, dgsum, dZ,
+                                  dZb, N, E, c->Ep, k, st));
   EC_KERNEL("router_dgrad_gemm", 1,
             tc_router_dgrad(dZb, at<void>(c, c->o_wrpad), dXr, N, d, c->Ep, status, st));
   EC_KERNEL("dx_combine", 1,

@@ -54,6 +54,13 @@ struct Args {
   const int* vm_tiles;          // [vm_E + 1] cumulative PADR-row blocks
   const int* vm_count;          // [vm_E] rows per expert
   int vm_E;
+  // Gate per row (row b*M + m of a uniform batch, the padded row of variable rows), or
+  // NULL for 1. SWIGLU_FWD writes U scaled by it; SWIGLU_BWD scales its accumulator by it
+  // and writes the row's gate gradient <acc, silu(A)*B> as partial sums (one per n-tile
+  // and column part) to dgate_part[(nt*parts + part) * dgate_stride + row].
+  const float* gate;
+  float* dgate_part;
+  int64_t dgate_stride;
 };
 
 constexpr int PADR = 256;       // row padding unit of variable-row expert regions
@@ -546,6 +553,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
       const uint32_t tacc = tmem_base + (uint32_t)(a * BN) + ((uint32_t)(q * 32) << 16);
       const int64_t row_off =
           VARM == 1 ? (int64_t)gm * p.ld : (int64_t)T.b * p.bstride + (int64_t)gm * p.ld;
+      const int64_t grow = VARM == 1 ? (int64_t)gm : (int64_t)T.b * p.M + gm;   // gate row
       // zero output: an empty expert's weight gradient, or a padding row
       const bool no_k = (VARM == 2 && T.kbl == 0) || (VARM == 1 && !row_ok);
       uint32_t v[32];
@@ -602,6 +610,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
           tmem_wait_ld();
           const int n = nt * (BN / 2) + c * 32;
           if (row_st && n < p.N) {
+            const float gs = (p.gate && row_ok) ? __ldg(p.gate + grow) : 1.0f;
             float g[32];
 #pragma unroll
             for (int i = 0; i < 32; ++i) {
@@ -612,7 +621,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
             store_bf16x32(reinterpret_cast<bf16*>(p.out0) + row_off + n, f);
             store_bf16x32(reinterpret_cast<bf16*>(p.out1) + row_off + n, g);
 #pragma unroll
-            for (int i = 0; i < 32; ++i) f[i] = f[i] * sigmoid_fast(f[i]) * g[i];
+            for (int i = 0; i < 32; ++i) f[i] = gs * (f[i] * sigmoid_fast(f[i]) * g[i]);
             store_bf16x32(reinterpret_cast<bf16*>(p.out2) + row_off + n, f);
           }
         }
@@ -632,6 +641,8 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
           }
         };
         fetch(c32, ra, rb);
+        const float gs = (p.gate && row_ok) ? __ldg(p.gate + grow) : 1.0f;
+        float dot = 0.f;   // <acc, silu(A) * B> over this warp's columns of the row
 #pragma unroll 1
         for (int c = c32; c < c32 + NC32; ++c) {
           if (c + 1 < c32 + NC32) fetch(c + 1, na, nb);
@@ -652,9 +663,11 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
             }
 #pragma unroll
             for (int i = 0; i < 32; ++i) {
-              const float du = f32(v[i]);
+              const float acc = f32(v[i]);
+              const float du = gs * acc;
               const float sg = sigmoid_fast(av[i]);
               const float das = du * sg;
+              dot = fmaf(acc, av[i] * sg * bv[i], dot);
               f[i] = das * bv[i] * fmaf(av[i], 1.0f - sg, 1.0f);
               db[i] = das * av[i];
             }
@@ -664,6 +677,8 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
 #pragma unroll
           for (int i = 0; i < 4; ++i) { ra[i] = na[i]; rb[i] = nb[i]; }
         }
+        if (p.dgate_part && row_ok)
+          p.dgate_part[(int64_t)(nt * NPART + part) * p.dgate_stride + grow] = dot;
       } else if constexpr (EPI == EPI_ROUTER) {
         const int E = p.n_valid;
         float mx = -INFINITY;
@@ -915,7 +930,7 @@ static cudaError_t launch_rows(const CUtensorMap& a0, const CUtensorMap& a1, con
 
 cudaError_t tc_expert_up(const void* H, const void* Wg, const void* Wu, void* A, void* B, void* U,
                          int E, int M, int d, int F, int* status, cudaStream_t st,
-                         const VarRows* vr) {
+                         const VarRows* vr, const float* gate) {
   CUtensorMap ma, mg, mu;
   TC_TRY(act_map(&ma, H, d, E, M, vr, BM));
   TC_TRY(make_map(&mg, Wg, F, d, E, 64));
@@ -924,6 +939,7 @@ cudaError_t tc_expert_up(const void* H, const void* Wg, const void* Wu, void* A,
   p.out0 = A;
   p.out1 = B;
   p.out2 = U;
+  p.gate = gate;
   p.ld = F;
   p.bstride = (int64_t)M * F;
   return launch_rows<256, false, true, true, false, EPI_SWIGLU_FWD>(ma, ma, mg, mu, p, vr, st);
@@ -943,7 +959,8 @@ cudaError_t tc_expert_down(const void* U, const void* Wd, void* O, int E, int M,
 
 cudaError_t tc_expert_dgrad_up(const void* dO, const void* Wd, const void* A, const void* B,
                                void* dA, void* dB, int E, int M, int d, int F, int* status,
-                               cudaStream_t st, const VarRows* vr) {
+                               cudaStream_t st, const VarRows* vr, const float* gate,
+                               float* dgate_part, int64_t dgate_stride) {
   CUtensorMap ma, mb;
   TC_TRY(act_map(&ma, dO, d, E, M, vr, BM));
   TC_TRY(make_map(&mb, Wd, d, F, E, 128));   // B[n=f][k=i] = Wd[f][i]: K-major, half per CTA
@@ -952,6 +969,9 @@ cudaError_t tc_expert_dgrad_up(const void* dO, const void* Wd, const void* A, co
   p.in1 = B;
   p.out0 = dA;
   p.out1 = dB;
+  p.gate = gate;
+  p.dgate_part = dgate_part;
+  p.dgate_stride = dgate_stride;
   p.ld = F;
   p.bstride = (int64_t)M * F;
   return launch_rows<256, false, false, false, false, EPI_SWIGLU_BWD>(ma, ma, mb, mb, p, vr, st);

@@ -26,20 +26,25 @@ cudaError_t tc_router_softmax(const void* X, const void* Wr, void* Wr_pad, const
                               float* S, float* ST, int N, int d, int E, int* status,
                               cudaStream_t st);
 
-// [A | B] = H.[Wg | Wu] per expert; U = silu(A) * B. H [E][M][d]; Wg, Wu [E][d][F];
-// A, B, U [E][M][F] bf16.
+// [A | B] = H.[Wg | Wu] per expert; U = g * silu(A) * B with g the row's gate (gate [E*M]
+// or, with vr, [P]; NULL: g = 1). H [E][M][d]; Wg, Wu [E][d][F]; A, B, U [E][M][F] bf16.
 cudaError_t tc_expert_up(const void* H, const void* Wg, const void* Wu, void* A, void* B, void* U,
                          int E, int M, int d, int F, int* status, cudaStream_t st,
-                         const VarRows* vr = nullptr);
+                         const VarRows* vr = nullptr, const float* gate = nullptr);
 
 // O = U.Wd per expert. U [E][M][F]; Wd [E][F][d]; O [E][M][d] bf16.
 cudaError_t tc_expert_down(const void* U, const void* Wd, void* O, int E, int M, int d, int F,
                            int* status, cudaStream_t st, const VarRows* vr = nullptr);
 
-// dU = dO.Wd^T per expert, then dA = dU * B * silu'(A), dB = dU * silu(A) (bf16 out).
+// dU' = dO.Wd^T per expert, dU = g dU' (g the row's gate as in tc_expert_up, NULL: 1), then
+// dA = dU * B * silu'(A), dB = dU * silu(A) (bf16 out). With dgate_part, also the row's
+// gate gradient <dU', silu(A) * B> as 2*ceil(F/256) partial sums, partial j of row r at
+// dgate_part[j * dgate_stride + r].
 cudaError_t tc_expert_dgrad_up(const void* dO, const void* Wd, const void* A, const void* B,
                                void* dA, void* dB, int E, int M, int d, int F, int* status,
-                               cudaStream_t st, const VarRows* vr = nullptr);
+                               cudaStream_t st, const VarRows* vr = nullptr,
+                               const float* gate = nullptr, float* dgate_part = nullptr,
+                               int64_t dgate_stride = 0);
 
 // dH = dA.Wg^T + dB.Wu^T per expert (one K loop over both halves). dH [E][M][d] bf16.
 cudaError_t tc_expert_dgrad_h(const void* dA, const void* dB, const void* Wg, const void* Wu,

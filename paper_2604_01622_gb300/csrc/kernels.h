@@ -43,7 +43,8 @@ cudaError_t launch_tc_softmax_bwd(const float* S, const int* choice, const float
 template <typename T>
 cudaError_t launch_gather(const T* X, const int* idx, T* H, int64_t P, int d, cudaStream_t st,
                           const int* p_used = nullptr);
-// Y_t = R_t + R2_t (each if given) + sum over the experts that chose t of gate * O row.
+// Y_t = R_t + R2_t (each if given) + sum over the experts that chose t of gate * O row
+// (gate NULL: 1, for O rows already scaled by their gates).
 template <typename T>
 cudaError_t launch_combine(const T* O, const float* gate, const int* slot, const T* R, const T* R2,
                            T* Y, int N, int E, int M, int d, cudaStream_t st);

@@ -59,7 +59,7 @@ __device__ __forceinline__ int token_pairs(const int* __restrict__ slot, const f
         const int p = cnt + __popc(ball & ((1u << lane) - 1u));
         s_e[p] = e;
         s_m[p] = m;
-        if (s_g) s_g[p] = gate[(size_t)e * M + m];
+        if (s_g) s_g[p] = gate ? gate[(size_t)e * M + m] : 1.0f;
       }
       cnt += __popc(ball);
     }
@@ -175,29 +175,40 @@ cudaError_t launch_bwd_gather_scale(const T* dY, const T* O, const int* idx, con
 // lo = bf16(dZ - hi), zero in the padding columns E..Ep-1: the tensor-core operands of the
 // router-gradient GEMMs, which sum the products of both planes (hi + lo carries dZ to
 // about 16 significant bits, so the GEMMs keep near-fp32 accuracy).
+// One warp per token; lane l holds experts l, l+32, ... (E <= 512) in registers.
 __global__ void softmax_bwd_kernel(const float* __restrict__ S, const int* __restrict__ slot,
                                    const float* __restrict__ dgate, float* __restrict__ dZ,
                                    bf16* __restrict__ dZb, int N, int E, int Ep, int M) {
+  constexpr int MAXC = 16;
   const int t = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (t >= N) return;
+  float ds[MAXC], sv[MAXC];
   float dot = 0.f;
-  for (int e = lane; e < E; e += 32) {
-    const int m = slot[(size_t)t * E + e];
-    const float ds = m >= 0 ? dgate[(size_t)e * M + m] : 0.f;
-    dot = fmaf(ds, S[(size_t)t * E + e], dot);
+#pragma unroll
+  for (int i = 0; i < MAXC; ++i) {
+    const int e = lane + 32 * i;
+    ds[i] = 0.f;
+    sv[i] = 0.f;
+    if (e < E) {
+      const int m = slot[(size_t)t * E + e];
+      ds[i] = m >= 0 ? dgate[(size_t)e * M + m] : 0.f;
+      sv[i] = S[(size_t)t * E + e];
+      dot = fmaf(ds[i], sv[i], dot);
+    }
   }
   dot = warp_sum(dot);
-  for (int e = lane; e < E; e += 32) {
-    const int m = slot[(size_t)t * E + e];
-    const float ds = m >= 0 ? dgate[(size_t)e * M + m] : 0.f;
-    const float s = S[(size_t)t * E + e];
-    const float z = s * (ds - dot);
-    dZ[(size_t)t * E + e] = z;
-    if (dZb) {
-      const bf16 hi = __float2bfloat16_rn(z);
-      dZb[(size_t)t * Ep + e] = hi;
-      dZb[(size_t)N * Ep + (size_t)t * Ep + e] = __float2bfloat16_rn(z - __bfloat162float(hi));
+#pragma unroll
+  for (int i = 0; i < MAXC; ++i) {
+    const int e = lane + 32 * i;
+    if (e < E) {
+      const float z = sv[i] * (ds[i] - dot);
+      dZ[(size_t)t * E + e] = z;
+      if (dZb) {
+        const bf16 hi = __float2bfloat16_rn(z);
+        dZb[(size_t)t * Ep + e] = hi;
+        dZb[(size_t)N * Ep + (size_t)t * Ep + e] = __float2bfloat16_rn(z - __bfloat162float(hi));
+      }
     }
   }
   if (dZb)
@@ -210,6 +221,7 @@ __global__ void softmax_bwd_kernel(const float* __restrict__ S, const int* __res
 cudaError_t launch_softmax_bwd(const float* S, const int* slot, const float* dgate, float* dZ,
                                bf16* dZb, int N, int E, int Ep, int M, cudaStream_t st) {
   if (N == 0) return cudaSuccess;
+  if (E > 512) return cudaErrorInvalidValue;
   softmax_bwd_kernel<<<(N + 7) / 8, 256, 0, st>>>(S, slot, dgate, dZ, dZb, N, E, Ep, M);
   return cudaGetLastError();
 }

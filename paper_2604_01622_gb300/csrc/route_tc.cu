@@ -168,7 +168,8 @@ cudaError_t launch_tc_route(const float* S, int N, int E, int k, int cap, int* c
 
 // Gradient through the normalised gates and the softmax, one warp per token:
 // dS_tj = (dg_tj - sum_{j' kept} dg_tj' g_tj') / Z_t for the k chosen j (dg = 0 if dropped),
-// dZ = S * (dS - <dS, S>). dg comes from the per-row gate gradients through the slot map.
+// dZ = S * (dS - <dS, S>). dg comes from the per-row gate gradients through the slot map;
+// lane r < k holds the token's r-th choice.
 __global__ void tc_softmax_bwd_kernel(const float* __restrict__ S, const int* __restrict__ choice,
                                       const float* __restrict__ tgate, const float* __restrict__ Z,
                                       const int* __restrict__ slot,
@@ -177,33 +178,27 @@ __global__ void tc_softmax_bwd_kernel(const float* __restrict__ S, const int* __
   const int t = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (t >= N) return;
-  float common = 0.f;
-  for (int r = 0; r < k; ++r) {
-    const int e = choice[(size_t)t * k + r];
-    const int row = slot[(size_t)t * E + e];
-    if (row >= 0) common += row_dgate[row] * tgate[(size_t)t * k + r];
+  int my_e = -1;
+  float dg = 0.f, g = 0.f, s_e = 0.f;
+  if (lane < k) {
+    my_e = choice[(size_t)t * k + lane];
+    const int row = slot[(size_t)t * E + my_e];
+    dg = row >= 0 ? row_dgate[row] : 0.f;
+    g = tgate[(size_t)t * k + lane];
+    s_e = S[(size_t)t * E + my_e];
   }
-  const float invZ = 1.0f / Z[t];
-  float dot = 0.f;
-  for (int e = lane; e < E; e += 32) {
+  const float common = warp_sum(dg * g);
+  const float my_ds = lane < k ? (dg - common) / Z[t] : 0.f;
+  const float dot = warp_sum(my_ds * s_e);
+  for (int e = lane; e < Ep; e += 32) {   // Ep is a multiple of 32: every lane iterates alike
     float ds = 0.f;
-    for (int r = 0; r < k; ++r)
-      if (choice[(size_t)t * k + r] == e) {
-        const int row = slot[(size_t)t * E + e];
-        ds = ((row >= 0 ? row_dgate[row] : 0.f) - common) * invZ;
-      }
-    dot = fmaf(ds, S[(size_t)t * E + e], dot);
-  }
-  dot = warp_sum(dot);
-  for (int e = lane; e < Ep; e += 32) {
+    for (int r = 0; r < k; ++r) {
+      const int er = __shfl_sync(0xffffffffu, my_e, r);
+      const float dr = __shfl_sync(0xffffffffu, my_ds, r);
+      if (er == e) ds = dr;
+    }
     float z = 0.f;
     if (e < E) {
-      float ds = 0.f;
-      for (int r = 0; r < k; ++r)
-        if (choice[(size_t)t * k + r] == e) {
-          const int row = slot[(size_t)t * E + e];
-          ds = ((row >= 0 ? row_dgate[row] : 0.f) - common) * invZ;
-        }
       z = S[(size_t)t * E + e] * (ds - dot);
       dZ[(size_t)t * E + e] = z;
     }
@@ -220,6 +215,7 @@ cudaError_t launch_tc_softmax_bwd(const float* S, const int* choice, const float
                                   float* dZ, bf16* dZb, int N, int E, int Ep, int k,
                                   cudaStream_t st) {
   if (N == 0) return cudaSuccess;
+  if (k > 32 || Ep % 32) return cudaErrorInvalidValue;
   tc_softmax_bwd_kernel<<<(N + 7) / 8, 256, 0, st>>>(S, choice, tgate, Z, slot, row_dgate, dZ, dZb,
                                                      N, E, Ep, k);
   return cudaGetLastError();
