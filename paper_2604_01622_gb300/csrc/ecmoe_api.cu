@@ -45,7 +45,7 @@ struct ec_ctx {
   // token choice (k > 0): k experts per token, per-expert cap (< 0: none), padded rows
   int tc_k = 0, tc_cap = -1;
   int64_t P_tc = 0;
-  size_t o_choice = 0, o_tgate = 0, o_Zs = 0, o_count = 0, o_tiles = 0, o_kept = 0;
+  size_t o_choice = 0, o_tgate = 0, o_Zs = 0, o_count = 0, o_tiles = 0, o_kept = 0, o_tcscr = 0;
   std::string err;
 };
 
@@ -122,6 +122,7 @@ void layout(ec_ctx* c) {
   c->o_Zs = take(c->tc_k ? N * 4 : 0);
   c->o_count = take(c->tc_k ? (E + 1) * 4 : 0);
   c->o_tiles = take(c->tc_k ? (E + 1) * 4 : 0);
+  c->o_tcscr = take(c->tc_k ? (size_t)tc_route_scratch_ints((int)N, (int)E) * 4 : 0);
   c->o_goff = take((G + 1) * 4);
   c->o_kg = take(G * 4);
   c->o_koff = take((G + 1) * 4);
@@ -525,10 +526,11 @@ ec_status run_tc_forward(ec_ctx* c, const void* X, const void* Wr, const float* 
   EC_KERNEL("router_gemm_softmax", 2,
             tc_router_softmax(X, Wr, at<void>(c, c->o_wrpad), br, S, at<float>(c, c->o_ST), N, d,
                               E, status, st));
-  EC_KERNEL("tc_route", 4,
+  EC_KERNEL("tc_route", 5,
             launch_tc_route(S, N, E, k, c->tc_cap, at<int>(c, c->o_choice),
                             at<float>(c, c->o_tgate), at<float>(c, c->o_Zs), count, tiles,
-                            row_token, row_gate, slot, at<int>(c, c->o_kept), st));
+                            row_token, row_gate, slot, at<int>(c, c->o_kept),
+                            at<int>(c, c->o_tcscr), st));
   const VarRows vr{tiles, count, (int)c->P_tc};
   EC_KERNEL("gather", 1, launch_gather<bf16>(Xt, row_token, H, c->P_tc, d, st, count + E));
   EC_KERNEL("gemm_gate_up_swiglu", 1,

@@ -22,14 +22,17 @@ cudaError_t launch_topk(const float* ST, int N, int E, int G, const int* group_o
 // Row top-k of S [N][E] (k <= 32, E <= 512), per-expert counts capped at cap (cap < 0:
 // dropless), padded expert regions (tiles[e] in 256-row blocks), row->token map (-1 in
 // padding), row gates, slot map [N][E] (absolute row or -1) and kept flags [N][k].
-// Token-choice routing of the scores S [N][E] (k <= 32, E <= 512; cap < 0: no cap):
+// Token-choice routing of the scores S [N][E] (k <= 32, E <= 256; cap < 0: no cap):
 // choice/tgate/kept [N][k] (experts best first, normalised gates, kept flags), Z [N] (sum of
 // the k chosen scores), count [E+1] (kept rows per expert; count[E] = padded rows in use),
 // tiles [E+1] (cumulative 256-row blocks), row_token/row_gate [P] per padded row (-1 / 0 in
 // padding), slot [N][E] absolute padded row of each kept pair, else -1.
+// scratch: tc_route_scratch_ints(N, E) ints. Five kernels (and a memset of slot).
 cudaError_t launch_tc_route(const float* S, int N, int E, int k, int cap, int* choice,
                             float* tgate, float* Z, int* count, int* tiles, int* row_token,
-                            float* row_gate, int* slot, int* kept, cudaStream_t st);
+                            float* row_gate, int* slot, int* kept, int* scratch,
+                            cudaStream_t st);
+int64_t tc_route_scratch_ints(int N, int E);
 // Router gradient of token choice: dZ [N][E] (and optionally the bf16 hi/lo planes
 // dZb [2][N][Ep]) from the per-row gate gradients row_dgate [P].
 cudaError_t launch_tc_softmax_bwd(const float* S, const int* choice, const float* tgate,

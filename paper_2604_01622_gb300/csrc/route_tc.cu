@@ -80,73 +80,139 @@ __global__ void tc_topk_rows_kernel(const float* __restrict__ S, int N, int E, i
   if (lane == 0) Z[t] = sum;
 }
 
-// Per expert (one CTA): how many tokens chose it.
-__global__ void tc_count_kernel(const int* __restrict__ choice, int N, int k,
-                                int* __restrict__ count) {
-  __shared__ int s_warp[33];
-  __shared__ int s_total;
-  const int e = blockIdx.x;
-  int c = 0;
-  for (int t = threadIdx.x; t < N; t += blockDim.x)
-    for (int r = 0; r < k; ++r) c += choice[(size_t)t * k + r] == e;
-  int tot;
-  block_scan_excl(c, s_warp, &tot);
-  if (threadIdx.x == 0) {
-    s_total = tot;
-    count[e] = s_total;
-  }
-}
+// The position of token t in expert e's list is the number of tokens before t that chose
+// e: an exclusive scan, in token order, of the 0/1 column "chose e". It is done in three
+// levels: warp ballots within each 256-token block, warps within the block, blocks.
+constexpr int kRankBlock = 256;   // tokens per ranking block (8 warps)
+constexpr int kMaxE = 256;        // experts the ranking handles (8 mask words)
 
-// One thread: kept rows per expert (capped), padded region offsets in PADR-row blocks,
-// and in count[E] the padded rows in use.
-__global__ void tc_offsets_kernel(int E, int cap, int* __restrict__ count,
-                                  int* __restrict__ tiles) {
-  if (threadIdx.x != 0 || blockIdx.x != 0) return;
-  int acc = 0;
-  tiles[0] = 0;
-  for (int e = 0; e < E; ++e) {
-    int c = count[e];
-    if (cap >= 0 && c > cap) c = cap;
-    count[e] = c;
-    acc += (c + kPadRows - 1) / kPadRows;
-    tiles[e + 1] = acc;
-  }
-  count[E] = acc * kPadRows;
-}
-
-// Per expert (one CTA): walk tokens in order, give the first count[e] that chose e their rows
-// (row-to-token map, gate, slot map), mark the rest dropped, zero-fill the padding rows.
-__global__ void tc_fill_kernel(const int* __restrict__ choice, const float* __restrict__ tgate,
-                               int N, int E, int k, const int* __restrict__ count,
-                               const int* __restrict__ tiles, int* __restrict__ row_token,
-                               float* __restrict__ row_gate, int* __restrict__ slot,
-                               int* __restrict__ kept) {
-  __shared__ int s_warp[33];
-  const int e = blockIdx.x;
-  const int kept_e = count[e];
-  const int base = tiles[e] * kPadRows;
-  const int end = tiles[e + 1] * kPadRows;
-  int before = 0;   // tokens that chose e in earlier chunks
-  for (int t0 = 0; t0 < N; t0 += blockDim.x) {
-    const int t = t0 + threadIdx.x;
-    int r_hit = -1;
-    if (t < N)
-      for (int r = 0; r < k; ++r)
-        if (choice[(size_t)t * k + r] == e) r_hit = r;
-    int chunk_total;
-    const int pos = before + block_scan_excl(r_hit >= 0, s_warp, &chunk_total);
-    if (r_hit >= 0) {
-      const bool keep = pos < kept_e;
-      kept[(size_t)t * k + r_hit] = keep;
-      if (keep) {
-        row_token[base + pos] = t;
-        row_gate[base + pos] = tgate[(size_t)t * k + r_hit];
-        slot[(size_t)t * E + e] = base + pos;
-      }
+// Per 256-token block: hist[blk][e] = tokens of the block that chose e; for each chosen
+// (t, e), slot[t][e] = rank of t among the block's tokens that chose e (made absolute by
+// tc_fill_kernel). slot holds -1 elsewhere.
+__global__ void __launch_bounds__(kRankBlock)
+tc_rank_kernel(const int* __restrict__ choice, int N, int E, int k, int* __restrict__ slot,
+               int* __restrict__ hist) {
+  __shared__ int s_cnt[kRankBlock / 32][kMaxE];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int t = blockIdx.x * kRankBlock + threadIdx.x;
+  uint32_t mask[kMaxE / 32];
+#pragma unroll
+  for (int w = 0; w < kMaxE / 32; ++w) mask[w] = 0u;
+  if (t < N)
+    for (int r = 0; r < k; ++r) {
+      const int e = choice[(size_t)t * k + r];
+#pragma unroll
+      for (int w = 0; w < kMaxE / 32; ++w)
+        if ((e >> 5) == w) mask[w] |= 1u << (e & 31);
     }
-    before += chunk_total;
+  const uint32_t lt = (1u << lane) - 1u;
+  // pass 1: per-warp counts
+#pragma unroll
+  for (int w = 0; w < kMaxE / 32; ++w) {
+    const uint32_t m = mask[w];
+    const int nb = min(32, E - 32 * w);   // experts in this mask word (<= 0: none)
+    for (int b = 0; b < nb; ++b) {
+      const uint32_t bal = __ballot_sync(0xffffffffu, (m >> b) & 1u);
+      if (lane == 0) s_cnt[warp][32 * w + b] = __popc(bal);
+    }
   }
-  for (int row = base + kept_e + threadIdx.x; row < end; row += blockDim.x) {
+  __syncthreads();
+  // warp offsets within the block, block totals
+  for (int e = threadIdx.x; e < E; e += kRankBlock) {
+    int acc = 0;
+#pragma unroll
+    for (int w = 0; w < kRankBlock / 32; ++w) {
+      const int c = s_cnt[w][e];
+      s_cnt[w][e] = acc;
+      acc += c;
+    }
+    hist[(size_t)blockIdx.x * E + e] = acc;
+  }
+  __syncthreads();
+  // pass 2: ranks
+#pragma unroll
+  for (int w = 0; w < kMaxE / 32; ++w) {
+    const uint32_t m = mask[w];
+    const int nb = min(32, E - 32 * w);
+    for (int b = 0; b < nb; ++b) {
+      const bool mine = (m >> b) & 1u;
+      const uint32_t bal = __ballot_sync(0xffffffffu, mine);
+      if (mine) slot[(size_t)t * E + 32 * w + b] = s_cnt[warp][32 * w + b] + __popc(bal & lt);
+    }
+  }
+}
+
+// One CTA per expert: boff[blk][e] = tokens of earlier blocks that chose e (exclusive scan
+// over the blocks), total[e] = all tokens that chose e.
+__global__ void tc_block_scan_kernel(const int* __restrict__ hist, int nblk, int E,
+                                     int* __restrict__ boff, int* __restrict__ total) {
+  __shared__ int s_warp[33];
+  const int e = blockIdx.x;
+  int carry = 0;
+  for (int b0 = 0; b0 < nblk; b0 += blockDim.x) {
+    const int b = b0 + threadIdx.x;
+    const int h = b < nblk ? hist[(size_t)b * E + e] : 0;
+    int chunk;
+    const int ex = block_scan_excl(h, s_warp, &chunk);
+    if (b < nblk) boff[(size_t)b * E + e] = carry + ex;
+    carry += chunk;
+  }
+  if (threadIdx.x == 0) total[e] = carry;
+}
+
+// One CTA (E <= blockDim): kept rows per expert count[e] = min(total, cap) (cap < 0: no cap),
+// padded regions tiles[e] (cumulative 256-row blocks, tiles[E] the total) and in count[E]
+// the padded rows in use.
+__global__ void tc_offsets_kernel(int E, int cap, const int* __restrict__ total,
+                                  int* __restrict__ count, int* __restrict__ tiles) {
+  __shared__ int s_warp[33];
+  const int e = threadIdx.x;
+  int c = e < E ? total[e] : 0;
+  if (cap >= 0 && c > cap) c = cap;
+  const int nb = (c + kPadRows - 1) / kPadRows;
+  int all;
+  const int off = block_scan_excl(nb, s_warp, &all);
+  if (e < E) {
+    count[e] = c;
+    tiles[e] = off;
+  }
+  if (threadIdx.x == 0) {
+    tiles[E] = all;
+    count[E] = all * kPadRows;
+  }
+}
+
+// One thread per (token, choice) pair: absolute position, keep/drop, row maps; then one
+// thread per possible padding row of each expert: row_token -1, gate 0.
+__global__ void tc_fill_kernel(const int* __restrict__ choice, const float* __restrict__ tgate,
+                               int N, int E, int k, const int* __restrict__ boff,
+                               const int* __restrict__ count, const int* __restrict__ tiles,
+                               int* __restrict__ row_token, float* __restrict__ row_gate,
+                               int* __restrict__ slot, int* __restrict__ kept) {
+  const int64_t j = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const int64_t NK = (int64_t)N * k;
+  if (j < NK) {
+    const int t = (int)(j / k);
+    const int e = choice[j];
+    int* sl = slot + (size_t)t * E + e;
+    const int pos = boff[(size_t)(t / kRankBlock) * E + e] + *sl;
+    const bool keep = pos < count[e];
+    kept[j] = keep;
+    if (keep) {
+      const int row = tiles[e] * kPadRows + pos;
+      *sl = row;
+      row_token[row] = t;
+      row_gate[row] = tgate[j];
+    } else {
+      *sl = -1;
+    }
+    return;
+  }
+  const int64_t q = j - NK;
+  const int e = (int)(q / kPadRows);
+  if (e >= E) return;
+  const int row = tiles[e] * kPadRows + count[e] + (int)(q % kPadRows);
+  if (row < tiles[e + 1] * kPadRows) {
     row_token[row] = -1;
     row_gate[row] = 0.f;
   }
@@ -154,16 +220,30 @@ __global__ void tc_fill_kernel(const int* __restrict__ choice, const float* __re
 
 cudaError_t launch_tc_route(const float* S, int N, int E, int k, int cap, int* choice,
                             float* tgate, float* Z, int* count, int* tiles, int* row_token,
-                            float* row_gate, int* slot, int* kept, cudaStream_t st) {
+                            float* row_gate, int* slot, int* kept, int* scratch,
+                            cudaStream_t st) {
   if (N == 0) return cudaSuccess;
-  cudaError_t e = cudaMemsetAsync(slot, 0xFF, (size_t)N * E * sizeof(int), st);   // -1
-  if (e != cudaSuccess) return e;
+  if (E > kMaxE || k > 32 || k > E) return cudaErrorInvalidValue;
+  const int nblk = (N + kRankBlock - 1) / kRankBlock;
+  int* hist = scratch;                          // [nblk][E]
+  int* boff = scratch + (size_t)nblk * E;       // [nblk][E]
+  int* total = boff + (size_t)nblk * E;         // [E]
+  cudaError_t err = cudaMemsetAsync(slot, 0xFF, (size_t)N * E * sizeof(int), st);   // -1
+  if (err != cudaSuccess) return err;
   tc_topk_rows_kernel<<<(N + 7) / 8, 256, 0, st>>>(S, N, E, k, choice, tgate, Z);
-  tc_count_kernel<<<E, 512, 0, st>>>(choice, N, k, count);
-  tc_offsets_kernel<<<1, 32, 0, st>>>(E, cap, count, tiles);
-  tc_fill_kernel<<<E, 512, 0, st>>>(choice, tgate, N, E, k, count, tiles, row_token, row_gate,
-                                    slot, kept);
+  tc_rank_kernel<<<nblk, kRankBlock, 0, st>>>(choice, N, E, k, slot, hist);
+  tc_block_scan_kernel<<<E, 256, 0, st>>>(hist, nblk, E, boff, total);
+  tc_offsets_kernel<<<1, kMaxE, 0, st>>>(E, cap, total, count, tiles);
+  const int64_t threads = (int64_t)N * k + (int64_t)E * kPadRows;
+  tc_fill_kernel<<<(unsigned)((threads + 255) / 256), 256, 0, st>>>(
+      choice, tgate, N, E, k, boff, count, tiles, row_token, row_gate, slot, kept);
   return cudaGetLastError();
+}
+
+// Scratch ints launch_tc_route needs for N tokens and E experts.
+int64_t tc_route_scratch_ints(int N, int E) {
+  const int64_t nblk = (N + kRankBlock - 1) / kRankBlock;
+  return 2 * nblk * E + E;
 }
 
 // Gradient through the normalised gates and the softmax, one warp per token:
