@@ -176,8 +176,12 @@ __device__ __forceinline__ void cluster_sync() {
   asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" :::
                    "memory");
 }
+// Arrive on an mbarrier of either CTA of the cluster. Release at CTA scope: the arrival only
+// tells the MMA issuer that this warp's TMEM loads have completed (tcgen05.wait::ld ran
+// before it), so the warp's earlier global stores need not be made visible cluster-wide
+// first (a cluster-scope release would stall on them).
 __device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {
-  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr)
+  asm volatile("mbarrier.arrive.release.cta.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr)
                : "memory");
 }
 // TMA load whose completion is signalled on an mbarrier of either CTA of the pair.

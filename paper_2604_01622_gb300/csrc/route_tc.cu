@@ -42,40 +42,56 @@ __device__ __forceinline__ int block_scan_excl(int v, int* s_warp, int* total) {
 }
 }  // namespace
 
-// One warp per token: k rounds of a warp argmax over the E scores (larger score first, then
-// lower expert index). Writes the choices best first, normalised gates and their sum Z.
+// Order-preserving unsigned key of a score (larger score, larger key; -0 == +0; NaN ranks
+// with -inf). Key 0 is below every score: it marks an expert already taken.
+__device__ __forceinline__ uint32_t score_key(float v) {
+  v = v + 0.0f;
+  if (v != v) v = -INFINITY;
+  const uint32_t u = __float_as_uint(v);
+  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+
+// One warp per token, lane l holding experts l, l+32, ... (E <= 256) in registers: k rounds
+// of a warp argmax (largest key by a max-reduction, then the lowest expert index holding
+// it by a min-reduction). Writes the choices best first, the normalised gates and their
+// sum Z (summed in choice order).
 __global__ void tc_topk_rows_kernel(const float* __restrict__ S, int N, int E, int k,
                                     int* __restrict__ choice, float* __restrict__ tgate,
                                     float* __restrict__ Z) {
+  constexpr int MAXC = 8;
   const int t = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (t >= N) return;
   const float* row = S + (size_t)t * E;
-  uint32_t taken[16] = {};   // bit e%32 of word e/32: expert e already chosen (E <= 512)
-  float sum = 0.f;
-  int my_e = 0;              // lane r keeps the r-th choice
-  for (int r = 0; r < k; ++r) {
-    float best = -INFINITY;
-    int bi = 0x7fffffff;
-    for (int e = lane; e < E; e += 32) {
-      if (taken[e >> 5] & (1u << (e & 31))) continue;
-      float v = row[e] + 0.0f;
-      if (v != v) v = -INFINITY;   // a NaN score ranks last, so every round finds an expert
-      if (v > best || (v == best && e < bi)) { best = v; bi = e; }
-    }
+  float val[MAXC];
+  uint32_t key[MAXC];
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      const float ov = __shfl_xor_sync(0xffffffffu, best, o);
-      const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
-      if (ov > best || (ov == best && oi < bi)) { best = ov; bi = oi; }
-    }
-    taken[bi >> 5] |= 1u << (bi & 31);   // every lane holds the same winner
-    if (lane == r) my_e = bi;
-    sum += row[bi];
+  for (int i = 0; i < MAXC; ++i) {
+    const int e = lane + 32 * i;
+    val[i] = e < E ? row[e] : 0.f;
+    key[i] = e < E ? score_key(val[i]) : 0u;
+  }
+  float sum = 0.f, my_v = 0.f;
+  int my_e = 0;   // lane r keeps the r-th choice
+  for (int r = 0; r < k; ++r) {
+    uint32_t best = 0u;
+    int bi = 0x7fffffff;
+#pragma unroll
+    for (int i = 0; i < MAXC; ++i)          // ascending expert index: ties keep the first
+      if (key[i] > best) { best = key[i]; bi = lane + 32 * i; }
+    const uint32_t m = __reduce_max_sync(0xffffffffu, best);
+    const int e = (int)__reduce_min_sync(0xffffffffu, best == m ? (uint32_t)bi : 0x7fffffffu);
+    float v = 0.f;
+#pragma unroll
+    for (int i = 0; i < MAXC; ++i)
+      if (lane + 32 * i == e) { v = val[i]; key[i] = 0u; }
+    v = __shfl_sync(0xffffffffu, v, e & 31);
+    if (lane == r) { my_e = e; my_v = v; }
+    sum += v;
   }
   if (lane < k) {
     choice[(size_t)t * k + lane] = my_e;
-    tgate[(size_t)t * k + lane] = row[my_e] / sum;
+    tgate[(size_t)t * k + lane] = my_v / sum;
   }
   if (lane == 0) Z[t] = sum;
 }
