@@ -265,10 +265,14 @@ __host__ __device__ constexpr uint32_t tmem_cols() {
   return 2 * BN <= 32 ? 32 : 2 * BN <= 64 ? 64 : 2 * BN <= 128 ? 128 : 2 * BN <= 256 ? 256 : 512;
 }
 
-template <int BN, int STAGES, bool PAIR>
+// Epilogue staging: one 4 KB buffer per epilogue warp (a 32 x 32 fp32 chunk, or two 32 x 32
+// bf16 chunks), written by the warp and stored to global memory by TMA.
+constexpr uint32_t STAGE_BUF = 4096;
+
+template <int BN, int STAGES, bool PAIR, int EPW, bool STAGED>
 __host__ __device__ constexpr uint32_t smem_bytes() {
   return 1024 /*align slack*/ + STAGES * (BM * BK * 2 + (PAIR ? BN / 2 : BN) * BK * 2) +
-         256 /*barriers*/;
+         (STAGED ? EPW * STAGE_BUF : 0) + 256 /*barriers*/;
 }
 
 __device__ __forceinline__ float f32(uint32_t u) { return __uint_as_float(u); }
@@ -282,13 +286,43 @@ __device__ __forceinline__ float sigmoid_fast(float a) {
   return fmaf(0.5f, t, 0.5f);
 }
 
-__device__ __forceinline__ void store_bf16x32(void* dst, const float* v) {
-  uint4* d = reinterpret_cast<uint4*>(dst);
+// Stage this thread's row (row r of the warp's 32) of a 32 x 32 chunk for a TMA store:
+// fp32 rows of 128 bytes in the 128-byte swizzle, bf16 rows of 64 bytes in the 64-byte
+// swizzle (16-byte unit j of row r at unit j ^ (row bits of the address)), so the warp's
+// 16-byte shared stores are free of bank conflicts.
+__device__ __forceinline__ void stage_f32(uint8_t* buf, int r, const float* v) {
 #pragma unroll
-  for (int i = 0; i < 4; ++i)
-    d[i] = make_uint4(pack_bf16x2(v[8 * i], v[8 * i + 1]), pack_bf16x2(v[8 * i + 2], v[8 * i + 3]),
-                      pack_bf16x2(v[8 * i + 4], v[8 * i + 5]),
-                      pack_bf16x2(v[8 * i + 6], v[8 * i + 7]));
+  for (int j = 0; j < 8; ++j)
+    *reinterpret_cast<float4*>(buf + r * 128 + ((j ^ (r & 7)) << 4)) =
+        make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+}
+__device__ __forceinline__ void stage_bf16(uint8_t* buf, int r, const float* v) {
+#pragma unroll
+  for (int j = 0; j < 4; ++j)
+    *reinterpret_cast<uint4*>(buf + r * 64 + ((j ^ ((r >> 1) & 3)) << 4)) =
+        make_uint4(pack_bf16x2(v[8 * j], v[8 * j + 1]), pack_bf16x2(v[8 * j + 2], v[8 * j + 3]),
+                   pack_bf16x2(v[8 * j + 4], v[8 * j + 5]),
+                   pack_bf16x2(v[8 * j + 6], v[8 * j + 7]));
+}
+__device__ __forceinline__ void fence_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+__device__ __forceinline__ void tma_store_3d(const CUtensorMap* map, uint32_t src, int c0, int c1,
+                                             int c2) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%2, %3, %4}], [%1];" ::"l"(
+          reinterpret_cast<uint64_t>(map)),
+      "r"(src), "r"(c0), "r"(c1), "r"(c2)
+      : "memory");
+  asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+}
+// Wait until at most N of this thread's bulk store groups still read shared memory.
+template <int N>
+__device__ __forceinline__ void bulk_wait_read() {
+  asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(N) : "memory");
+}
+__device__ __forceinline__ void bulk_wait_all() {
+  asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
 }
 
 // ------------------------------------------------------------------ tile decode
@@ -349,7 +383,8 @@ template <int BN, bool A_MN, bool B_MN, bool B_SPLIT, bool K_SPLIT, int EPI, int
 __global__ void __launch_bounds__(64 + 32 * EPW, 1)
 tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ CUtensorMap mA1,
                const __grid_constant__ CUtensorMap mB0, const __grid_constant__ CUtensorMap mB1,
-               const Args p) {
+               const __grid_constant__ CUtensorMap mO0, const __grid_constant__ CUtensorMap mO1,
+               const __grid_constant__ CUtensorMap mO2, const Args p) {
   constexpr int BNL = PAIR ? BN / 2 : BN;     // B columns held by this CTA
   constexpr int TM = PAIR ? 2 * BM : BM;      // tile rows
   constexpr uint32_t A_BYTES = BM * BK * 2;
@@ -360,13 +395,16 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
   static_assert(!PAIR || BN % 128 == 0, "pair tiles split B in two 64-column multiples");
   static_assert(EPW == 4 || EPW == 8, "epilogue warps: one or two per TMEM lane quarter");
   static_assert(EPI != EPI_ROUTER || EPW == 4, "the row softmax needs whole rows per thread");
+  // every epilogue except the router's writes through shared memory and TMA stores
+  constexpr bool STAGED = EPI != EPI_ROUTER;
 
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
   uint8_t* sA = smem;
   uint8_t* sB = smem + STAGES * A_BYTES;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sB + STAGES * B_BYTES);
+  uint8_t* sStage = sB + STAGES * B_BYTES;   // 1024-aligned: A_BYTES, B_BYTES are multiples
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sStage + (STAGED ? EPW * STAGE_BUF : 0));
   uint64_t* full = bars;
   uint64_t* empty = bars + STAGES;
   uint64_t* tfull = bars + 2 * STAGES;
@@ -398,6 +436,12 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
     prefetch_map(&mB0);
     if (K_SPLIT) prefetch_map(&mA1);
     if (K_SPLIT || B_SPLIT) prefetch_map(&mB1);
+  }
+  if (STAGED && warp >= 2 && lane == 0) {
+    prefetch_map(&mO0);
+    if (EPI == EPI_SWIGLU_FWD || EPI == EPI_SWIGLU_BWD || EPI == EPI_STORE_F32_SPLIT)
+      prefetch_map(&mO1);
+    if (EPI == EPI_SWIGLU_FWD) prefetch_map(&mO2);
   }
   if (warp == 1) {
     if constexpr (PAIR) tmem_alloc_pair(tmem_holder, TCOLS);
@@ -540,6 +584,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
     const int r = q * 32 + lane;        // row within the tile
     constexpr int NPART = EPW / 4;      // warps sharing a lane quarter split the columns
     const int part = (warp - 2) / 4;
+    int slot = 0;   // staging half of the next bf16 chunk (warp-uniform)
     int it = 0;
     for (int tile = cid; tile < total; tile += nwalk, ++it) {
       const int a = it & 1;
@@ -553,7 +598,6 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
       // Variable rows: a 256-row tile never leaves its expert's padded region, and the
       // region's unused rows are written as zeros (the weight gradients run their K loop
       // over them). Uniform batches store only the valid rows.
-      const bool row_st = VARM == 1 ? true : row_ok;
       const uint32_t tacc = tmem_base + (uint32_t)(a * BN) + ((uint32_t)(q * 32) << 16);
       const int64_t row_off =
           VARM == 1 ? (int64_t)gm * p.ld : (int64_t)T.b * p.bstride + (int64_t)gm * p.ld;
@@ -563,6 +607,32 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
       uint32_t v[32];
       float f[32];
 
+      // Outputs leave through the warp's staging buffer: the warp writes a 32-row x 32-column
+      // chunk (thread = row) into shared memory and lane 0 stores it with one TMA copy, which
+      // also clips the rows past the tensor's end (rows that are not valid in a uniform batch).
+      const int srow = T.row0 + q * 32;                    // first row of the warp's block
+      const int sbat = VARM == 1 ? 0 : T.b;                // batch coordinate of the output
+      const bool st_any = VARM == 1 || T.valid > q * 32;   // the block has a row to store
+      auto put_bf16 = [&](const CUtensorMap* m, int n, const float* vals) {
+        if (lane == 0) bulk_wait_read<1>();   // this slot's previous store has read it
+        __syncwarp();
+        uint8_t* b = sStage + (warp - 2) * STAGE_BUF + slot * 2048;
+        stage_bf16(b, lane, vals);
+        fence_async_smem();
+        __syncwarp();
+        if (lane == 0) tma_store_3d(m, smem_u32(b), n, srow, sbat);
+        slot ^= 1;
+      };
+      auto put_f32 = [&](const CUtensorMap* m, int n, const float* vals) {
+        if (lane == 0) bulk_wait_read<0>();
+        __syncwarp();
+        uint8_t* b = sStage + (warp - 2) * STAGE_BUF;
+        stage_f32(b, lane, vals);
+        fence_async_smem();
+        __syncwarp();
+        if (lane == 0) tma_store_3d(m, smem_u32(b), n, srow, sbat);
+      };
+
       constexpr int NC32 = BN / 32 / NPART;   // 32-column chunks per warp
       const int c32 = part * NC32;
       if constexpr (EPI == EPI_STORE_BF16 || EPI == EPI_STORE_F32) {
@@ -570,20 +640,12 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
         for (int c = c32; c < c32 + NC32; ++c) {
           tmem_ld32(tacc + c * 32, v);
           tmem_wait_ld();
-          if (no_k)
-#pragma unroll
-            for (int i = 0; i < 32; ++i) v[i] = 0u;
           const int n = nt * BN + c * 32;
-          if (row_st && n < p.N) {
+          if (st_any && n < p.N) {
 #pragma unroll
-            for (int i = 0; i < 32; ++i) f[i] = f32(v[i]);
-            if constexpr (EPI == EPI_STORE_BF16) {
-              store_bf16x32(reinterpret_cast<bf16*>(p.out0) + row_off + n, f);
-            } else {
-              float4* d4 = reinterpret_cast<float4*>(reinterpret_cast<float*>(p.out0) + row_off + n);
-#pragma unroll
-              for (int i = 0; i < 8; ++i) d4[i] = make_float4(f[4 * i], f[4 * i + 1], f[4 * i + 2], f[4 * i + 3]);
-            }
+            for (int i = 0; i < 32; ++i) f[i] = no_k ? 0.f : f32(v[i]);
+            if constexpr (EPI == EPI_STORE_BF16) put_bf16(&mO0, n, f);
+            else put_f32(&mO0, n, f);
           }
         }
       } else if constexpr (EPI == EPI_STORE_F32_SPLIT) {
@@ -591,49 +653,47 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
         for (int c = c32; c < c32 + NC32; ++c) {
           tmem_ld32(tacc + c * 32, v);
           tmem_wait_ld();
-          if (no_k)
-#pragma unroll
-            for (int i = 0; i < 32; ++i) v[i] = 0u;
           const int half = c >= BN / 64;
           const int n = nt * (BN / 2) + (c % (BN / 64)) * 32;
-          if (row_st && n < p.N) {
-            float* out = reinterpret_cast<float*>(half ? p.out1 : p.out0) + row_off + n;
-            float4* d4 = reinterpret_cast<float4*>(out);
+          if (st_any && n < p.N) {
 #pragma unroll
-            for (int i = 0; i < 8; ++i)
-              d4[i] = make_float4(f32(v[4 * i]), f32(v[4 * i + 1]), f32(v[4 * i + 2]), f32(v[4 * i + 3]));
+            for (int i = 0; i < 32; ++i) f[i] = no_k ? 0.f : f32(v[i]);
+            put_f32(half ? &mO1 : &mO0, n, f);
           }
         }
       } else if constexpr (EPI == EPI_SWIGLU_FWD) {
         uint32_t w[32];
         constexpr int NC64 = BN / 64 / NPART;
+        const float gs = (p.gate && row_ok) ? __ldg(p.gate + grow) : 1.0f;
 #pragma unroll 1
         for (int c = part * NC64; c < (part + 1) * NC64; ++c) {
           tmem_ld32(tacc + c * 32, v);
           tmem_ld32(tacc + BN / 2 + c * 32, w);
           tmem_wait_ld();
           const int n = nt * (BN / 2) + c * 32;
-          if (row_st && n < p.N) {
-            const float gs = (p.gate && row_ok) ? __ldg(p.gate + grow) : 1.0f;
+          if (st_any && n < p.N) {
             float g[32];
 #pragma unroll
             for (int i = 0; i < 32; ++i) {
-              const float av = f32(v[i]), bv = f32(w[i]);
-              f[i] = no_k ? 0.f : av;
-              g[i] = no_k ? 0.f : bv;
+              f[i] = no_k ? 0.f : f32(v[i]);
+              g[i] = no_k ? 0.f : f32(w[i]);
             }
-            store_bf16x32(reinterpret_cast<bf16*>(p.out0) + row_off + n, f);
-            store_bf16x32(reinterpret_cast<bf16*>(p.out1) + row_off + n, g);
+            put_bf16(&mO0, n, f);
+            put_bf16(&mO1, n, g);
 #pragma unroll
             for (int i = 0; i < 32; ++i) f[i] = gs * (f[i] * sigmoid_fast(f[i]) * g[i]);
-            store_bf16x32(reinterpret_cast<bf16*>(p.out2) + row_off + n, f);
+            put_bf16(&mO2, n, f);
           }
         }
       } else if constexpr (EPI == EPI_SWIGLU_BWD) {
-        // A and B of the next chunk are requested before the current one is computed
+        // A and B of the next chunk are requested before the current one is computed (not
+        // with variable rows, whose tile decode leaves too few registers for the second set)
+        constexpr bool PREFETCH = VARM != 1;
         const bf16* pa = reinterpret_cast<const bf16*>(p.in0) + row_off + nt * BN;
         const bf16* pb = reinterpret_cast<const bf16*>(p.in1) + row_off + nt * BN;
         uint4 ra[4], rb[4], na[4], nb[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) ra[i] = rb[i] = na[i] = nb[i] = make_uint4(0, 0, 0, 0);
         auto fetch = [&](int c, uint4* xa, uint4* xb) {
           const int n = nt * BN + c * 32;
           if (row_ok && n < p.N) {
@@ -644,42 +704,44 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
             }
           }
         };
-        fetch(c32, ra, rb);
+        if (PREFETCH) fetch(c32, ra, rb);
         const float gs = (p.gate && row_ok) ? __ldg(p.gate + grow) : 1.0f;
         float dot = 0.f;   // <acc, silu(A) * B> over this warp's columns of the row
 #pragma unroll 1
         for (int c = c32; c < c32 + NC32; ++c) {
-          if (c + 1 < c32 + NC32) fetch(c + 1, na, nb);
+          if (!PREFETCH) fetch(c, ra, rb);
+          else if (c + 1 < c32 + NC32) fetch(c + 1, na, nb);
           tmem_ld32(tacc + c * 32, v);
           tmem_wait_ld();
           const int n = nt * BN + c * 32;
-          if (no_k && row_st && n < p.N) {
+          if (st_any && n < p.N) {
+            float av[32], bv[32];   // av ends up holding dB
+            if (no_k) {
 #pragma unroll
-            for (int i = 0; i < 32; ++i) f[i] = 0.f;
-            store_bf16x32(reinterpret_cast<bf16*>(p.out0) + row_off + n, f);
-            store_bf16x32(reinterpret_cast<bf16*>(p.out1) + row_off + n, f);
-          } else if (row_ok && n < p.N) {
-            float av[32], bv[32], db[32];
+              for (int i = 0; i < 32; ++i) f[i] = av[i] = 0.f;
+            } else {
 #pragma unroll
-            for (int i = 0; i < 4; ++i) {
-              unpack16(ra[i], av + 8 * i, bf16());
-              unpack16(rb[i], bv + 8 * i, bf16());
+              for (int i = 0; i < 4; ++i) {
+                unpack16(ra[i], av + 8 * i, bf16());
+                unpack16(rb[i], bv + 8 * i, bf16());
+              }
+#pragma unroll
+              for (int i = 0; i < 32; ++i) {
+                const float a = av[i];
+                const float acc = f32(v[i]);
+                const float sg = sigmoid_fast(a);
+                const float das = gs * acc * sg;
+                dot = fmaf(acc, a * sg * bv[i], dot);
+                f[i] = das * bv[i] * fmaf(a, 1.0f - sg, 1.0f);
+                av[i] = das * a;
+              }
             }
-#pragma unroll
-            for (int i = 0; i < 32; ++i) {
-              const float acc = f32(v[i]);
-              const float du = gs * acc;
-              const float sg = sigmoid_fast(av[i]);
-              const float das = du * sg;
-              dot = fmaf(acc, av[i] * sg * bv[i], dot);
-              f[i] = das * bv[i] * fmaf(av[i], 1.0f - sg, 1.0f);
-              db[i] = das * av[i];
-            }
-            store_bf16x32(reinterpret_cast<bf16*>(p.out0) + row_off + n, f);
-            store_bf16x32(reinterpret_cast<bf16*>(p.out1) + row_off + n, db);
+            put_bf16(&mO0, n, f);
+            put_bf16(&mO1, n, av);
           }
+          if (PREFETCH)
 #pragma unroll
-          for (int i = 0; i < 4; ++i) { ra[i] = na[i]; rb[i] = nb[i]; }
+            for (int i = 0; i < 4; ++i) { ra[i] = na[i]; rb[i] = nb[i]; }
         }
         if (p.dgate_part && row_ok)
           p.dgate_part[(int64_t)(nt * NPART + part) * p.dgate_stride + grow] = dot;
@@ -733,6 +795,9 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
         else mbar_arrive(&tempty[a]);
       }
     }
+    // the TMA stores read the staging buffers until they complete
+    if (STAGED && lane == 0) bulk_wait_all();
+    __syncwarp();
   }
   tc_fence_before();
   __syncthreads();
@@ -778,6 +843,24 @@ cudaError_t make_map(CUtensorMap* m, const void* base, uint64_t cols, uint64_t r
   return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
 
+// 3-D output tensor [batch][rows][cols] for the epilogue's TMA stores: box of 32 rows x 32
+// columns, bf16 with the 64-byte swizzle or fp32 with the 128-byte swizzle (one staged chunk).
+cudaError_t make_out_map(CUtensorMap* m, const void* base, bool f32, uint64_t cols, uint64_t rows,
+                         uint64_t batch) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return cudaErrorNotSupported;
+  const uint64_t es = f32 ? 4 : 2;
+  cuuint64_t dims[3] = {cols, rows, batch};
+  cuuint64_t strides[2] = {cols * es, cols * rows * es};
+  cuuint32_t box[3] = {32, 32, 1};
+  cuuint32_t estr[3] = {1, 1, 1};
+  CUresult r = fn(m, f32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3,
+                  const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                  f32 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B,
+                  CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
 int sm_count() {
   static int n = 0;
   if (!n) {
@@ -792,9 +875,11 @@ int sm_count() {
 template <int BN, bool A_MN, bool B_MN, bool B_SPLIT, bool K_SPLIT, int EPI, int STAGES,
           int EPW = 8, bool PAIR = false, int VARM = 0>
 cudaError_t launch(const CUtensorMap& a0, const CUtensorMap& a1, const CUtensorMap& b0,
-                   const CUtensorMap& b1, Args p, cudaStream_t st) {
+                   const CUtensorMap& b1, const CUtensorMap& o0, const CUtensorMap& o1,
+                   const CUtensorMap& o2, Args p, cudaStream_t st) {
   auto kern = tc_gemm_kernel<BN, A_MN, B_MN, B_SPLIT, K_SPLIT, EPI, STAGES, EPW, PAIR, VARM>;
-  constexpr uint32_t smem = smem_bytes<BN, STAGES, PAIR>();
+  constexpr uint32_t smem = smem_bytes<BN, STAGES, PAIR, EPW, EPI != EPI_ROUTER>();
+  static_assert(smem <= 232448, "dynamic shared memory above the 227 KB per-block limit");
   constexpr int threads = 64 + 32 * EPW;
   static bool attr = false;
   static int max_clusters = 0;
@@ -829,10 +914,10 @@ cudaError_t launch(const CUtensorMap& a0, const CUtensorMap& a1, const CUtensorM
   if (PAIR) {
     const int clusters = total < max_clusters ? total : max_clusters;
     cfg.gridDim = dim3(2 * clusters);
-    return cudaLaunchKernelEx(&cfg, kern, a0, a1, b0, b1, p);
+    return cudaLaunchKernelEx(&cfg, kern, a0, a1, b0, b1, o0, o1, o2, p);
   }
   const int grid = total < sm_count() ? total : sm_count();
-  kern<<<grid, threads, smem, st>>>(a0, a1, b0, b1, p);
+  kern<<<grid, threads, smem, st>>>(a0, a1, b0, b1, o0, o1, o2, p);
   return cudaGetLastError();
 }
 
@@ -898,10 +983,15 @@ cudaError_t tc_router_softmax(const void* X, const void* Wr, void* Wr_pad, const
   p.bias = br;
   p.n_valid = E;
   switch (Ep) {
-    case 64: return launch<64, false, true, false, false, EPI_ROUTER, 8, 4>(ma, ma, mb, mb, p, st);
-    case 128: return launch<128, false, true, false, false, EPI_ROUTER, 6, 4>(ma, ma, mb, mb, p, st);
-    case 192: return launch<192, false, true, false, false, EPI_ROUTER, 5, 4>(ma, ma, mb, mb, p, st);
-    case 256: return launch<256, false, true, false, false, EPI_ROUTER, 4, 4>(ma, ma, mb, mb, p, st);
+    // the router epilogue writes S and S^T itself: the output maps are unused
+    case 64:
+      return launch<64, false, true, false, false, EPI_ROUTER, 8, 4>(ma, ma, mb, mb, ma, ma, ma, p, st);
+    case 128:
+      return launch<128, false, true, false, false, EPI_ROUTER, 6, 4>(ma, ma, mb, mb, ma, ma, ma, p, st);
+    case 192:
+      return launch<192, false, true, false, false, EPI_ROUTER, 5, 4>(ma, ma, mb, mb, ma, ma, ma, p, st);
+    case 256:
+      return launch<256, false, true, false, false, EPI_ROUTER, 4, 4>(ma, ma, mb, mb, ma, ma, ma, p, st);
   }
   return cudaErrorInvalidValue;
 }
@@ -912,6 +1002,12 @@ cudaError_t tc_router_softmax(const void* X, const void* Wr, void* Wr_pad, const
 static cudaError_t act_map(CUtensorMap* m, const void* base, int cols, int E, int M,
                            const VarRows* vr, uint32_t box_rows) {
   return vr ? make_map(m, base, cols, vr->P, 1, box_rows) : make_map(m, base, cols, M, E, box_rows);
+}
+
+// Output map of an expert activation tensor, laid out like the inputs of act_map.
+static cudaError_t act_out_map(CUtensorMap* m, const void* base, int cols, int E, int M,
+                               const VarRows* vr) {
+  return vr ? make_out_map(m, base, false, cols, vr->P, 1) : make_out_map(m, base, false, cols, M, E);
 }
 
 static Args row_args(int E, int M, int N, int K, int BN_tile, int* status, const VarRows* vr) {
@@ -926,19 +1022,26 @@ static Args row_args(int E, int M, int N, int K, int BN_tile, int* status, const
 
 template <int BN, bool A_MN, bool B_MN, bool B_SPLIT, bool K_SPLIT, int EPI>
 static cudaError_t launch_rows(const CUtensorMap& a0, const CUtensorMap& a1, const CUtensorMap& b0,
-                               const CUtensorMap& b1, const Args& p, const VarRows* vr,
+                               const CUtensorMap& b1, const CUtensorMap& o0, const CUtensorMap& o1,
+                               const CUtensorMap& o2, const Args& p, const VarRows* vr,
                                cudaStream_t st) {
-  if (vr) return launch<BN, A_MN, B_MN, B_SPLIT, K_SPLIT, EPI, 6, 8, true, 1>(a0, a1, b0, b1, p, st);
-  return launch<BN, A_MN, B_MN, B_SPLIT, K_SPLIT, EPI, 6, 8, true, 0>(a0, a1, b0, b1, p, st);
+  if (vr)
+    return launch<BN, A_MN, B_MN, B_SPLIT, K_SPLIT, EPI, 6, 8, true, 1>(a0, a1, b0, b1, o0, o1, o2,
+                                                                         p, st);
+  return launch<BN, A_MN, B_MN, B_SPLIT, K_SPLIT, EPI, 6, 8, true, 0>(a0, a1, b0, b1, o0, o1, o2, p,
+                                                                       st);
 }
 
 cudaError_t tc_expert_up(const void* H, const void* Wg, const void* Wu, void* A, void* B, void* U,
                          int E, int M, int d, int F, int* status, cudaStream_t st,
                          const VarRows* vr, const float* gate) {
-  CUtensorMap ma, mg, mu;
+  CUtensorMap ma, mg, mu, oa, ob, ou;
   TC_TRY(act_map(&ma, H, d, E, M, vr, BM));
   TC_TRY(make_map(&mg, Wg, F, d, E, 64));
   TC_TRY(make_map(&mu, Wu, F, d, E, 64));
+  TC_TRY(act_out_map(&oa, A, F, E, M, vr));
+  TC_TRY(act_out_map(&ob, B, F, E, M, vr));
+  TC_TRY(act_out_map(&ou, U, F, E, M, vr));
   Args p = row_args(E, M, F, d, 128, status, vr);
   p.out0 = A;
   p.out1 = B;
@@ -946,28 +1049,33 @@ cudaError_t tc_expert_up(const void* H, const void* Wg, const void* Wu, void* A,
   p.gate = gate;
   p.ld = F;
   p.bstride = (int64_t)M * F;
-  return launch_rows<256, false, true, true, false, EPI_SWIGLU_FWD>(ma, ma, mg, mu, p, vr, st);
+  return launch_rows<256, false, true, true, false, EPI_SWIGLU_FWD>(ma, ma, mg, mu, oa, ob, ou, p,
+                                                                    vr, st);
 }
 
 cudaError_t tc_expert_down(const void* U, const void* Wd, void* O, int E, int M, int d, int F,
                            int* status, cudaStream_t st, const VarRows* vr) {
-  CUtensorMap ma, mb;
+  CUtensorMap ma, mb, mo;
   TC_TRY(act_map(&ma, U, F, E, M, vr, BM));
   TC_TRY(make_map(&mb, Wd, d, F, E, 64));
+  TC_TRY(act_out_map(&mo, O, d, E, M, vr));
   Args p = row_args(E, M, d, F, 256, status, vr);
   p.out0 = O;
   p.ld = d;
   p.bstride = (int64_t)M * d;
-  return launch_rows<256, false, true, false, false, EPI_STORE_BF16>(ma, ma, mb, mb, p, vr, st);
+  return launch_rows<256, false, true, false, false, EPI_STORE_BF16>(ma, ma, mb, mb, mo, mo, mo, p,
+                                                                     vr, st);
 }
 
 cudaError_t tc_expert_dgrad_up(const void* dO, const void* Wd, const void* A, const void* B,
                                void* dA, void* dB, int E, int M, int d, int F, int* status,
                                cudaStream_t st, const VarRows* vr, const float* gate,
                                float* dgate_part, int64_t dgate_stride) {
-  CUtensorMap ma, mb;
+  CUtensorMap ma, mb, oa, ob;
   TC_TRY(act_map(&ma, dO, d, E, M, vr, BM));
   TC_TRY(make_map(&mb, Wd, d, F, E, 128));   // B[n=f][k=i] = Wd[f][i]: K-major, half per CTA
+  TC_TRY(act_out_map(&oa, dA, F, E, M, vr));
+  TC_TRY(act_out_map(&ob, dB, F, E, M, vr));
   Args p = row_args(E, M, F, d, 256, status, vr);
   p.in0 = A;
   p.in1 = B;
@@ -978,7 +1086,8 @@ cudaError_t tc_expert_dgrad_up(const void* dO, const void* Wd, const void* A, co
   p.dgate_stride = dgate_stride;
   p.ld = F;
   p.bstride = (int64_t)M * F;
-  return launch_rows<256, false, false, false, false, EPI_SWIGLU_BWD>(ma, ma, mb, mb, p, vr, st);
+  return launch_rows<256, false, false, false, false, EPI_SWIGLU_BWD>(ma, ma, mb, mb, oa, ob, ob, p,
+                                                                      vr, st);
 }
 
 cudaError_t tc_expert_dgrad_h(const void* dA, const void* dB, const void* Wg, const void* Wu,
@@ -989,12 +1098,15 @@ cudaError_t tc_expert_dgrad_h(const void* dA, const void* dB, const void* Wg, co
   TC_TRY(act_map(&ma1, dB, F, E, M, vr, BM));
   TC_TRY(make_map(&mb0, Wg, F, d, E, 128));  // B[n=i][k=f] = Wg[i][f]: K-major, half per CTA
   TC_TRY(make_map(&mb1, Wu, F, d, E, 128));
+  CUtensorMap mo;
+  TC_TRY(act_out_map(&mo, dH, d, E, M, vr));
   Args p = row_args(E, M, d, 2 * F, 256, status, vr);
   p.k_blocks0 = F / BK;
   p.out0 = dH;
   p.ld = d;
   p.bstride = (int64_t)M * d;
-  return launch_rows<256, false, false, false, true, EPI_STORE_BF16>(ma0, ma1, mb0, mb1, p, vr, st);
+  return launch_rows<256, false, false, false, true, EPI_STORE_BF16>(ma0, ma1, mb0, mb1, mo, mo, mo,
+                                                                     p, vr, st);
 }
 
 cudaError_t tc_expert_wgrad(const void* H, const void* U, const void* dO, const void* dA,
@@ -1013,35 +1125,40 @@ cudaError_t tc_expert_wgrad(const void* H, const void* U, const void* dO, const 
   };
   {
     // dWd[e] [F][d] = U[e]^T . dO[e]: A[m=f][k=t] = U[t][f] (MN-major), B[k=t][n=i] = dO[t][i]
-    CUtensorMap ma, mb;
+    CUtensorMap ma, mb, mo;
     TC_TRY(act_map(&ma, U, F, E, M, vr, 64));
     TC_TRY(act_map(&mb, dO, d, E, M, vr, 64));
+    TC_TRY(make_out_map(&mo, dWd, true, d, F, E));
     Args p = wg_args(F, d, 256);
     p.out0 = dWd;
     p.ld = d;
     p.bstride = (int64_t)F * d;
     if (vr)
-      TC_TRY((launch<256, true, true, false, false, EPI_STORE_F32, 6, 8, true, 2>(ma, ma, mb, mb, p, st)));
+      TC_TRY((launch<256, true, true, false, false, EPI_STORE_F32, 6, 8, true, 2>(ma, ma, mb, mb, mo, mo,
+                                                                                mo, p, st)));
     else
-      TC_TRY((launch<256, true, true, false, false, EPI_STORE_F32, 6, 8, true>(ma, ma, mb, mb, p, st)));
+      TC_TRY((launch<256, true, true, false, false, EPI_STORE_F32, 6, 8, true>(ma, ma, mb, mb, mo, mo, mo,
+                                                                             p, st)));
   }
   {
     // [dWg | dWu][e] [d][F] = H[e]^T . [dA | dB][e]
-    CUtensorMap ma, mb0, mb1;
+    CUtensorMap ma, mb0, mb1, mo0, mo1;
     TC_TRY(act_map(&ma, H, d, E, M, vr, 64));
     TC_TRY(act_map(&mb0, dA, F, E, M, vr, 64));
     TC_TRY(act_map(&mb1, dB, F, E, M, vr, 64));
+    TC_TRY(make_out_map(&mo0, dWg, true, F, d, E));
+    TC_TRY(make_out_map(&mo1, dWu, true, F, d, E));
     Args p = wg_args(d, F, 128);
     p.out0 = dWg;
     p.out1 = dWu;
     p.ld = F;
     p.bstride = (int64_t)d * F;
     if (vr)
-      TC_TRY((launch<256, true, true, true, false, EPI_STORE_F32_SPLIT, 6, 8, true, 2>(ma, ma, mb0, mb1,
-                                                                                     p, st)));
+      TC_TRY((launch<256, true, true, true, false, EPI_STORE_F32_SPLIT, 6, 8, true, 2>(
+          ma, ma, mb0, mb1, mo0, mo1, mo1, p, st)));
     else
-      TC_TRY((launch<256, true, true, true, false, EPI_STORE_F32_SPLIT, 6, 8, true>(ma, ma, mb0, mb1, p,
-                                                                                  st)));
+      TC_TRY((launch<256, true, true, true, false, EPI_STORE_F32_SPLIT, 6, 8, true>(
+          ma, ma, mb0, mb1, mo0, mo1, mo1, p, st)));
   }
   return cudaSuccess;
 }
@@ -1056,12 +1173,14 @@ cudaError_t tc_router_dgrad(const void* dZb, const void* Wr_pad, float* dXr, int
   TC_TRY(make_map(&ma0, hi, Ep, N, 1, BM));
   TC_TRY(make_map(&ma1, hi + (size_t)N * Ep, Ep, N, 1, BM));
   TC_TRY(make_map(&mb, Wr_pad, Ep, d, 1, 256));
+  CUtensorMap mo;
+  TC_TRY(make_out_map(&mo, dXr, true, d, N, 1));
   Args p = base_args(1, N, d, 2 * Ep, 256, status);
   p.k_blocks0 = Ep / BK;
   p.out0 = dXr;
   p.ld = d;
   p.bstride = 0;
-  return launch<256, false, false, false, true, EPI_STORE_F32, 4>(ma0, ma1, mb, mb, p, st);
+  return launch<256, false, false, false, true, EPI_STORE_F32, 4>(ma0, ma1, mb, mb, mo, mo, mo, p, st);
 }
 
 cudaError_t tc_router_wgrad(const void* X, const void* dZb, float* part, int N, int d, int Ep,
@@ -1075,6 +1194,9 @@ cudaError_t tc_router_wgrad(const void* X, const void* dZb, float* part, int N, 
   TC_TRY(make_map(&ma, X, d, rows, splits, 64));
   TC_TRY(make_map(&mb0, hi, Ep, rows, splits, 64));
   TC_TRY(make_map(&mb1, hi + (size_t)N * Ep, Ep, rows, splits, 64));
+  CUtensorMap mo0, mo1;
+  TC_TRY(make_out_map(&mo0, part, true, Ep, d, splits));
+  TC_TRY(make_out_map(&mo1, part + (size_t)splits * d * Ep, true, Ep, d, splits));
   const int BNt = Ep > 64 ? 256 : 128;
   Args p = base_args(splits, d, Ep, rows, BNt / 2, status);
   p.out0 = part;
@@ -1082,8 +1204,10 @@ cudaError_t tc_router_wgrad(const void* X, const void* dZb, float* part, int N, 
   p.ld = Ep;
   p.bstride = (int64_t)d * Ep;
   if (BNt == 128)
-    return launch<128, true, true, true, false, EPI_STORE_F32_SPLIT, 6>(ma, ma, mb0, mb1, p, st);
-  return launch<256, true, true, true, false, EPI_STORE_F32_SPLIT, 4>(ma, ma, mb0, mb1, p, st);
+    return launch<128, true, true, true, false, EPI_STORE_F32_SPLIT, 6>(ma, ma, mb0, mb1, mo0, mo1, mo1,
+                                                                        p, st);
+  return launch<256, true, true, true, false, EPI_STORE_F32_SPLIT, 4>(ma, ma, mb0, mb1, mo0, mo1, mo1,
+                                                                      p, st);
 }
 
 cudaError_t tc_wait_probe(int* status, unsigned long long limit_ns, cudaStream_t st) {
