@@ -98,7 +98,23 @@ __global__ void combine_kernel(const T* __restrict__ O, const float* __restrict_
 #pragma unroll
       for (int j = 0; j < VN; ++j) acc[j] += r[j];
     }
-    for (int p = 0; p < cnt; ++p) {
+    // rows are summed in ascending expert order; loads are issued four pairs at a time
+    int p = 0;
+    for (; p + 4 <= cnt; p += 4) {
+      uint4 u[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q)
+        u[q] = __ldg(reinterpret_cast<const uint4*>(O + ((size_t)s_e[p + q] * M + s_m[p + q]) * d) + v);
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        float o[VN];
+        unpack16(u[q], o, T());
+        const float g = s_g[p + q];
+#pragma unroll
+        for (int j = 0; j < VN; ++j) acc[j] = fmaf(g, o[j], acc[j]);
+      }
+    }
+    for (; p < cnt; ++p) {
       const size_t row = (size_t)s_e[p] * M + s_m[p];
       const uint4 u = __ldg(reinterpret_cast<const uint4*>(O + row * d) + v);
       float o[VN];
