@@ -26,6 +26,7 @@ struct ec_ctx {
   int wr_splits = 1;   // split-K factor of dWr = X^T dZ
   int dg_parts = 1;    // partial sums per gate gradient (tensor-core dU epilogue)
   size_t o_dgsum = 0;  // the gate gradients summed over their partials
+  size_t o_colsum = 0; // partial column sums of dZ (router bias gradient)
   int Ep = 64;         // experts rounded up to 64 (tensor-core router operands)
   // per-kernel event timing (off by default) and kernel launch counter
   bool prof = false;
@@ -161,6 +162,7 @@ void layout(ec_ctx* c) {
   c->o_f32a = take(f32n * 4);
   c->o_f32b = take((use_tc(c) ? 0 : big) * 4);
   c->o_dXr = take(N * d * 4);
+  c->o_colsum = take((size_t)colsum_scratch_floats((int)N, (int)E) * 4);
   // split-K partials of dWr = X^T dZ (tensor cores: equal token blocks, so N % splits == 0)
   if (use_tc(c)) {
     c->wr_splits = 1;
@@ -499,7 +501,8 @@ ec_status run_backward(ec_ctx* c, const void* dY, void* dX, float* dWr, float* d
     EC_KERNEL("router_wgrad_reduce", 1,
               launch_reduce_splits(part, dWr, (int64_t)d * E, c->wr_splits, st));
   }
-  if (dbr) EC_KERNEL("router_dbias", 1, launch_colsum(dZ, dbr, N, E, st));
+  if (dbr)
+    EC_KERNEL("router_dbias", 2, launch_colsum(dZ, dbr, N, E, at<float>(c, c->o_colsum), st));
   return EC_OK;
 }
 
@@ -597,7 +600,8 @@ ec_status run_tc_backward(ec_ctx* c, const void* dY, void* dX, float* dWr, float
             tc_router_wgrad(c->X, dZb, part, N, d, c->Ep, c->wr_splits, status, st));
   EC_KERNEL("router_wgrad_reduce", 1,
             launch_reduce_partials(part, dWr, d, E, c->Ep, 2 * c->wr_splits, st));
-  if (dbr) EC_KERNEL("router_dbias", 1, launch_colsum(dZ, dbr, N, E, st));
+  if (dbr)
+    EC_KERNEL("router_dbias", 2, launch_colsum(dZ, dbr, N, E, at<float>(c, c->o_colsum), st));
   return EC_OK;
 }
 

@@ -65,7 +65,11 @@ cudaError_t launch_reduce_partials(const float* part, float* out, int rows, int 
 template <typename T>
 cudaError_t launch_dx_combine(const T* dH, const int* slot, const float* dXr, const T* R,
                               const T* R2, T* dX, int N, int E, int M, int d, cudaStream_t st);
-cudaError_t launch_colsum(const float* Z, float* out, int N, int E, cudaStream_t st);
+// out[e] = sum over the N rows of Z [N][E]; scratch: colsum_scratch_floats(N, E) floats.
+// Two kernels.
+cudaError_t launch_colsum(const float* Z, float* out, int N, int E, float* scratch,
+                          cudaStream_t st);
+int64_t colsum_scratch_floats(int N, int E);
 template <typename T>
 cudaError_t launch_swiglu_fwd_ew(const float* Ag, const float* Bu, T* A, T* B, T* U, int64_t n,
                                  cudaStream_t st);

@@ -323,24 +323,50 @@ cudaError_t launch_dx_combine(const T* dH, const int* slot, const float* dXr, co
 }
 
 // ------------------------------------------------------------------ column sums of Z [N][E]
-__global__ void colsum_kernel(const float* __restrict__ Z, float* __restrict__ out, int N, int E) {
-  __shared__ float part[8][33];
+// Two passes, deterministic: partial sums over blocks of kColRows rows (32 columns per
+// block, 8 warps over the rows), then the partials summed in block order.
+constexpr int kColRows = 512;
+
+__global__ void colsum_part_kernel(const float* __restrict__ Z, float* __restrict__ part, int N,
+                                   int E) {
+  __shared__ float sh[8][33];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int e = blockIdx.x * 32 + lane;
+  const int r0 = blockIdx.y * kColRows;
+  const int r1 = min(N, r0 + kColRows);
   float s = 0.f;
   if (e < E)
-    for (int t = warp; t < N; t += 8) s += Z[(size_t)t * E + e];
-  part[warp][lane] = s;
+#pragma unroll 8
+    for (int t = r0 + warp; t < r1; t += 8) s += Z[(size_t)t * E + e];
+  sh[warp][lane] = s;
   __syncthreads();
   if (warp == 0 && e < E) {
     float r = 0.f;
-    for (int w = 0; w < 8; ++w) r += part[w][lane];
-    out[e] = r;
+#pragma unroll
+    for (int w = 0; w < 8; ++w) r += sh[w][lane];
+    part[(size_t)blockIdx.y * E + e] = r;
   }
 }
 
-cudaError_t launch_colsum(const float* Z, float* out, int N, int E, cudaStream_t st) {
-  colsum_kernel<<<(E + 31) / 32, 256, 0, st>>>(Z, out, N, E);
+__global__ void colsum_final_kernel(const float* __restrict__ part, int nrb, int E,
+                                    float* __restrict__ out) {
+  const int e = blockIdx.x * blockDim.x + threadIdx.x;
+  if (e >= E) return;
+  float s = 0.f;
+  for (int b = 0; b < nrb; ++b) s += part[(size_t)b * E + e];
+  out[e] = s;
+}
+
+int64_t colsum_scratch_floats(int N, int E) {
+  return (int64_t)((N + kColRows - 1) / kColRows) * E;
+}
+
+cudaError_t launch_colsum(const float* Z, float* out, int N, int E, float* scratch,
+                          cudaStream_t st) {
+  const int nrb = (N + kColRows - 1) / kColRows;
+  if (nrb == 0) return cudaMemsetAsync(out, 0, (size_t)E * sizeof(float), st);
+  colsum_part_kernel<<<dim3((E + 31) / 32, nrb), 256, 0, st>>>(Z, scratch, N, E);
+  colsum_final_kernel<<<(E + 127) / 128, 128, 0, st>>>(scratch, nrb, E, out);
   return cudaGetLastError();
 }
 
