@@ -623,6 +623,23 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
         if (lane == 0) tma_store_3d(m, smem_u32(b), n, srow, sbat);
         slot ^= 1;
       };
+      // two bf16 chunks at once (both halves of the buffer, one proxy fence): each store is
+      // its own bulk group, the first one (half 0) the older
+      auto put2_bf16 = [&](const CUtensorMap* m0, const CUtensorMap* m1, int n, const float* v0,
+                           const float* v1) {
+        if (lane == 0) bulk_wait_read<0>();
+        __syncwarp();
+        uint8_t* b = sStage + (warp - 2) * STAGE_BUF;
+        stage_bf16(b, lane, v0);
+        stage_bf16(b + 2048, lane, v1);
+        fence_async_smem();
+        __syncwarp();
+        if (lane == 0) {
+          tma_store_3d(m0, smem_u32(b), n, srow, sbat);
+          tma_store_3d(m1, smem_u32(b + 2048), n, srow, sbat);
+        }
+        slot = 0;   // the next single chunk goes to half 0 once its store (the older) has read it
+      };
       auto put_f32 = [&](const CUtensorMap* m, int n, const float* vals) {
         if (lane == 0) bulk_wait_read<0>();
         __syncwarp();
@@ -678,8 +695,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
               f[i] = no_k ? 0.f : f32(v[i]);
               g[i] = no_k ? 0.f : f32(w[i]);
             }
-            put_bf16(&mO0, n, f);
-            put_bf16(&mO1, n, g);
+            put2_bf16(&mO0, &mO1, n, f, g);
 #pragma unroll
             for (int i = 0; i < 32; ++i) f[i] = gs * (f[i] * sigmoid_fast(f[i]) * g[i]);
             put_bf16(&mO2, n, f);
@@ -736,8 +752,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
                 av[i] = das * a;
               }
             }
-            put_bf16(&mO0, n, f);
-            put_bf16(&mO1, n, av);
+            put2_bf16(&mO0, &mO1, n, f, av);
           }
           if (PREFETCH)
 #pragma unroll
