@@ -61,6 +61,11 @@ CASES = [
     # skewed router bias: experts with several 256-row tiles next to nearly empty ones
     ("skew_dropless", dict(router_bias=True, E=4, L=512), 2, None),
     ("skew_cf1", dict(router_bias=True, E=4, L=512), 2, 1.0),
+    # ragged: N = 2 x 350 (not a multiple of the 256-token ranking block), 12 experts (not a
+    # multiple of 32 or 64), k = 3, a tight cap
+    ("ragged_e12_k3", dict(L=350, E=12, router_bias=True), 3, 0.6),
+    # 100 experts over two 64-column router tiles, every expert a tail of 256-row padding
+    ("e100_k5", dict(L=384, E=100, d=64, d_ff=64), 5, None),
 ]
 
 
