@@ -320,6 +320,16 @@ def run_ours(args):
             h = ybuf[0]
     else:
         rows = [w.E * int(inp.k_g.sum())] * w.layers
+    # token coverage of the first layer: tokens no expert picked (expert choice) or
+    # token-expert pairs dropped by the capacity (token choice)
+    if tc:
+        coverage = {"pairs_dropped_frac": round(1.0 - rows[0] / (w.N * args.tc_k), 6)}
+    else:
+        l0, wts0, ybuf0 = stack[0][0], stack[0][1], stack[0][2]
+        idx0 = l0.forward(X, *wts0, Y=ybuf0[0], outputs=True, shared=stack[0][4])[1]
+        picked = torch.zeros(w.N, dtype=torch.bool, device=device)
+        picked[idx0.flatten().long()] = True
+        coverage = {"tokens_unpicked_frac": round(1.0 - picked.float().mean().item(), 6)}
 
     # ---- device-timed steps (inputs resident), per-kernel events on the same stream
     for l_ in stack:
@@ -510,6 +520,7 @@ def run_ours(args):
     out["graph"] = {"ms_per_step": round(graph_ms, 4),
                     "value": round(ws * w.N / (graph_ms * 1e-3), 1), "unit": UNIT,
                     "note": "same step captured in one CUDA graph, replayed; no per-kernel events"}
+    out["coverage"] = coverage
     out["gpu_launches"] = int(launches)
     out["kernel_ms_per_step"] = {k: round(sum(v) / args.steps, 4) for k, v in per.items()}
     out["clocks"] = clk

@@ -7,6 +7,8 @@
 #include <cstring>
 #include <cstdarg>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "../../include/ecmoe.h"
 #include "common.cuh"
 #include "kernels.h"
@@ -33,6 +35,7 @@ struct ec_ctx {
   std::vector<cudaEvent_t> ev;
   std::vector<const char*> ev_name;
   int ev_n = 0;
+  bool nvtx_open = false;   // an NVTX range named after the current phase is open
   int64_t launches = 0;
   // state saved by the forward pass
   bool residual = false;   // Y = X + EC(X), dX = dY + EC input gradient
@@ -75,9 +78,13 @@ ec_status cuda_fail(ec_ctx* c, cudaError_t e, const char* where) {
   } while (0)
 
 // Phase marker: with profiling on, records an event named after the kernel about to be
-// launched (or "end" after the last one) on the call's stream.
+// launched (or "end" after the last one) on the call's stream, and opens an NVTX range of
+// the same name (closed at the next marker) for profilers that filter by range.
 void mark(ec_ctx* c, const char* name, cudaStream_t st) {
   if (!c->prof) return;
+  if (c->nvtx_open) nvtxRangePop();
+  c->nvtx_open = std::strcmp(name, "end") != 0;
+  if (c->nvtx_open) nvtxRangePushA(name);
   if (c->ev_n == (int)c->ev.size()) {
     cudaEvent_t e;
     if (cudaEventCreate(&e) != cudaSuccess) return;

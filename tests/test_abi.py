@@ -78,3 +78,45 @@ def test_host_validation_without_device(lib):
         assert e.value.status == ec.EC_ERR_WORKSPACE
     finally:
         ec.ec_ctx_destroy(ctx)
+
+
+def test_token_choice_host_validation_without_device(lib):
+    # bf16 only; 1 <= k <= min(E, 32); at most 256 experts; d, d_ff multiples of 64
+    for args, status in (((256, 64, 8, 128, 2, -1, ec.EC_F32), ec.EC_ERR_UNSUPPORTED),
+                         ((256, 64, 8, 128, 0, -1, ec.EC_BF16), ec.EC_ERR_SHAPE),
+                         ((256, 64, 8, 128, 9, -1, ec.EC_BF16), ec.EC_ERR_SHAPE),
+                         ((256, 64, 64, 128, 33, -1, ec.EC_BF16), ec.EC_ERR_SHAPE),
+                         ((256, 64, 300, 128, 2, -1, ec.EC_BF16), ec.EC_ERR_UNSUPPORTED),
+                         ((256, 96, 8, 128, 2, -1, ec.EC_BF16), ec.EC_ERR_UNSUPPORTED)):
+        with pytest.raises(ec.ECError) as e:
+            ec.ec_tc_ctx_create(*args)
+        assert e.value.status == status, args
+    ctx = ec.ec_tc_ctx_create(1000, 64, 12, 128, 3, 250, ec.EC_BF16)
+    try:
+        # the padded rows (N k + 255 E, in 256-row blocks) make the workspace larger than an
+        # expert-choice one of the same shape and capacity
+        ec_ctx = ec.ec_ctx_create(1000, 64, 12, 128, 1, [0, 1000], [250], ec.EC_BF16)
+        assert ec.ec_workspace_bytes(ctx) > ec.ec_workspace_bytes(ec_ctx)
+        ec.ec_ctx_destroy(ec_ctx)
+        # expert-choice calls are refused on a token-choice context
+        with pytest.raises(ec.ECError) as e:
+            ec.ec_ctx_set_capacity(ctx, [4])
+        assert e.value.status == ec.EC_ERR_STATE
+        with pytest.raises(ec.ECError) as e:
+            ec.ec_ctx_set_shared(ctx, 64)
+        assert e.value.status == ec.EC_ERR_STATE
+        # and compute calls need a workspace first
+        with pytest.raises(ec.ECError) as e:
+            ec.ec_tc_forward(ctx, 16, 16, None, 16, 16, 16, 16, None, None, None, None, None,
+                             None)
+        assert e.value.status == ec.EC_ERR_WORKSPACE
+    finally:
+        ec.ec_ctx_destroy(ctx)
+    # token-choice calls are refused on an expert-choice context (after the workspace check)
+    ctx = ec.ec_ctx_create(256, 64, 8, 128, 2, [0, 128, 256], [16, 16], ec.EC_F32)
+    try:
+        with pytest.raises(ec.ECError) as e:
+            ec.ec_tc_backward(ctx, 16, 16, 16, None, 16, 16, 16, None)
+        assert e.value.status == ec.EC_ERR_WORKSPACE
+    finally:
+        ec.ec_ctx_destroy(ctx)
