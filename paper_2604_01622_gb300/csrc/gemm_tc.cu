@@ -1035,16 +1035,20 @@ static Args row_args(int E, int M, int N, int K, int BN_tile, int* status, const
   return p;
 }
 
+constexpr int kDuStages = 5;
+
 template <int BN, bool A_MN, bool B_MN, bool B_SPLIT, bool K_SPLIT, int EPI>
 static cudaError_t launch_rows(const CUtensorMap& a0, const CUtensorMap& a1, const CUtensorMap& b0,
                                const CUtensorMap& b1, const CUtensorMap& o0, const CUtensorMap& o1,
                                const CUtensorMap& o2, const Args& p, const VarRows* vr,
                                cudaStream_t st) {
+  // the dU GEMM's epilogue reads A and B through L1: a 5-deep ring leaves it 32 KB more
+  constexpr int ST = EPI == EPI_SWIGLU_BWD ? kDuStages : 6;
   if (vr)
-    return launch<BN, A_MN, B_MN, B_SPLIT, K_SPLIT, EPI, 6, 8, true, 1>(a0, a1, b0, b1, o0, o1, o2,
-                                                                         p, st);
-  return launch<BN, A_MN, B_MN, B_SPLIT, K_SPLIT, EPI, 6, 8, true, 0>(a0, a1, b0, b1, o0, o1, o2, p,
-                                                                       st);
+    return launch<BN, A_MN, B_MN, B_SPLIT, K_SPLIT, EPI, ST, 8, true, 1>(a0, a1, b0, b1, o0, o1, o2,
+                                                                          p, st);
+  return launch<BN, A_MN, B_MN, B_SPLIT, K_SPLIT, EPI, ST, 8, true, 0>(a0, a1, b0, b1, o0, o1, o2, p,
+                                                                        st);
 }
 
 cudaError_t tc_expert_up(const void* H, const void* Wg, const void* Wu, void* A, void* B, void* U,
