@@ -466,10 +466,10 @@ def run_ours(args):
         "router_gemm_softmax": N * d * b + 2 * N * E * 4,
         "topk": 2 * N * E * 4 + 2 * P * 4,
         "tc_route": 2 * N * E * 4 + 3 * P * 4,
-        "gather": 2 * P * d * b,
+        "gather": (N + P) * d * b,          # token-major: each X row read once, P rows written
         "combine": P * d * b + N * d * b,
         "bwd_gather_scale": 3 * P * d * b,
-        "gather_dy": 2 * P * d * b,
+        "gather_dy": (N + P) * d * b,
         "softmax_bwd": 3 * N * E * 4,
         "dgate_reduce": (2 * math.ceil(w.d_ff / 256) + 1) * P * 4,
         "dx_combine": P * d * b + N * d * 4 + N * d * b,

@@ -423,7 +423,9 @@ ec_status run_forward(ec_ctx* c, const void* X, const void* Wg, const void* Wu, 
   const float* gate = at<float>(c, c->o_gate);
   // tensor cores: the gate is applied in the gate/up epilogue (O rows come out gated)
   const bool fused_gate = use_tc(c);
-  EC_KERNEL("gather", pz, launch_gather<T>(Xt, idx, H, P, d, st));
+  // token-major: each X row is read once and written to the rows of the experts that chose it
+  EC_KERNEL("gather", N > 0 && pz,
+            launch_scatter_rows<T>(Xt, at<int>(c, c->o_slot), H, N, E, M, d, st));
   EC_TRY(ffn_forward<T>(c, kRouted, H, Wg, Wu, Wd, at<T>(c, c->o_A), at<T>(c, c->o_B),
                         at<T>(c, c->o_U), O, E, M, F, st, fused_gate ? gate : nullptr));
   EC_KERNEL("combine", N > 0,
@@ -454,7 +456,7 @@ ec_status run_backward(ec_ctx* c, const void* dY, void* dX, float* dWr, float* d
 
   if (use_tc(c)) {
     // dO holds dY[idx] ungated; the dU epilogue applies the gate and forms dgate
-    EC_KERNEL("gather_dy", pz, launch_gather<T>(dYt, idx, dO, P, d, st));
+    EC_KERNEL("gather_dy", N > 0 && pz, launch_scatter_rows<T>(dYt, slot, dO, N, E, M, d, st));
     EC_TRY(ffn_backward<T>(c, kRouted, dO, at<T>(c, c->o_H), at<T>(c, c->o_A), at<T>(c, c->o_B),
                            at<T>(c, c->o_U), c->Wg, c->Wu, c->Wd, at<T>(c, c->o_dA),
                            at<T>(c, c->o_dB), dH, dWg, dWu, dWd, E, M, F, st, gate, dgate));
@@ -514,6 +516,14 @@ ec_status run_backward(ec_ctx* c, const void* dY, void* dX, float* dWr, float* d
 }
 
 // ---------------------------------------------------------------- token choice (bf16)
+// Token-major copy of X (or dY) rows into the padded expert regions, padding rows zeroed.
+cudaError_t tc_scatter(const bf16* X, const int* slot, const int* count, const int* tiles, bf16* H,
+                       int N, int E, int d, cudaStream_t st) {
+  cudaError_t e = launch_scatter_rows<bf16>(X, slot, H, N, E, 0, d, st);
+  if (e != cudaSuccess) return e;
+  return launch_zero_pad_rows<bf16>(count, tiles, H, E, d, st);
+}
+
 // Sec. 2.2 "Token-choice": router -> per-token top-k with renormalised gates and the
 // per-expert cap -> gather into padded expert regions -> variable-row expert GEMMs ->
 // gated combine through the token->row map.
@@ -542,7 +552,7 @@ ec_status run_tc_forward(ec_ctx* c, const void* X, const void* Wr, const float* 
                             row_token, row_gate, slot, at<int>(c, c->o_kept),
                             at<int>(c, c->o_tcscr), st));
   const VarRows vr{tiles, count, (int)c->P_tc};
-  EC_KERNEL("gather", 1, launch_gather<bf16>(Xt, row_token, H, c->P_tc, d, st, count + E));
+  EC_KERNEL("gather", 2, tc_scatter(Xt, slot, count, tiles, H, N, E, d, st));
   EC_KERNEL("gemm_gate_up_swiglu", 1,
             tc_expert_up(H, Wg, Wu, at<bf16>(c, c->o_A), at<bf16>(c, c->o_B), U, E, 0, d, F,
                          status, st, &vr, row_gate));
@@ -577,8 +587,7 @@ ec_status run_tc_backward(ec_ctx* c, const void* dY, void* dX, float* dWr, float
   float* row_dgate = at<float>(c, c->o_dgate);
   const int* slot = at<int>(c, c->o_slot);
   // dO = dY rows ungated; the dU epilogue applies the row gates and forms their gradients
-  EC_KERNEL("gather_dy", 1,
-            launch_gather<bf16>(dYt, at<int>(c, c->o_idx), dO, c->P_tc, d, st, count + E));
+  EC_KERNEL("gather_dy", 2, tc_scatter(dYt, slot, count, vr.tiles, dO, N, E, d, st));
   EC_KERNEL("gemm_dgrad_up_swiglu", 1,
             tc_expert_dgrad_up(dO, c->Wd, at<bf16>(c, c->o_A), at<bf16>(c, c->o_B), dA, dB, E, 0,
                                d, F, status, st, &vr, at<float>(c, c->o_gate), row_dgate,

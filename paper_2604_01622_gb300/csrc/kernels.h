@@ -46,6 +46,16 @@ cudaError_t launch_tc_softmax_bwd(const float* S, const int* choice, const float
 template <typename T>
 cudaError_t launch_gather(const T* X, const int* idx, T* H, int64_t P, int d, cudaStream_t st,
                           const int* p_used = nullptr);
+// Token-major form of the gather: for each token t, X row t is copied to row e*M + slot[t][e]
+// of H for every expert e with slot[t][e] >= 0 (M = 0: slot holds absolute rows).
+template <typename T>
+cudaError_t launch_scatter_rows(const T* X, const int* slot, T* H, int N, int E, int M, int d,
+                                cudaStream_t st);
+// Zeros the unused (padding) rows of variable-row expert regions (count [E], tiles [E+1] in
+// 256-row blocks, device arrays).
+template <typename T>
+cudaError_t launch_zero_pad_rows(const int* count, const int* tiles, T* H, int E, int d,
+                                 cudaStream_t st);
 // Y_t = R_t + R2_t (each if given) + sum over the experts that chose t of gate * O row
 // (gate NULL: 1, for O rows already scaled by their gates).
 template <typename T>

@@ -136,6 +136,62 @@ cudaError_t launch_combine(const T* O, const float* gate, const int* slot, const
   return cudaGetLastError();
 }
 
+// ------------------------------------------------------------------ token-major scatter
+// H[row] = X[t] for every (expert, row) that selected token t, one CTA per token: each X row
+// is read once (the expert-major gather above reads it once per selecting expert, mostly
+// from DRAM), and written to its rows in ascending expert order.
+template <typename T>
+__global__ void scatter_rows_kernel(const T* __restrict__ X, const int* __restrict__ slot,
+                                    T* __restrict__ H, int N, int E, int M, int d) {
+  extern __shared__ int sh[];
+  int* s_e = sh;
+  int* s_m = sh + E;
+  __shared__ int s_cnt;
+  const int t = blockIdx.x;
+  const int cnt = token_pairs(slot, nullptr, t, E, M, s_e, s_m, nullptr, &s_cnt);
+  if (cnt == 0) return;
+  const int nv = d * (int)sizeof(T) / 16;
+  const uint4* src = reinterpret_cast<const uint4*>(X + (size_t)t * d);
+  for (int v = threadIdx.x; v < nv; v += blockDim.x) {
+    const uint4 u = __ldg(src + v);
+    for (int p = 0; p < cnt; ++p)
+      reinterpret_cast<uint4*>(H + ((size_t)s_e[p] * M + s_m[p]) * d)[v] = u;
+  }
+}
+
+template <typename T>
+cudaError_t launch_scatter_rows(const T* X, const int* slot, T* H, int N, int E, int M, int d,
+                                cudaStream_t st) {
+  if (N == 0) return cudaSuccess;
+  const size_t smem = (size_t)2 * E * sizeof(int);
+  scatter_rows_kernel<T><<<N, 128, smem, st>>>(X, slot, H, N, E, M, d);
+  return cudaGetLastError();
+}
+
+// Zero the padding rows of variable-row expert regions: rows count[e] .. 256*(tiles[e+1] -
+// tiles[e]) - 1 of expert e's region (one warp per possible padding row).
+template <typename T>
+__global__ void zero_pad_rows_kernel(const int* __restrict__ count, const int* __restrict__ tiles,
+                                     T* __restrict__ H, int E, int d) {
+  const int64_t w = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  const int e = (int)(w / 256);
+  if (e >= E) return;
+  const int64_t row = (int64_t)tiles[e] * 256 + count[e] + (w % 256);
+  if (row >= (int64_t)tiles[e + 1] * 256) return;
+  uint4* dst = reinterpret_cast<uint4*>(H + row * d);
+  const int nv = d * (int)sizeof(T) / 16;
+  for (int v = lane; v < nv; v += 32) dst[v] = make_uint4(0, 0, 0, 0);
+}
+
+template <typename T>
+cudaError_t launch_zero_pad_rows(const int* count, const int* tiles, T* H, int E, int d,
+                                 cudaStream_t st) {
+  const int64_t warps = (int64_t)E * 256;
+  zero_pad_rows_kernel<T><<<(unsigned)((warps + 7) / 8), 256, 0, st>>>(count, tiles, H, E, d);
+  return cudaGetLastError();
+}
+
 // ------------------------------------------------------------------ backward: dO = g dY_t, dgate = <dY_t, O>
 template <typename T>
 __global__ void bwd_gather_scale_kernel(const T* __restrict__ dY, const T* __restrict__ O,
@@ -451,6 +507,9 @@ cudaError_t launch_reduce_splits(const float* part, float* out, int64_t n, int s
 #define ECMOE_INST(T)                                                                            \
   template cudaError_t launch_gather<T>(const T*, const int*, T*, int64_t, int, cudaStream_t,     \
                                         const int*);                                              \
+  template cudaError_t launch_scatter_rows<T>(const T*, const int*, T*, int, int, int, int,       \
+                                              cudaStream_t);                                      \
+  template cudaError_t launch_zero_pad_rows<T>(const int*, const int*, T*, int, int, cudaStream_t); \
   template cudaError_t launch_combine<T>(const T*, const float*, const int*, const T*, const T*,  \
                                          T*, int, int, int, int, cudaStream_t);                   \
   template cudaError_t launch_bwd_gather_scale<T>(const T*, const T*, const int*, const float*,   \
