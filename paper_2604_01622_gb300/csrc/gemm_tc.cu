@@ -286,6 +286,36 @@ __device__ __forceinline__ float sigmoid_fast(float a) {
   return fmaf(0.5f, t, 0.5f);
 }
 
+// Paired fp32 arithmetic (one instruction on both lanes of a 64-bit register pair, each lane
+// rounded as the scalar instruction would): the SwiGLU epilogues work on column pairs.
+__device__ __forceinline__ uint64_t f2(float lo, float hi) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+  return r;
+}
+__device__ __forceinline__ void f2_split(uint64_t r, float& lo, float& hi) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(r));
+}
+__device__ __forceinline__ uint64_t f2_fma(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+__device__ __forceinline__ uint64_t f2_mul(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+// sigmoid of both lanes, as sigmoid_fast
+__device__ __forceinline__ uint64_t f2_sigmoid(uint64_t a) {
+  const uint64_t half = f2(0.5f, 0.5f);
+  float h0, h1, t0, t1;
+  f2_split(f2_mul(a, half), h0, h1);
+  asm("tanh.approx.f32 %0, %1;" : "=f"(t0) : "f"(h0));
+  asm("tanh.approx.f32 %0, %1;" : "=f"(t1) : "f"(h1));
+  return f2_fma(f2(t0, t1), half, half);
+}
+
 // Stage this thread's row (row r of the warp's 32) of a 32 x 32 chunk for a TMA store:
 // fp32 rows of 128 bytes in the 128-byte swizzle, bf16 rows of 64 bytes in the 64-byte
 // swizzle (16-byte unit j of row r at unit j ^ (row bits of the address)), so the warp's
@@ -696,8 +726,14 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
               g[i] = no_k ? 0.f : f32(w[i]);
             }
             put2_bf16(&mO0, &mO1, n, f, g);
+            const uint64_t gs2 = f2(gs, gs);
 #pragma unroll
-            for (int i = 0; i < 32; ++i) f[i] = gs * (f[i] * sigmoid_fast(f[i]) * g[i]);
+            for (int i = 0; i < 32; i += 2) {   // U = gs * silu(A) * B, two columns at a time
+              const uint64_t a2 = f2(f[i], f[i + 1]);
+              const uint64_t u2 =
+                  f2_mul(gs2, f2_mul(f2_mul(a2, f2_sigmoid(a2)), f2(g[i], g[i + 1])));
+              f2_split(u2, f[i], f[i + 1]);
+            }
             put_bf16(&mO2, n, f);
           }
         }
@@ -722,7 +758,8 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
         };
         if (PREFETCH) fetch(c32, ra, rb);
         const float gs = (p.gate && row_ok) ? __ldg(p.gate + grow) : 1.0f;
-        float dot = 0.f;   // <acc, silu(A) * B> over this warp's columns of the row
+        // <acc, silu(A) * B> over this warp's columns of the row: even and odd columns
+        uint64_t dot2 = f2(0.f, 0.f);
 #pragma unroll 1
         for (int c = c32; c < c32 + NC32; ++c) {
           if (!PREFETCH) fetch(c, ra, rb);
@@ -741,15 +778,20 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
                 unpack16(ra[i], av + 8 * i, bf16());
                 unpack16(rb[i], bv + 8 * i, bf16());
               }
+              // two columns at a time: dU = gs acc, sg = sigma(a), dA = dU b sg (1 + a (1 - sg)),
+              // dB = dU a sg, and the gate-gradient terms acc a sg b
+              const uint64_t gs2 = f2(gs, gs), one2 = f2(1.f, 1.f), mone2 = f2(-1.f, -1.f);
 #pragma unroll
-              for (int i = 0; i < 32; ++i) {
-                const float a = av[i];
-                const float acc = f32(v[i]);
-                const float sg = sigmoid_fast(a);
-                const float das = gs * acc * sg;
-                dot = fmaf(acc, a * sg * bv[i], dot);
-                f[i] = das * bv[i] * fmaf(a, 1.0f - sg, 1.0f);
-                av[i] = das * a;
+              for (int i = 0; i < 32; i += 2) {
+                const uint64_t a2 = f2(av[i], av[i + 1]);
+                const uint64_t b2 = f2(bv[i], bv[i + 1]);
+                const uint64_t c2 = f2(f32(v[i]), f32(v[i + 1]));
+                const uint64_t sg2 = f2_sigmoid(a2);
+                const uint64_t das2 = f2_mul(f2_mul(gs2, c2), sg2);
+                dot2 = f2_fma(c2, f2_mul(f2_mul(a2, sg2), b2), dot2);
+                const uint64_t q2 = f2_fma(a2, f2_fma(sg2, mone2, one2), one2);
+                f2_split(f2_mul(f2_mul(das2, b2), q2), f[i], f[i + 1]);
+                f2_split(f2_mul(das2, a2), av[i], av[i + 1]);
               }
             }
             put2_bf16(&mO0, &mO1, n, f, av);
@@ -758,8 +800,11 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
 #pragma unroll
             for (int i = 0; i < 4; ++i) { ra[i] = na[i]; rb[i] = nb[i]; }
         }
-        if (p.dgate_part && row_ok)
-          p.dgate_part[(int64_t)(nt * NPART + part) * p.dgate_stride + grow] = dot;
+        if (p.dgate_part && row_ok) {
+          float de, dd;
+          f2_split(dot2, de, dd);
+          p.dgate_part[(int64_t)(nt * NPART + part) * p.dgate_stride + grow] = de + dd;
+        }
       } else if constexpr (EPI == EPI_ROUTER) {
         const int E = p.n_valid;
         float mx = -INFINITY;
