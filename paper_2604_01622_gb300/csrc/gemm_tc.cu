@@ -1,16 +1,19 @@
 // Persistent, warp-specialised tcgen05 GEMM for sm_103a with fused epilogues.
 //
-// One CTA per SM walks a static list of 128 x BN output tiles over a uniform batch of
+// Each CTA (or 2-CTA cluster, PAIR) walks a static list of output tiles over a batch of
 // problems (one per expert: expert choice gives every expert the same M rows, arXiv
-// 2604.01622 Sec. 2.2). Roles:
+// 2604.01622 Sec. 2.2; token choice gives each expert its own padded row region, VARM).
+// Roles:
 //   warp 0      TMA producer: 3-D tensor-map loads of A and B k-slices (64 deep, 128-byte
 //               swizzle) into a STAGES-deep shared-memory ring, one mbarrier per slot.
 //   warp 1      allocates TMEM; one thread issues tcgen05.mma (kind::f16, bf16 in, fp32
-//               accumulate) into one of two TMEM accumulators and commits slot releases
-//               and "accumulator full" to mbarriers.
-//   warps 2..5  epilogue: tcgen05.ld of the accumulator (one TMEM lane = one output row),
-//               fused math (router softmax, SwiGLU, SwiGLU backward, casts), global
-//               stores; then release the accumulator so the next tile's MMAs can reuse it.
+//               accumulate; M = 256 across the pair's two CTAs) into one of two TMEM
+//               accumulators and commits slot releases and "accumulator full" to mbarriers.
+//   warps 2..   epilogue (4 or 8 warps): tcgen05.ld of the accumulator (one TMEM lane = one
+//               output row), fused math (router softmax, SwiGLU with the gate, SwiGLU
+//               backward with the gate gradient, casts); outputs staged in swizzled shared
+//               memory and written by TMA stores; then the accumulator is released so the
+//               next tile's MMAs can reuse it.
 // Operands may be K-major or MN-major in global memory (tensor-core transpose bits), so
 // no operand is ever repacked. Every mbarrier wait is bounded in time: on expiry the CTA
 // records DEV_TIMEOUT in the status word, all roles leave their loops, and TMEM is freed.

@@ -41,11 +41,6 @@ cudaError_t launch_tc_softmax_bwd(const float* S, const int* choice, const float
                                   cudaStream_t st);
 
 // ---------------------------------------------------------------- data movement
-// H row r = X row idx[r] (zeros where idx[r] < 0), rows r < P and, if p_used is given,
-// r < *p_used (a device count).
-template <typename T>
-cudaError_t launch_gather(const T* X, const int* idx, T* H, int64_t P, int d, cudaStream_t st,
-                          const int* p_used = nullptr);
 // Token-major form of the gather: for each token t, X row t is copied to row e*M + slot[t][e]
 // of H for every expert e with slot[t][e] >= 0 (M = 0: slot holds absolute rows).
 template <typename T>
@@ -62,11 +57,10 @@ template <typename T>
 cudaError_t launch_combine(const T* O, const float* gate, const int* slot, const T* R, const T* R2,
                            T* Y, int N, int E, int M, int d, cudaStream_t st);
 // dO row r = gate[r] dY row idx[r], dgate[r] = <dY row idx[r], O row r> (zero rows where
-// idx[r] < 0); rows as in launch_gather.
+// idx[r] < 0), for the P rows (fp32 path).
 template <typename T>
 cudaError_t launch_bwd_gather_scale(const T* dY, const T* O, const int* idx, const float* gate,
-                                    T* dO, float* dgate, int64_t P, int d, cudaStream_t st,
-                                    const int* p_used = nullptr);
+                                    T* dO, float* dgate, int64_t P, int d, cudaStream_t st);
 cudaError_t launch_softmax_bwd(const float* S, const int* slot, const float* dgate, float* dZ,
                                __nv_bfloat16* dZb, int N, int E, int Ep, int M, cudaStream_t st);
 cudaError_t launch_reduce_partials(const float* part, float* out, int rows, int cols, int ld,

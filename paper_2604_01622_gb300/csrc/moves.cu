@@ -1,4 +1,4 @@
-// Bandwidth kernels of the EC-MoE layer: gather into expert-major rows, gated combine
+// Bandwidth kernels of the EC-MoE layer: token-major gather into expert rows, gated combine
 // (arXiv 2604.01622, Sec. 2.2: y_t = sum_{e: t in T_e} g_te FFN_e(x_t)), and their
 // backward (gate gradient, softmax Jacobian, scatter of the input gradient).
 //
@@ -13,34 +13,6 @@ namespace ecmoe {
 static unsigned grid_for(int64_t n, int64_t cap) {
   const int64_t b = (n + 255) / 256;
   return (unsigned)(b < cap ? b : cap);
-}
-
-// ------------------------------------------------------------------ gather H[e][m] = X[idx[e][m]]
-template <typename T>
-__global__ void gather_kernel(const T* __restrict__ X, const int* __restrict__ idx,
-                              T* __restrict__ H, int64_t P, int d, const int* __restrict__ p_used) {
-  const int64_t row = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
-  const int lane = threadIdx.x & 31;
-  if (row >= P || (p_used && row >= *p_used)) return;
-  const int t = idx[row];     // -1: a padding row of a variable-row expert region
-  const int nv = d * (int)sizeof(T) / 16;
-  uint4* dst = reinterpret_cast<uint4*>(H + (size_t)row * d);
-  if (t < 0) {
-    for (int v = lane; v < nv; v += 32) dst[v] = make_uint4(0, 0, 0, 0);
-    return;
-  }
-  const uint4* src = reinterpret_cast<const uint4*>(X + (size_t)t * d);
-  for (int v = lane; v < nv; v += 32) dst[v] = __ldg(src + v);
-}
-
-template <typename T>
-cudaError_t launch_gather(const T* X, const int* idx, T* H, int64_t P, int d, cudaStream_t st,
-                          const int* p_used) {
-  if (P == 0) return cudaSuccess;
-  const int warps = 8;
-  gather_kernel<T><<<(unsigned)((P + warps - 1) / warps), warps * 32, 0, st>>>(X, idx, H, P, d,
-                                                                                p_used);
-  return cudaGetLastError();
 }
 
 // ------------------------------------------------------------------ per-token pair lists
@@ -138,8 +110,8 @@ cudaError_t launch_combine(const T* O, const float* gate, const int* slot, const
 
 // ------------------------------------------------------------------ token-major scatter
 // H[row] = X[t] for every (expert, row) that selected token t, one CTA per token: each X row
-// is read once (the expert-major gather above reads it once per selecting expert, mostly
-// from DRAM), and written to its rows in ascending expert order.
+// is read once (an expert-major gather, row by row of H, would read it once per selecting
+// expert, mostly from DRAM), and written to its rows in ascending expert order.
 template <typename T>
 __global__ void scatter_rows_kernel(const T* __restrict__ X, const int* __restrict__ slot,
                                     T* __restrict__ H, int N, int E, int M, int d) {
@@ -197,10 +169,10 @@ template <typename T>
 __global__ void bwd_gather_scale_kernel(const T* __restrict__ dY, const T* __restrict__ O,
                                         const int* __restrict__ idx, const float* __restrict__ gate,
                                         T* __restrict__ dO, float* __restrict__ dgate, int64_t P,
-                                        int d, const int* __restrict__ p_used) {
+                                        int d) {
   const int64_t row = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
-  if (row >= P || (p_used && row >= *p_used)) return;
+  if (row >= P) return;
   const int t = idx[row];
   const float g = gate[row];
   constexpr int VN = 16 / sizeof(T);
@@ -232,12 +204,11 @@ __global__ void bwd_gather_scale_kernel(const T* __restrict__ dY, const T* __res
 
 template <typename T>
 cudaError_t launch_bwd_gather_scale(const T* dY, const T* O, const int* idx, const float* gate,
-                                    T* dO, float* dgate, int64_t P, int d, cudaStream_t st,
-                                    const int* p_used) {
+                                    T* dO, float* dgate, int64_t P, int d, cudaStream_t st) {
   if (P == 0) return cudaSuccess;
   const int warps = 8;
   bwd_gather_scale_kernel<T><<<(unsigned)((P + warps - 1) / warps), warps * 32, 0, st>>>(
-      dY, O, idx, gate, dO, dgate, P, d, p_used);
+      dY, O, idx, gate, dO, dgate, P, d);
   return cudaGetLastError();
 }
 
@@ -505,16 +476,13 @@ cudaError_t launch_reduce_splits(const float* part, float* out, int64_t n, int s
 }
 
 #define ECMOE_INST(T)                                                                            \
-  template cudaError_t launch_gather<T>(const T*, const int*, T*, int64_t, int, cudaStream_t,     \
-                                        const int*);                                              \
   template cudaError_t launch_scatter_rows<T>(const T*, const int*, T*, int, int, int, int,       \
                                               cudaStream_t);                                      \
   template cudaError_t launch_zero_pad_rows<T>(const int*, const int*, T*, int, int, cudaStream_t); \
   template cudaError_t launch_combine<T>(const T*, const float*, const int*, const T*, const T*,  \
                                          T*, int, int, int, int, cudaStream_t);                   \
   template cudaError_t launch_bwd_gather_scale<T>(const T*, const T*, const int*, const float*,   \
-                                                  T*, float*, int64_t, int, cudaStream_t,         \
-                                                  const int*);                                    \
+                                                  T*, float*, int64_t, int, cudaStream_t);        \
   template cudaError_t launch_dx_combine<T>(const T*, const int*, const float*, const T*,         \
                                             const T*, T*, int, int, int, int, cudaStream_t);      \
   template cudaError_t launch_swiglu_fwd_ew<T>(const float*, const float*, T*, T*, T*, int64_t,   \
