@@ -280,14 +280,6 @@ __host__ __device__ constexpr uint32_t smem_bytes() {
 
 __device__ __forceinline__ float f32(uint32_t u) { return __uint_as_float(u); }
 
-// Logistic sigmoid for the bf16 epilogues from the identity sigma(a) = (1 + tanh(a/2)) / 2,
-// with the hardware tanh approximation (relative error ~2^-11, below the 2^-8 of the bf16
-// values these epilogues write): one special-function op and one FMA per element.
-__device__ __forceinline__ float sigmoid_fast(float a) {
-  float t;
-  asm("tanh.approx.f32 %0, %1;" : "=f"(t) : "f"(0.5f * a));
-  return fmaf(0.5f, t, 0.5f);
-}
 
 // Paired fp32 arithmetic (one instruction on both lanes of a 64-bit register pair, each lane
 // rounded as the scalar instruction would): the SwiGLU epilogues work on column pairs.
@@ -309,7 +301,9 @@ __device__ __forceinline__ uint64_t f2_mul(uint64_t a, uint64_t b) {
   asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
   return d;
 }
-// sigmoid of both lanes, as sigmoid_fast
+// Logistic sigmoid of both lanes from the identity sigma(a) = (1 + tanh(a/2)) / 2, with the
+// hardware tanh approximation (relative error ~2^-11, below the 2^-8 of the bf16 values the
+// epilogues write): one special-function op per lane and one paired FMA.
 __device__ __forceinline__ uint64_t f2_sigmoid(uint64_t a) {
   const uint64_t half = f2(0.5f, 0.5f);
   float h0, h1, t0, t1;
