@@ -56,46 +56,67 @@ __global__ void combine_kernel(const T* __restrict__ O, const float* __restrict_
   const int cnt = token_pairs(slot, gate, t, E, M, s_e, s_m, s_g, &s_cnt);
   constexpr int VN = 16 / sizeof(T);
   const int nv = d / VN;
-  for (int v = threadIdx.x; v < nv; v += blockDim.x) {
-    float acc[VN];
-    if (R) {
-      unpack16(__ldg(reinterpret_cast<const uint4*>(R + (size_t)t * d) + v), acc, T());
-    } else {
+  // each thread sums two 16-byte column groups of the row (v and v + blockDim), eight O loads
+  // in flight; rows are summed in ascending expert order
+  const uint4* ob = reinterpret_cast<const uint4*>(O);
+  const int64_t rs = d / VN;   // uint4 per row
+  for (int v0 = threadIdx.x; v0 < nv; v0 += 2 * blockDim.x) {
+    const int v1 = v0 + blockDim.x;
+    const bool two = v1 < nv;
+    float acc0[VN], acc1[VN];
 #pragma unroll
-      for (int j = 0; j < VN; ++j) acc[j] = 0.f;
+    for (int j = 0; j < VN; ++j) acc0[j] = acc1[j] = 0.f;
+    if (R) {
+      unpack16(__ldg(reinterpret_cast<const uint4*>(R + (size_t)t * d) + v0), acc0, T());
+      if (two) unpack16(__ldg(reinterpret_cast<const uint4*>(R + (size_t)t * d) + v1), acc1, T());
     }
     if (R2) {
       float r[VN];
-      unpack16(__ldg(reinterpret_cast<const uint4*>(R2 + (size_t)t * d) + v), r, T());
+      unpack16(__ldg(reinterpret_cast<const uint4*>(R2 + (size_t)t * d) + v0), r, T());
 #pragma unroll
-      for (int j = 0; j < VN; ++j) acc[j] += r[j];
+      for (int j = 0; j < VN; ++j) acc0[j] += r[j];
+      if (two) {
+        unpack16(__ldg(reinterpret_cast<const uint4*>(R2 + (size_t)t * d) + v1), r, T());
+#pragma unroll
+        for (int j = 0; j < VN; ++j) acc1[j] += r[j];
+      }
     }
-    // rows are summed in ascending expert order; loads are issued four pairs at a time
     int p = 0;
     for (; p + 4 <= cnt; p += 4) {
-      uint4 u[4];
+      uint4 u0[4], u1[4];
 #pragma unroll
-      for (int q = 0; q < 4; ++q)
-        u[q] = __ldg(reinterpret_cast<const uint4*>(O + ((size_t)s_e[p + q] * M + s_m[p + q]) * d) + v);
+      for (int q = 0; q < 4; ++q) {
+        const int64_t row = (int64_t)s_e[p + q] * M + s_m[p + q];
+        u0[q] = __ldg(ob + row * rs + v0);
+        u1[q] = two ? __ldg(ob + row * rs + v1) : make_uint4(0, 0, 0, 0);
+      }
 #pragma unroll
       for (int q = 0; q < 4; ++q) {
         float o[VN];
-        unpack16(u[q], o, T());
         const float g = s_g[p + q];
+        unpack16(u0[q], o, T());
 #pragma unroll
-        for (int j = 0; j < VN; ++j) acc[j] = fmaf(g, o[j], acc[j]);
+        for (int j = 0; j < VN; ++j) acc0[j] = fmaf(g, o[j], acc0[j]);
+        unpack16(u1[q], o, T());
+#pragma unroll
+        for (int j = 0; j < VN; ++j) acc1[j] = fmaf(g, o[j], acc1[j]);
       }
     }
     for (; p < cnt; ++p) {
-      const size_t row = (size_t)s_e[p] * M + s_m[p];
-      const uint4 u = __ldg(reinterpret_cast<const uint4*>(O + row * d) + v);
-      float o[VN];
-      unpack16(u, o, T());
+      const int64_t row = (int64_t)s_e[p] * M + s_m[p];
       const float g = s_g[p];
+      float o[VN];
+      unpack16(__ldg(ob + row * rs + v0), o, T());
 #pragma unroll
-      for (int j = 0; j < VN; ++j) acc[j] = fmaf(g, o[j], acc[j]);
+      for (int j = 0; j < VN; ++j) acc0[j] = fmaf(g, o[j], acc0[j]);
+      if (two) {
+        unpack16(__ldg(ob + row * rs + v1), o, T());
+#pragma unroll
+        for (int j = 0; j < VN; ++j) acc1[j] = fmaf(g, o[j], acc1[j]);
+      }
     }
-    reinterpret_cast<uint4*>(Y + (size_t)t * d)[v] = pack16(acc, T());
+    reinterpret_cast<uint4*>(Y + (size_t)t * d)[v0] = pack16(acc0, T());
+    if (two) reinterpret_cast<uint4*>(Y + (size_t)t * d)[v1] = pack16(acc1, T());
   }
 }
 
