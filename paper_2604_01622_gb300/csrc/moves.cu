@@ -4,6 +4,8 @@
 //
 // The token->slot map slot[t][e] (row m of expert e, or -1) makes every per-token sum run
 // over experts in ascending order with no atomics, so results are deterministic.
+#include <algorithm>
+
 #include "common.cuh"
 #include "kernels.h"
 
@@ -81,38 +83,31 @@ __global__ void combine_kernel(const T* __restrict__ O, const float* __restrict_
         for (int j = 0; j < VN; ++j) acc1[j] += r[j];
       }
     }
-    int p = 0;
-    for (; p + 4 <= cnt; p += 4) {
+    // up to four pairs per batch (the last batch partial), all their loads issued first
+    for (int p = 0; p < cnt; p += 4) {
+      const int nb = cnt - p < 4 ? cnt - p : 4;
       uint4 u0[4], u1[4];
 #pragma unroll
       for (int q = 0; q < 4; ++q) {
-        const int64_t row = (int64_t)s_e[p + q] * M + s_m[p + q];
-        u0[q] = __ldg(ob + row * rs + v0);
-        u1[q] = two ? __ldg(ob + row * rs + v1) : make_uint4(0, 0, 0, 0);
+        u0[q] = u1[q] = make_uint4(0, 0, 0, 0);
+        if (q < nb) {
+          const int64_t row = (int64_t)s_e[p + q] * M + s_m[p + q];
+          u0[q] = __ldg(ob + row * rs + v0);
+          if (two) u1[q] = __ldg(ob + row * rs + v1);
+        }
       }
 #pragma unroll
       for (int q = 0; q < 4; ++q) {
-        float o[VN];
-        const float g = s_g[p + q];
-        unpack16(u0[q], o, T());
+        if (q < nb) {
+          float o[VN];
+          const float g = s_g[p + q];
+          unpack16(u0[q], o, T());
 #pragma unroll
-        for (int j = 0; j < VN; ++j) acc0[j] = fmaf(g, o[j], acc0[j]);
-        unpack16(u1[q], o, T());
+          for (int j = 0; j < VN; ++j) acc0[j] = fmaf(g, o[j], acc0[j]);
+          unpack16(u1[q], o, T());
 #pragma unroll
-        for (int j = 0; j < VN; ++j) acc1[j] = fmaf(g, o[j], acc1[j]);
-      }
-    }
-    for (; p < cnt; ++p) {
-      const int64_t row = (int64_t)s_e[p] * M + s_m[p];
-      const float g = s_g[p];
-      float o[VN];
-      unpack16(__ldg(ob + row * rs + v0), o, T());
-#pragma unroll
-      for (int j = 0; j < VN; ++j) acc0[j] = fmaf(g, o[j], acc0[j]);
-      if (two) {
-        unpack16(__ldg(ob + row * rs + v1), o, T());
-#pragma unroll
-        for (int j = 0; j < VN; ++j) acc1[j] = fmaf(g, o[j], acc1[j]);
+          for (int j = 0; j < VN; ++j) acc1[j] = fmaf(g, o[j], acc1[j]);
+        }
       }
     }
     reinterpret_cast<uint4*>(Y + (size_t)t * d)[v0] = pack16(acc0, T());
@@ -125,7 +120,10 @@ cudaError_t launch_combine(const T* O, const float* gate, const int* slot, const
                            T* Y, int N, int E, int M, int d, cudaStream_t st) {
   if (N == 0) return cudaSuccess;
   const size_t smem = (size_t)3 * E * sizeof(int);
-  combine_kernel<T><<<N, 128, smem, st>>>(O, gate, slot, R, R2, Y, N, E, M, d);
+  // two 16-byte column groups per thread: half a row's groups per CTA, 32 to 128 threads
+  const int nv = d * (int)sizeof(T) / 16;
+  const int threads = std::min(128, std::max(32, (nv / 2 + 31) / 32 * 32));
+  combine_kernel<T><<<N, threads, smem, st>>>(O, gate, slot, R, R2, Y, N, E, M, d);
   return cudaGetLastError();
 }
 
