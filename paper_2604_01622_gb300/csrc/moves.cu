@@ -323,39 +323,67 @@ __global__ void dx_combine_kernel(const T* __restrict__ dH, const int* __restric
   const int cnt = token_pairs(slot, nullptr, t, E, M, s_e, s_m, nullptr, &s_cnt);
   constexpr int VN = 16 / sizeof(T);
   const int nv = d / VN;
-  for (int v = threadIdx.x; v < nv; v += blockDim.x) {
-    float acc[VN];
-    if (dXr) {
-      const float4* r = reinterpret_cast<const float4*>(dXr + (size_t)t * d + (size_t)v * VN);
+  // as the combine: two 16-byte column groups per thread, up to four dH rows per batch with
+  // all their loads issued first; rows added in ascending expert order
+  const uint4* hb = reinterpret_cast<const uint4*>(dH);
+  const int64_t rs = d / VN;
+  for (int v0 = threadIdx.x; v0 < nv; v0 += 2 * blockDim.x) {
+    const int v1 = v0 + blockDim.x;
+    const bool two = v1 < nv;
+    float acc0[VN], acc1[VN];
+    auto init = [&](int v, float* acc) {
+      if (dXr) {
+        const float4* r = reinterpret_cast<const float4*>(dXr + (size_t)t * d + (size_t)v * VN);
 #pragma unroll
-      for (int j = 0; j < VN / 4; ++j) {
-        float4 q = r[j];
-        acc[4 * j] = q.x; acc[4 * j + 1] = q.y; acc[4 * j + 2] = q.z; acc[4 * j + 3] = q.w;
+        for (int j = 0; j < VN / 4; ++j) {
+          const float4 q = r[j];
+          acc[4 * j] = q.x; acc[4 * j + 1] = q.y; acc[4 * j + 2] = q.z; acc[4 * j + 3] = q.w;
+        }
+      } else {
+#pragma unroll
+        for (int j = 0; j < VN; ++j) acc[j] = 0.f;
       }
-    } else {
-#pragma unroll
-      for (int j = 0; j < VN; ++j) acc[j] = 0.f;
-    }
-    if (R) {
       float r[VN];
-      unpack16(__ldg(reinterpret_cast<const uint4*>(R + (size_t)t * d) + v), r, T());
+      if (R) {
+        unpack16(__ldg(reinterpret_cast<const uint4*>(R + (size_t)t * d) + v), r, T());
 #pragma unroll
-      for (int j = 0; j < VN; ++j) acc[j] += r[j];
-    }
-    if (R2) {
-      float r[VN];
-      unpack16(__ldg(reinterpret_cast<const uint4*>(R2 + (size_t)t * d) + v), r, T());
+        for (int j = 0; j < VN; ++j) acc[j] += r[j];
+      }
+      if (R2) {
+        unpack16(__ldg(reinterpret_cast<const uint4*>(R2 + (size_t)t * d) + v), r, T());
 #pragma unroll
-      for (int j = 0; j < VN; ++j) acc[j] += r[j];
-    }
-    for (int p = 0; p < cnt; ++p) {
-      const size_t row = (size_t)s_e[p] * M + s_m[p];
-      float h[VN];
-      unpack16(__ldg(reinterpret_cast<const uint4*>(dH + row * d) + v), h, T());
+        for (int j = 0; j < VN; ++j) acc[j] += r[j];
+      }
+    };
+    init(v0, acc0);
+    if (two) init(v1, acc1);
+    for (int p = 0; p < cnt; p += 4) {
+      const int nb = cnt - p < 4 ? cnt - p : 4;
+      uint4 u0[4], u1[4];
 #pragma unroll
-      for (int j = 0; j < VN; ++j) acc[j] += h[j];
+      for (int q = 0; q < 4; ++q) {
+        u0[q] = u1[q] = make_uint4(0, 0, 0, 0);
+        if (q < nb) {
+          const int64_t row = (int64_t)s_e[p + q] * M + s_m[p + q];
+          u0[q] = __ldg(hb + row * rs + v0);
+          if (two) u1[q] = __ldg(hb + row * rs + v1);
+        }
+      }
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        if (q < nb) {
+          float h[VN];
+          unpack16(u0[q], h, T());
+#pragma unroll
+          for (int j = 0; j < VN; ++j) acc0[j] += h[j];
+          unpack16(u1[q], h, T());
+#pragma unroll
+          for (int j = 0; j < VN; ++j) acc1[j] += h[j];
+        }
+      }
     }
-    reinterpret_cast<uint4*>(dX + (size_t)t * d)[v] = pack16(acc, T());
+    reinterpret_cast<uint4*>(dX + (size_t)t * d)[v0] = pack16(acc0, T());
+    if (two) reinterpret_cast<uint4*>(dX + (size_t)t * d)[v1] = pack16(acc1, T());
   }
 }
 
@@ -364,7 +392,9 @@ cudaError_t launch_dx_combine(const T* dH, const int* slot, const float* dXr, co
                               const T* R2, T* dX, int N, int E, int M, int d, cudaStream_t st) {
   if (N == 0) return cudaSuccess;
   const size_t smem = (size_t)2 * E * sizeof(int);
-  dx_combine_kernel<T><<<N, 128, smem, st>>>(dH, slot, dXr, R, R2, dX, N, E, M, d);
+  const int nv = d * (int)sizeof(T) / 16;
+  const int threads = std::min(128, std::max(32, (nv / 2 + 31) / 32 * 32));
+  dx_combine_kernel<T><<<N, threads, smem, st>>>(dH, slot, dXr, R, R2, dX, N, E, M, d);
   return cudaGetLastError();
 }
 
