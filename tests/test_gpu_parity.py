@@ -152,3 +152,45 @@ def test_set_capacity_matches_fresh_context():
     lay.check()
     fresh.check()
     assert torch.equal(idx1, idx2) and torch.equal(Y1, Y2)
+
+
+# ------------------------------------------------------------------ bf16 edge cases
+def test_bf16_ragged_groups_and_capacity_edges():
+    """Tensor-core path with an empty group, a one-token group, k = 0 and k = L: 11 experts
+    of M = 168 rows (one 128-row tile and a 40-row tail) over 333 tokens."""
+    w = I.scaled(I.WORKLOADS["ec_d2048_e64"], G=1, L=333, d=128, E=11, d_ff=64, seed=13,
+                 router_bias=True, layers=1)
+    inp = I.make_inputs(w)
+    inp.group_off = np.array([0, 0, 150, 151, 333], np.int32)
+    inp.k_g = np.array([0, 150, 1, 17], np.int32)
+    _check_layer(inp)
+
+
+def test_bf16_few_tokens_minimum_widths():
+    """Five tokens, d = d_ff = 64 (one k-step, one column block): M = 2 rows per expert."""
+    w = I.scaled(I.WORKLOADS["ec_d2048_e64"], G=1, L=5, d=64, E=3, d_ff=64, k_base=2, seed=15,
+                 layers=1)
+    _check_layer(I.make_inputs(w))
+
+
+def test_bf16_single_expert_is_a_dense_mlp():
+    """E = 1 and k = L: every token goes to the one expert with gate S = 1 (a plain SwiGLU
+    MLP), and the router gets no gradient: dZ = S (dS - <dS, S>) is exactly zero."""
+    w = I.scaled(I.WORKLOADS["ec_d2048_e64"], G=2, L=200, d=64, E=1, d_ff=128, k_base=200,
+                 seed=14, layers=1)
+    inp = I.make_inputs(w)
+    _, out = gpu_layer(inp)
+    assert not out["dWr"].any()
+    assert torch.equal(out["gate"], torch.ones_like(out["gate"]))
+    _check_layer(inp)
+
+
+def test_bf16_zero_capacity_everywhere():
+    """k_g = 0 in every group: no expert rows, so Y, dX and every gradient are exact zeros."""
+    w = I.scaled(I.WORKLOADS["ec_d2048_e64"], G=2, L=100, d=128, E=4, d_ff=64, k_base=0,
+                 seed=16, router_bias=True, layers=1)
+    inp = I.make_inputs(w)
+    _, out = gpu_layer(inp)
+    assert out["idx"].numel() == 0
+    for k in ("Y", "dX", "dWr", "dbr", "dWg", "dWu", "dWd"):
+        assert not out[k].any(), k

@@ -66,6 +66,8 @@ CASES = [
     ("ragged_e12_k3", dict(L=350, E=12, router_bias=True), 3, 0.6),
     # 100 experts over two 64-column router tiles, every expert a tail of 256-row padding
     ("e100_k5", dict(L=384, E=100, d=64, d_ff=64), 5, None),
+    # one expert: every token's single choice, normalised gate 1, no router gradient
+    ("e1_k1", dict(E=1, L=300), 1, None),
 ]
 
 
