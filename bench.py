@@ -39,6 +39,7 @@ UNIT = "tokens/s"
 # DRAM traffic per launch of the grouped-GEMM kernels, from one ncu capture of this
 # workload (dram__bytes_read.sum + dram__bytes_write.sum), keyed by the hash of the
 # kernel source it was taken on; a changed kernel reports null until re-captured.
+TILE_POLICY = {"auto": 0, "256": 1, "512": 2}   # EC_TILES_AUTO / EC_TILES_256 / EC_TILES_512
 TRAFFIC = {"c96e6ee59950": 2863566891}   # mean of the six expert-GEMM launches of one step
 
 
@@ -270,6 +271,7 @@ def run_ours(args):
                                device=device, d_ff_shared=Fs)
         if w.layers > 1:
             lay_l.set_residual(True)
+        lay_l.set_tiles(TILE_POLICY[args.tiles])
         g = {"dX": torch.empty_like(X),
              "dWr": torch.empty(w.d, w.E, dtype=torch.float32, device=device),
              "dbr": None if Ld.br is None else torch.empty(w.E, dtype=torch.float32,
@@ -497,6 +499,7 @@ def run_ours(args):
         "config": {"workload": w.name, "sequences": w.G, "seq_len": w.L, "tokens": w.N,
                    "d_model": w.d, "experts": w.E, "d_ff": w.d_ff, "k_per_seq": w.k_base,
                    "layers": w.layers, "shared_experts": args.shared_experts,
+                   "tiles": args.tiles,
                    "parallelism": f"replicas{ws}" if ws > 1 else "single",
                    "l2": "inputs and activations larger than L2 (no flush)"},
     }
@@ -591,6 +594,8 @@ def main():
                     help="token-choice capacity factor (default: dropless)")
     ap.add_argument("--tc-cpu-tokens", type=int, default=32,
                     help="tokens of the token-choice oracle's CPU sample (both arms)")
+    ap.add_argument("--tiles", choices=sorted(TILE_POLICY), default="auto",
+                    help="expert-GEMM tile policy (bf16 path): auto, 256 or 512 columns")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-tokens", type=int, default=8192,
                     help="tokens of the oracle's CPU baseline sample")

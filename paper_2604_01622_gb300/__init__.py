@@ -28,8 +28,9 @@ EXPORTS = (
     "ec_ctx_set_profiling", "ec_ctx_profile", "ec_kernel_launches", "ec_select_static",
     "ec_selftest_bounded_wait", "ec_ctx_set_residual", "ec_capacity_schedule",
     "ec_ctx_set_shared", "ec_moe_forward_shared", "ec_moe_backward_shared",
-    "ec_tc_ctx_create", "ec_tc_forward", "ec_tc_backward",
+    "ec_tc_ctx_create", "ec_tc_forward", "ec_tc_backward", "ec_ctx_set_tiles",
 )
+EC_TILES_AUTO, EC_TILES_256, EC_TILES_512 = 0, 1, 2
 
 EC_SCHEDULERS = {"static": 0, "linear": 1, "linear_reverse": 2, "cosine": 3,
                  "cosine_reverse": 4, "gaussian": 5, "gaussian_reverse": 6}
@@ -74,6 +75,7 @@ def load():
         "ec_select_static": (i32, [vp, i32, i32, i32, P32, P32, vp, vp, vp]),
         "ec_selftest_bounded_wait": (i32, [vp, ctypes.c_uint64, vp]),
         "ec_ctx_set_residual": (i32, [vp, i32]),
+        "ec_ctx_set_tiles": (i32, [vp, i32]),
         "ec_ctx_set_shared": (i32, [vp, i32]),
         "ec_moe_forward_shared": (i32, [vp] * 15),
         "ec_moe_backward_shared": (i32, [vp] * 12),
@@ -128,6 +130,10 @@ def ec_ctx_set_capacity(ctx, k_g):
 
 def ec_ctx_set_residual(ctx, on: bool):
     _check(ctx, load().ec_ctx_set_residual(ctx, 1 if on else 0))
+
+
+def ec_ctx_set_tiles(ctx, policy: int):
+    _check(ctx, load().ec_ctx_set_tiles(ctx, int(policy)))
 
 
 def ec_rows_per_expert(ctx) -> int:

@@ -49,6 +49,7 @@ struct ec_ctx {
   // token choice (k > 0): k experts per token, per-expert cap (< 0: none), padded rows
   int tc_k = 0, tc_cap = -1;
   int64_t P_tc = 0;
+  int tiles = EC_TILES_AUTO;   // expert-GEMM tile policy (ec_ctx_set_tiles)
   size_t o_choice = 0, o_tgate = 0, o_Zs = 0, o_count = 0, o_tiles = 0, o_kept = 0, o_tcscr = 0;
   std::string err;
 };
@@ -316,8 +317,9 @@ ec_status ffn_forward(ec_ctx* c, const FfnNames& nm, const T* H, const void* Wg,
   if (P == 0) return EC_OK;
   int* status = at<int>(c, c->o_status);
   if (use_tc(c)) {
-    EC_KERNEL(nm.up, 1, tc_expert_up(H, Wg, Wu, A, B, U, E, M, d, F, status, st, nullptr, gate));
-    EC_KERNEL(nm.down, 1, tc_expert_down(U, Wd, O, E, M, d, F, status, st));
+    EC_KERNEL(nm.up, 1,
+              tc_expert_up(H, Wg, Wu, A, B, U, E, M, d, F, status, st, nullptr, gate, c->tiles));
+    EC_KERNEL(nm.down, 1, tc_expert_down(U, Wd, O, E, M, d, F, status, st, nullptr, c->tiles));
   } else {
     float* Ag = at<float>(c, c->o_f32a);
     float* Bu = at<float>(c, c->o_f32b);
@@ -359,9 +361,11 @@ ec_status ffn_backward(ec_ctx* c, const FfnNames& nm, const T* dO, const T* H, c
     EC_KERNEL(nm.dgrad_up, 1,
               tc_expert_dgrad_up(dO, Wd, A, B, dA, dB, E, M, d, F, status, st, nullptr, gate,
                                  dgate_part, P));
-    EC_KERNEL(nm.dgrad_h, 1, tc_expert_dgrad_h(dA, dB, Wg, Wu, dH, E, M, d, F, status, st));
+    EC_KERNEL(nm.dgrad_h, 1,
+              tc_expert_dgrad_h(dA, dB, Wg, Wu, dH, E, M, d, F, status, st, nullptr, c->tiles));
     EC_KERNEL(nm.wgrad, 2,
-              tc_expert_wgrad(H, U, dO, dA, dB, dWg, dWu, dWd, E, M, d, F, status, st));
+              tc_expert_wgrad(H, U, dO, dA, dB, dWg, dWu, dWd, E, M, d, F, status, st, nullptr,
+                              c->tiles));
   } else {
     float* dU32 = at<float>(c, c->o_f32a);
     float* dH32 = at<float>(c, c->o_f32b);
@@ -555,8 +559,8 @@ ec_status run_tc_forward(ec_ctx* c, const void* X, const void* Wr, const float* 
   EC_KERNEL("gather", 2, tc_scatter(Xt, slot, count, tiles, H, N, E, d, st));
   EC_KERNEL("gemm_gate_up_swiglu", 1,
             tc_expert_up(H, Wg, Wu, at<bf16>(c, c->o_A), at<bf16>(c, c->o_B), U, E, 0, d, F,
-                         status, st, &vr, row_gate));
-  EC_KERNEL("gemm_down", 1, tc_expert_down(U, Wd, O, E, 0, d, F, status, st, &vr));
+                         status, st, &vr, row_gate, c->tiles));
+  EC_KERNEL("gemm_down", 1, tc_expert_down(U, Wd, O, E, 0, d, F, status, st, &vr, c->tiles));
   EC_KERNEL("combine", 1,
             launch_combine<bf16>(O, nullptr, slot, c->residual ? Xt : nullptr, nullptr,
                                  static_cast<bf16*>(Y), N, E, 0, d, st));
@@ -593,10 +597,10 @@ ec_status run_tc_backward(ec_ctx* c, const void* dY, void* dX, float* dWr, float
                                d, F, status, st, &vr, at<float>(c, c->o_gate), row_dgate,
                                c->P_tc));
   EC_KERNEL("gemm_dgrad_h", 1,
-            tc_expert_dgrad_h(dA, dB, c->Wg, c->Wu, dH, E, 0, d, F, status, st, &vr));
+            tc_expert_dgrad_h(dA, dB, c->Wg, c->Wu, dH, E, 0, d, F, status, st, &vr, c->tiles));
   EC_KERNEL("gemm_wgrad", 2,
             tc_expert_wgrad(at<bf16>(c, c->o_H), at<bf16>(c, c->o_U), dO, dA, dB, dWg, dWu, dWd, E,
-                            0, d, F, status, st, &vr));
+                            0, d, F, status, st, &vr, c->tiles));
   float* dZ = at<float>(c, c->o_dZ);
   bf16* dZb = at<bf16>(c, c->o_dZb);
   float* dXr = at<float>(c, c->o_dXr);
@@ -897,6 +901,14 @@ ec_status ec_ctx_set_residual(ec_ctx* c, int32_t on) {
   if (!c) return EC_ERR_INVALID_ARG;
   c->residual = on != 0;
   c->have_fwd = false;
+  return EC_OK;
+}
+
+ec_status ec_ctx_set_tiles(ec_ctx* c, int32_t policy) {
+  if (!c) return EC_ERR_INVALID_ARG;
+  if (policy != EC_TILES_AUTO && policy != EC_TILES_256 && policy != EC_TILES_512)
+    return fail(c, EC_ERR_INVALID_ARG, "tile policy %d is not one of 0, 1, 2", policy);
+  c->tiles = policy;
   return EC_OK;
 }
 

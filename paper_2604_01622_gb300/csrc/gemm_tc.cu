@@ -8,7 +8,8 @@
 //               swizzle) into a STAGES-deep shared-memory ring, one mbarrier per slot.
 //   warp 1      allocates TMEM; one thread issues tcgen05.mma (kind::f16, bf16 in, fp32
 //               accumulate; M = 256 across the pair's two CTAs) into one of two TMEM
-//               accumulators and commits slot releases and "accumulator full" to mbarriers.
+//               accumulators (or, for 256 x 512 tiles, into the two halves of one that fills
+//               TMEM) and commits slot releases and "accumulator full" to mbarriers.
 //   warps 2..   epilogue (4 or 8 warps): tcgen05.ld of the accumulator (one TMEM lane = one
 //               output row), fused math (router softmax, SwiGLU with the gate, SwiGLU
 //               backward with the gate gradient, casts); outputs staged in swizzled shared
@@ -405,6 +406,14 @@ __device__ __forceinline__ Tile tile_at(const Args& p, int tile, int tiles_per_b
 // of A and half (BN/2 columns) of B; the leader CTA (rank 0) issues M = 256 MMAs that read
 // both CTAs' shared memory and write each CTA's 128 rows into that CTA's TMEM. Per SM this
 // halves the B traffic into shared memory.
+//
+// Wide tiles (BN = 512, pairs only): each k-slice feeds two N = 256 MMAs from one A slice, so
+// an SM takes in 48 KB of operands per 2 x 128 x 256 x 64 MMA work instead of 32 KB per half
+// of it (25% fewer bytes per FLOP). The accumulator then fills all 512 TMEM columns, so the
+// two 256-column halves are handed over separately: the last TAIL k-slices issue their
+// half-1 MMAs after half 0 has completed (the epilogue drains half 0 while they run), and the
+// next tile issues its half-0 MMAs as soon as half 0 is free, holding its k-slices for the
+// half-1 MMAs until the epilogue has drained half 1.
 template <int BN, bool A_MN, bool B_MN, bool B_SPLIT, bool K_SPLIT, int EPI, int STAGES, int EPW,
           bool PAIR, int VARM>
 __global__ void __launch_bounds__(64 + 32 * EPW, 1)
@@ -412,14 +421,20 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
                const __grid_constant__ CUtensorMap mB0, const __grid_constant__ CUtensorMap mB1,
                const __grid_constant__ CUtensorMap mO0, const __grid_constant__ CUtensorMap mO1,
                const __grid_constant__ CUtensorMap mO2, const Args p) {
+  constexpr bool WIDE = BN == 512;            // single accumulator handed over in two halves
+  constexpr int NH = WIDE ? 2 : 1;            // accumulator segments per tile
+  constexpr int SEGW = BN / NH;               // columns per segment = N of one MMA
+  constexpr int TAIL = 3;                     // wide: k-slices whose half-1 MMAs go last
   constexpr int BNL = PAIR ? BN / 2 : BN;     // B columns held by this CTA
   constexpr int TM = PAIR ? 2 * BM : BM;      // tile rows
   constexpr uint32_t A_BYTES = BM * BK * 2;
   constexpr uint32_t B_BYTES = BNL * BK * 2;
-  constexpr uint32_t TCOLS = tmem_cols<BN>();
-  constexpr uint32_t IDESC = instr_desc<BN, A_MN, B_MN, TM>();
-  static_assert(BN % 64 == 0 && BN <= 256, "BN");
+  constexpr uint32_t TCOLS = WIDE ? 512u : tmem_cols<BN>();
+  constexpr uint32_t IDESC = instr_desc<SEGW, A_MN, B_MN, TM>();
+  static_assert(BN % 64 == 0 && (BN <= 256 || (WIDE && PAIR)), "BN");
   static_assert(!PAIR || BN % 128 == 0, "pair tiles split B in two 64-column multiples");
+  static_assert(!WIDE || (EPI != EPI_SWIGLU_BWD && EPI != EPI_ROUTER && STAGES > TAIL),
+                "wide tiles: plain, split-column and SwiGLU forward epilogues");
   static_assert(EPW == 4 || EPW == 8, "epilogue warps: one or two per TMEM lane quarter");
   static_assert(EPI != EPI_ROUTER || EPW == 4, "the row softmax needs whole rows per thread");
   // every epilogue except the router's writes through shared memory and TMA stores
@@ -520,14 +535,20 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
             for (int j = 0; j < BM / 64; ++j) load_b(a_dst + j * 8192, mA, m0 + 64 * j, k0, ab);
           }
           if constexpr (PAIR) {
-            // this CTA's half of the B tile: for split tiles the gate (rank 0) or up half
+            // this CTA's half of each segment's B columns: for split tiles the gate (rank 0)
+            // or up half
             const CUtensorMap* mb = B_SPLIT ? (rank ? &mB1 : &mB0) : mB;
-            const int n0 = B_SPLIT ? nt * (BN / 2) : nt * BN + (int)rank * BNL;
-            if (!B_MN) {
-              load(b_dst, mb, k0, n0);
-            } else {
 #pragma unroll
-              for (int j = 0; j < BNL / 64; ++j) load(b_dst + j * 8192, mb, n0 + 64 * j, k0);
+            for (int h = 0; h < NH; ++h) {
+              uint8_t* bh = b_dst + h * (B_BYTES / NH);
+              const int n0 = B_SPLIT ? nt * (BN / 2) + h * (SEGW / 2)
+                                     : nt * BN + h * SEGW + (int)rank * (BNL / NH);
+              if (!B_MN) {
+                load(bh, mb, k0, n0);
+              } else {
+#pragma unroll
+                for (int j = 0; j < BNL / NH / 64; ++j) load(bh + j * 8192, mb, n0 + 64 * j, k0);
+              }
             }
           } else if (!B_MN) {
             if constexpr (B_SPLIT) {
@@ -567,34 +588,98 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
       uint32_t ph = 0;
       bool ok = true;
       int it = 0;
-      for (int tile = cid; tile < total && ok; tile += nwalk, ++it) {
-        const int a = it & 1;
-        const uint32_t use = (uint32_t)(it >> 1);
-        const int kbl = tile_at<VARM, TM>(p, tile, tiles_per_b, 0).kbl;
-        if (!mbar_wait(&tempty[a], (use & 1u) ^ 1u, abort_flag, p.status)) { ok = false; break; }
-        tc_fence_after();
-        const uint32_t tacc = tmem_base + (uint32_t)(a * BN);
-        for (int kb = 0; kb < kbl; ++kb) {
-          if (!mbar_wait(&full[s], ph, abort_flag, p.status)) { ok = false; break; }
-          tc_fence_after();
-          const uint32_t sa = smem_u32(sA + s * A_BYTES);
-          const uint32_t sb = smem_u32(sB + s * B_BYTES);
+      // the BK/16 MMAs of ring slot `st` with B segment h into TMEM column `tcol`; `first`: the
+      // tile's first k-slice (the accumulator starts from zero)
+      auto issue = [&](int st, int h, uint32_t tcol, bool first) {
+        const uint32_t sa = smem_u32(sA + st * A_BYTES);
+        const uint32_t sb = smem_u32(sB + st * B_BYTES + h * (B_BYTES / NH));
 #pragma unroll
-          for (int j = 0; j < BK / 16; ++j) {
-            const uint64_t ad = A_MN ? smem_desc(sa + j * 2048, 8192, 1024)
-                                     : smem_desc(sa + j * 32, 16, 1024);
-            const uint64_t bd = B_MN ? smem_desc(sb + j * 2048, 8192, 1024)
-                                     : smem_desc(sb + j * 32, 16, 1024);
-            if constexpr (PAIR) mma_bf16_pair(tacc, ad, bd, IDESC, (kb | j) != 0 ? 1u : 0u);
-            else mma_bf16(tacc, ad, bd, IDESC, (kb | j) != 0 ? 1u : 0u);
-          }
-          if constexpr (PAIR) mma_commit_pair(&empty[s], 0x3);
-          else mma_commit(&empty[s]);
-          if (++s == STAGES) { s = 0; ph ^= 1u; }
+        for (int j = 0; j < BK / 16; ++j) {
+          const uint64_t ad = A_MN ? smem_desc(sa + j * 2048, 8192, 1024)
+                                   : smem_desc(sa + j * 32, 16, 1024);
+          const uint64_t bd = B_MN ? smem_desc(sb + j * 2048, 8192, 1024)
+                                   : smem_desc(sb + j * 32, 16, 1024);
+          const uint32_t acc = (!first || j != 0) ? 1u : 0u;
+          if constexpr (PAIR) mma_bf16_pair(tcol, ad, bd, IDESC, acc);
+          else mma_bf16(tcol, ad, bd, IDESC, acc);
         }
-        if (!ok) break;
-        if constexpr (PAIR) mma_commit_pair(&tfull[a], 0x3);
-        else mma_commit(&tfull[a]);
+      };
+      // arrive on `bar` (in both CTAs of a pair) once the MMAs issued so far have completed
+      auto commit = [&](uint64_t* bar) {
+        if constexpr (PAIR) mma_commit_pair(bar, 0x3);
+        else mma_commit(bar);
+      };
+      for (int tile = cid; tile < total && ok; tile += nwalk, ++it) {
+        const int kbl = tile_at<VARM, TM>(p, tile, tiles_per_b, 0).kbl;
+        if constexpr (!WIDE) {
+          const int a = it & 1;
+          const uint32_t use = (uint32_t)(it >> 1);
+          if (!mbar_wait(&tempty[a], (use & 1u) ^ 1u, abort_flag, p.status)) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t tacc = tmem_base + (uint32_t)(a * BN);
+          for (int kb = 0; kb < kbl; ++kb) {
+            if (!mbar_wait(&full[s], ph, abort_flag, p.status)) { ok = false; break; }
+            tc_fence_after();
+            issue(s, 0, tacc, kb == 0);
+            commit(&empty[s]);
+            if (++s == STAGES) { s = 0; ph ^= 1u; }
+          }
+          if (!ok) break;
+          commit(&tfull[a]);
+        } else {
+          // segment h of the single accumulator: TMEM columns [h*SEGW, (h+1)*SEGW)
+          const uint32_t par = ((uint32_t)it & 1u) ^ 1u;   // previous tile's release of a half
+          if (!mbar_wait(&tempty[0], par, abort_flag, p.status)) { ok = false; break; }
+          tc_fence_after();
+          bool h1 = mbar_try_wait(smem_u32(&tempty[1]), par);
+          if (h1) tc_fence_after();
+          // k-slices whose half-1 MMAs are still to be issued: `held` consecutive ones from
+          // k-slice pk in ring slot ps (their slots stay occupied until then)
+          int held = 0, pk = 0, ps = s;
+          auto flush = [&]() {
+            int st = ps;
+            for (int i = 0; i < held; ++i) {
+              issue(st, 1, tmem_base + SEGW, pk + i == 0);
+              commit(&empty[st]);
+              if (++st == STAGES) st = 0;
+            }
+            held = 0;
+          };
+          for (int kb = 0; kb < kbl; ++kb) {
+            if (!h1) {
+              // every slot held: the producer is stalled, so wait for half 1 here
+              if (held == STAGES) {
+                if (!mbar_wait(&tempty[1], par, abort_flag, p.status)) { ok = false; break; }
+                h1 = true;
+              } else {
+                h1 = mbar_try_wait(smem_u32(&tempty[1]), par);
+              }
+              if (h1) {
+                tc_fence_after();
+                flush();
+              }
+            }
+            if (!mbar_wait(&full[s], ph, abort_flag, p.status)) { ok = false; break; }
+            tc_fence_after();
+            issue(s, 0, tmem_base, kb == 0);
+            if (h1 && kb < kbl - TAIL) {
+              issue(s, 1, tmem_base + SEGW, kb == 0);
+              commit(&empty[s]);
+            } else {
+              if (held == 0) { pk = kb; ps = s; }
+              ++held;
+            }
+            if (++s == STAGES) { s = 0; ph ^= 1u; }
+          }
+          if (!ok) break;
+          commit(&tfull[0]);   // half 0 is final once the MMAs issued so far complete
+          if (!h1) {
+            if (!mbar_wait(&tempty[1], par, abort_flag, p.status)) { ok = false; break; }
+            tc_fence_after();
+          }
+          flush();
+          commit(&tfull[1]);
+        }
       }
       if (!ok) {
         // wait for the MMAs already issued before TMEM is released
@@ -613,11 +698,8 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
     const int part = (warp - 2) / 4;
     int slot = 0;   // staging half of the next bf16 chunk (warp-uniform)
     int it = 0;
-    for (int tile = cid; tile < total; tile += nwalk, ++it) {
-      const int a = it & 1;
-      const uint32_t use = (uint32_t)(it >> 1);
-      if (!mbar_wait(&tfull[a], use & 1u, abort_flag, p.status)) break;
-      tc_fence_after();
+    bool stop = false;
+    for (int tile = cid; tile < total && !stop; tile += nwalk, ++it) {
       const Tile T = tile_at<VARM, TM>(p, tile, tiles_per_b, rank);
       const int nt = T.nt;
       const int gm = T.row0 + r;
@@ -625,7 +707,6 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
       // Variable rows: a 256-row tile never leaves its expert's padded region, and the
       // region's unused rows are written as zeros (the weight gradients run their K loop
       // over them). Uniform batches store only the valid rows.
-      const uint32_t tacc = tmem_base + (uint32_t)(a * BN) + ((uint32_t)(q * 32) << 16);
       const int64_t row_off =
           VARM == 1 ? (int64_t)gm * p.ld : (int64_t)T.b * p.bstride + (int64_t)gm * p.ld;
       const int64_t grow = VARM == 1 ? (int64_t)gm : (int64_t)T.b * p.M + gm;   // gate row
@@ -677,14 +758,24 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
         if (lane == 0) tma_store_3d(m, smem_u32(b), n, srow, sbat);
       };
 
-      constexpr int NC32 = BN / 32 / NPART;   // 32-column chunks per warp
+      // The accumulator segments (one, or a wide tile's two halves, each released as soon
+      // as it is drained): segment h holds tile columns [h*SEGW, (h+1)*SEGW).
+      for (int h = 0; h < NH; ++h) {
+      const int a = WIDE ? h : (it & 1);
+      const uint32_t par = WIDE ? (uint32_t)(it & 1) : (uint32_t)((it >> 1) & 1);
+      if (!mbar_wait(&tfull[a], par, abort_flag, p.status)) { stop = true; break; }
+      tc_fence_after();
+      const uint32_t tacc = tmem_base + (uint32_t)(WIDE ? h * SEGW : a * BN) +
+                            ((uint32_t)(q * 32) << 16);
+      const int cb = h * SEGW;                   // first tile column of the segment
+      constexpr int NC32 = SEGW / 32 / NPART;    // 32-column chunks per warp
       const int c32 = part * NC32;
       if constexpr (EPI == EPI_STORE_BF16 || EPI == EPI_STORE_F32) {
 #pragma unroll 1
         for (int c = c32; c < c32 + NC32; ++c) {
           tmem_ld32(tacc + c * 32, v);
           tmem_wait_ld();
-          const int n = nt * BN + c * 32;
+          const int n = nt * BN + cb + c * 32;
           if (st_any && n < p.N) {
 #pragma unroll
             for (int i = 0; i < 32; ++i) f[i] = no_k ? 0.f : f32(v[i]);
@@ -697,8 +788,8 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
         for (int c = c32; c < c32 + NC32; ++c) {
           tmem_ld32(tacc + c * 32, v);
           tmem_wait_ld();
-          const int half = c >= BN / 64;
-          const int n = nt * (BN / 2) + (c % (BN / 64)) * 32;
+          const int half = c >= SEGW / 64;
+          const int n = nt * (BN / 2) + cb / 2 + (c % (SEGW / 64)) * 32;
           if (st_any && n < p.N) {
 #pragma unroll
             for (int i = 0; i < 32; ++i) f[i] = no_k ? 0.f : f32(v[i]);
@@ -707,14 +798,14 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
         }
       } else if constexpr (EPI == EPI_SWIGLU_FWD) {
         uint32_t w[32];
-        constexpr int NC64 = BN / 64 / NPART;
+        constexpr int NC64 = SEGW / 64 / NPART;
         const float gs = (p.gate && row_ok) ? __ldg(p.gate + grow) : 1.0f;
 #pragma unroll 1
         for (int c = part * NC64; c < (part + 1) * NC64; ++c) {
           tmem_ld32(tacc + c * 32, v);
-          tmem_ld32(tacc + BN / 2 + c * 32, w);
+          tmem_ld32(tacc + SEGW / 2 + c * 32, w);
           tmem_wait_ld();
-          const int n = nt * (BN / 2) + c * 32;
+          const int n = nt * (BN / 2) + cb / 2 + c * 32;
           if (st_any && n < p.N) {
             float g[32];
 #pragma unroll
@@ -847,10 +938,11 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
       tc_fence_before();
       __syncwarp();
       if (lane == 0) {
-        // the accumulator is free again: tell the CTA that issues the MMAs
+        // the segment is free again: tell the CTA that issues the MMAs
         if constexpr (PAIR) mbar_arrive_cluster(mapa_shared(smem_u32(&tempty[a]), 0));
         else mbar_arrive(&tempty[a]);
       }
+      }   // segments
     }
     // the TMA stores read the staging buffers until they complete
     if (STAGED && lane == 0) bulk_wait_all();
@@ -1078,14 +1170,26 @@ static Args row_args(int E, int M, int N, int K, int BN_tile, int* status, const
 }
 
 constexpr int kDuStages = 5;
+constexpr int kWideStages = 4;
+
+// Wide (256 x 512) pair tiles where the output columns fill them exactly and the K loop is
+// long enough (k rows) to cover the epilogue's hand-over of the two accumulator halves:
+// measured, they gain 2-5% with k >= 1024 (k >= 2048 behind the SwiGLU epilogue, which
+// writes three outputs; at 1024 it only breaks even) and lose about 3% at k = 512.
+// `tiles`: 0 chooses so, 1 keeps 256-column tiles, 2 takes wide tiles wherever they fit.
+static bool wide_cols(int tiles, int n, int k, int k_min = 1024) {
+  if (tiles == 1 || n % 512 != 0) return false;
+  return tiles == 2 || k >= k_min;
+}
 
 template <int BN, bool A_MN, bool B_MN, bool B_SPLIT, bool K_SPLIT, int EPI>
 static cudaError_t launch_rows(const CUtensorMap& a0, const CUtensorMap& a1, const CUtensorMap& b0,
                                const CUtensorMap& b1, const CUtensorMap& o0, const CUtensorMap& o1,
                                const CUtensorMap& o2, const Args& p, const VarRows* vr,
                                cudaStream_t st) {
-  // the dU GEMM's epilogue reads A and B through L1: a 5-deep ring leaves it 32 KB more
-  constexpr int ST = EPI == EPI_SWIGLU_BWD ? kDuStages : 6;
+  // the dU GEMM's epilogue reads A and B through L1: a 5-deep ring leaves it 32 KB more;
+  // wide tiles take 48 KB per k-slice
+  constexpr int ST = BN == 512 ? kWideStages : EPI == EPI_SWIGLU_BWD ? kDuStages : 6;
   if (vr)
     return launch<BN, A_MN, B_MN, B_SPLIT, K_SPLIT, EPI, ST, 8, true, 1>(a0, a1, b0, b1, o0, o1, o2,
                                                                           p, st);
@@ -1095,7 +1199,7 @@ static cudaError_t launch_rows(const CUtensorMap& a0, const CUtensorMap& a1, con
 
 cudaError_t tc_expert_up(const void* H, const void* Wg, const void* Wu, void* A, void* B, void* U,
                          int E, int M, int d, int F, int* status, cudaStream_t st,
-                         const VarRows* vr, const float* gate) {
+                         const VarRows* vr, const float* gate, int tiles) {
   CUtensorMap ma, mg, mu, oa, ob, ou;
   TC_TRY(act_map(&ma, H, d, E, M, vr, BM));
   TC_TRY(make_map(&mg, Wg, F, d, E, 64));
@@ -1103,27 +1207,35 @@ cudaError_t tc_expert_up(const void* H, const void* Wg, const void* Wu, void* A,
   TC_TRY(act_out_map(&oa, A, F, E, M, vr));
   TC_TRY(act_out_map(&ob, B, F, E, M, vr));
   TC_TRY(act_out_map(&ou, U, F, E, M, vr));
-  Args p = row_args(E, M, F, d, 128, status, vr);
+  const bool wide = wide_cols(tiles, 2 * F, d, 2048);   // gate and up columns side by side
+  Args p = row_args(E, M, F, d, wide ? 256 : 128, status, vr);
   p.out0 = A;
   p.out1 = B;
   p.out2 = U;
   p.gate = gate;
   p.ld = F;
   p.bstride = (int64_t)M * F;
+  if (wide)
+    return launch_rows<512, false, true, true, false, EPI_SWIGLU_FWD>(ma, ma, mg, mu, oa, ob, ou, p,
+                                                                      vr, st);
   return launch_rows<256, false, true, true, false, EPI_SWIGLU_FWD>(ma, ma, mg, mu, oa, ob, ou, p,
                                                                     vr, st);
 }
 
 cudaError_t tc_expert_down(const void* U, const void* Wd, void* O, int E, int M, int d, int F,
-                           int* status, cudaStream_t st, const VarRows* vr) {
+                           int* status, cudaStream_t st, const VarRows* vr, int tiles) {
   CUtensorMap ma, mb, mo;
   TC_TRY(act_map(&ma, U, F, E, M, vr, BM));
   TC_TRY(make_map(&mb, Wd, d, F, E, 64));
   TC_TRY(act_out_map(&mo, O, d, E, M, vr));
-  Args p = row_args(E, M, d, F, 256, status, vr);
+  const bool wide = wide_cols(tiles, d, F);
+  Args p = row_args(E, M, d, F, wide ? 512 : 256, status, vr);
   p.out0 = O;
   p.ld = d;
   p.bstride = (int64_t)M * d;
+  if (wide)
+    return launch_rows<512, false, true, false, false, EPI_STORE_BF16>(ma, ma, mb, mb, mo, mo, mo,
+                                                                       p, vr, st);
   return launch_rows<256, false, true, false, false, EPI_STORE_BF16>(ma, ma, mb, mb, mo, mo, mo, p,
                                                                      vr, st);
 }
@@ -1153,7 +1265,7 @@ cudaError_t tc_expert_dgrad_up(const void* dO, const void* Wd, const void* A, co
 
 cudaError_t tc_expert_dgrad_h(const void* dA, const void* dB, const void* Wg, const void* Wu,
                               void* dH, int E, int M, int d, int F, int* status, cudaStream_t st,
-                              const VarRows* vr) {
+                              const VarRows* vr, int tiles) {
   CUtensorMap ma0, ma1, mb0, mb1;
   TC_TRY(act_map(&ma0, dA, F, E, M, vr, BM));
   TC_TRY(act_map(&ma1, dB, F, E, M, vr, BM));
@@ -1161,20 +1273,27 @@ cudaError_t tc_expert_dgrad_h(const void* dA, const void* dB, const void* Wg, co
   TC_TRY(make_map(&mb1, Wu, F, d, E, 128));
   CUtensorMap mo;
   TC_TRY(act_out_map(&mo, dH, d, E, M, vr));
-  Args p = row_args(E, M, d, 2 * F, 256, status, vr);
+  const bool wide = wide_cols(tiles, d, 2 * F);
+  Args p = row_args(E, M, d, 2 * F, wide ? 512 : 256, status, vr);
   p.k_blocks0 = F / BK;
   p.out0 = dH;
   p.ld = d;
   p.bstride = (int64_t)M * d;
+  if (wide)
+    return launch_rows<512, false, false, false, true, EPI_STORE_BF16>(ma0, ma1, mb0, mb1, mo, mo,
+                                                                       mo, p, vr, st);
   return launch_rows<256, false, false, false, true, EPI_STORE_BF16>(ma0, ma1, mb0, mb1, mo, mo, mo,
                                                                      p, vr, st);
 }
 
 cudaError_t tc_expert_wgrad(const void* H, const void* U, const void* dO, const void* dA,
                             const void* dB, float* dWg, float* dWu, float* dWd, int E, int M,
-                            int d, int F, int* status, cudaStream_t st, const VarRows* vr) {
+                            int d, int F, int* status, cudaStream_t st, const VarRows* vr,
+                            int tiles) {
   // Variable rows: the K loop of expert e runs over its own padded region (count rows,
   // rounded up to the 64-row k-step, the rest of which is zero in both operands).
+  // K rows per expert (variable rows: on average)
+  const int rows = vr ? vr->P / (E > 0 ? E : 1) : M;
   auto wg_args = [&](int Mo, int No, int BNt) {
     Args p = base_args(E, Mo, No, vr ? vr->P : M, BNt, status);
     if (vr) {
@@ -1190,16 +1309,24 @@ cudaError_t tc_expert_wgrad(const void* H, const void* U, const void* dO, const 
     TC_TRY(act_map(&ma, U, F, E, M, vr, 64));
     TC_TRY(act_map(&mb, dO, d, E, M, vr, 64));
     TC_TRY(make_out_map(&mo, dWd, true, d, F, E));
-    Args p = wg_args(F, d, 256);
+    const bool wide = wide_cols(tiles, d, rows);
+    Args p = wg_args(F, d, wide ? 512 : 256);
     p.out0 = dWd;
     p.ld = d;
     p.bstride = (int64_t)F * d;
-    if (vr)
-      TC_TRY((launch<256, true, true, false, false, EPI_STORE_F32, 6, 8, true, 2>(ma, ma, mb, mb, mo, mo,
-                                                                                mo, p, st)));
+    constexpr int EP = EPI_STORE_F32, WS = kWideStages;
+    if (wide && vr)
+      TC_TRY((launch<512, true, true, false, false, EP, WS, 8, true, 2>(ma, ma, mb, mb, mo, mo, mo, p,
+                                                                      st)));
+    else if (wide)
+      TC_TRY((launch<512, true, true, false, false, EP, WS, 8, true>(ma, ma, mb, mb, mo, mo, mo, p,
+                                                                   st)));
+    else if (vr)
+      TC_TRY((launch<256, true, true, false, false, EP, 6, 8, true, 2>(ma, ma, mb, mb, mo, mo, mo, p,
+                                                                     st)));
     else
-      TC_TRY((launch<256, true, true, false, false, EPI_STORE_F32, 6, 8, true>(ma, ma, mb, mb, mo, mo, mo,
-                                                                             p, st)));
+      TC_TRY((launch<256, true, true, false, false, EP, 6, 8, true>(ma, ma, mb, mb, mo, mo, mo, p,
+                                                                  st)));
   }
   {
     // [dWg | dWu][e] [d][F] = H[e]^T . [dA | dB][e]
@@ -1209,17 +1336,25 @@ cudaError_t tc_expert_wgrad(const void* H, const void* U, const void* dO, const 
     TC_TRY(act_map(&mb1, dB, F, E, M, vr, 64));
     TC_TRY(make_out_map(&mo0, dWg, true, F, d, E));
     TC_TRY(make_out_map(&mo1, dWu, true, F, d, E));
-    Args p = wg_args(d, F, 128);
+    const bool wide = wide_cols(tiles, 2 * F, rows);
+    Args p = wg_args(d, F, wide ? 256 : 128);
     p.out0 = dWg;
     p.out1 = dWu;
     p.ld = F;
     p.bstride = (int64_t)d * F;
-    if (vr)
-      TC_TRY((launch<256, true, true, true, false, EPI_STORE_F32_SPLIT, 6, 8, true, 2>(
-          ma, ma, mb0, mb1, mo0, mo1, mo1, p, st)));
+    constexpr int EP = EPI_STORE_F32_SPLIT, WS = kWideStages;
+    if (wide && vr)
+      TC_TRY((launch<512, true, true, true, false, EP, WS, 8, true, 2>(ma, ma, mb0, mb1, mo0, mo1, mo1,
+                                                                     p, st)));
+    else if (wide)
+      TC_TRY((launch<512, true, true, true, false, EP, WS, 8, true>(ma, ma, mb0, mb1, mo0, mo1, mo1, p,
+                                                                  st)));
+    else if (vr)
+      TC_TRY((launch<256, true, true, true, false, EP, 6, 8, true, 2>(ma, ma, mb0, mb1, mo0, mo1, mo1,
+                                                                    p, st)));
     else
-      TC_TRY((launch<256, true, true, true, false, EPI_STORE_F32_SPLIT, 6, 8, true>(
-          ma, ma, mb0, mb1, mo0, mo1, mo1, p, st)));
+      TC_TRY((launch<256, true, true, true, false, EP, 6, 8, true>(ma, ma, mb0, mb1, mo0, mo1, mo1, p,
+                                                                 st)));
   }
   return cudaSuccess;
 }

@@ -19,6 +19,11 @@ struct VarRows {
   int P;
 };
 
+// Tile shapes of the expert GEMMs (the `tiles` argument below): 0 chooses per GEMM (256 x 512
+// pair tiles where the output columns fill them and the K loop is long enough to hide the
+// hand-over of their two accumulator halves, else 256 x 256), 1 always 256 x 256, 2 wide
+// tiles wherever the columns fill them. The dU GEMM always takes 256 x 256 tiles.
+
 // Router: Z = X.Wr (+br), S = row softmax over the E experts, written as S [N][E] and
 // S^T [E][N]. X [N][d] bf16, Wr [d][E] bf16. Wr_pad: device scratch of d*round_up(E,64)
 // bf16 (zero-padded copy of Wr made on the stream).
@@ -30,11 +35,13 @@ cudaError_t tc_router_softmax(const void* X, const void* Wr, void* Wr_pad, const
 // or, with vr, [P]; NULL: g = 1). H [E][M][d]; Wg, Wu [E][d][F]; A, B, U [E][M][F] bf16.
 cudaError_t tc_expert_up(const void* H, const void* Wg, const void* Wu, void* A, void* B, void* U,
                          int E, int M, int d, int F, int* status, cudaStream_t st,
-                         const VarRows* vr = nullptr, const float* gate = nullptr);
+                         const VarRows* vr = nullptr, const float* gate = nullptr,
+                         int tiles = 0);
 
 // O = U.Wd per expert. U [E][M][F]; Wd [E][F][d]; O [E][M][d] bf16.
 cudaError_t tc_expert_down(const void* U, const void* Wd, void* O, int E, int M, int d, int F,
-                           int* status, cudaStream_t st, const VarRows* vr = nullptr);
+                           int* status, cudaStream_t st, const VarRows* vr = nullptr,
+                           int tiles = 0);
 
 // dU' = dO.Wd^T per expert, dU = g dU' (g the row's gate as in tc_expert_up, NULL: 1), then
 // dA = dU * B * silu'(A), dB = dU * silu(A) (bf16 out). With dgate_part, also the row's
@@ -49,14 +56,14 @@ cudaError_t tc_expert_dgrad_up(const void* dO, const void* Wd, const void* A, co
 // dH = dA.Wg^T + dB.Wu^T per expert (one K loop over both halves). dH [E][M][d] bf16.
 cudaError_t tc_expert_dgrad_h(const void* dA, const void* dB, const void* Wg, const void* Wu,
                               void* dH, int E, int M, int d, int F, int* status, cudaStream_t st,
-                              const VarRows* vr = nullptr);
+                              const VarRows* vr = nullptr, int tiles = 0);
 
 // Weight gradients per expert, fp32: dWd = U^T.dO, dWg = H^T.dA, dWu = H^T.dB.
 // With `vr`, each expert sums over its own rows (an expert with none gets zeros).
 cudaError_t tc_expert_wgrad(const void* H, const void* U, const void* dO, const void* dA,
                             const void* dB, float* dWg, float* dWu, float* dWd, int E, int M,
                             int d, int F, int* status, cudaStream_t st,
-                            const VarRows* vr = nullptr);
+                            const VarRows* vr = nullptr, int tiles = 0);
 
 // Router backward on the tensor cores. dZb [2][N][Ep] bf16: hi and lo planes of the
 // zero-padded softmax gradient (dZ ~ hi + lo); Wr_pad [d][Ep] bf16 (the padded router

@@ -11,6 +11,7 @@ import math
 
 from . import (EC_BF16, EC_F32, ec_check_device, ec_ctx_create, ec_ctx_destroy,
                ec_ctx_profile, ec_ctx_set_capacity, ec_ctx_set_profiling, ec_ctx_set_residual,
+               ec_ctx_set_tiles,
                ec_ctx_set_shared, ec_ctx_set_workspace, ec_kernel_launches,
                ec_moe_backward, ec_moe_backward_shared, ec_moe_forward, ec_moe_forward_shared,
                ec_route, ec_rows_per_expert, ec_tc_backward, ec_tc_ctx_create, ec_tc_forward,
@@ -55,6 +56,10 @@ class ECMoELayer:
     def set_residual(self, on: bool):
         """Y = X + EC(X) and dX = dY + EC input gradient (stacked layers)."""
         ec_ctx_set_residual(self.ctx, on)
+
+    def set_tiles(self, policy: int):
+        """Expert-GEMM tile policy: EC_TILES_AUTO, EC_TILES_256 or EC_TILES_512."""
+        ec_ctx_set_tiles(self.ctx, policy)
 
     def _empty(self, *shape, dtype=None):
         return torch.empty(*shape, dtype=dtype or self.tdtype, device=self.device)

@@ -33,12 +33,15 @@ def tol(w: I.Workload) -> float:
     return 1e-4 if w.dtype == "f32" else 2e-2
 
 
-def gpu_layer(inp: I.Inputs, layer: int = 0, X=None, dY=None, backward=True):
-    """Run one layer on the GPU through the C ABI; returns (layer, outputs dict of tensors)."""
+def gpu_layer(inp: I.Inputs, layer: int = 0, X=None, dY=None, backward=True, tiles=None):
+    """Run one layer on the GPU through the C ABI; returns (layer, outputs dict of tensors).
+    `tiles`: an expert-GEMM tile policy (EC_TILES_*), else the library's choice."""
     from paper_2604_01622_gb300.layer import ECMoELayer
     w = inp.w
     L = inp.layers[layer]
     lay = ECMoELayer(w.N, w.d, w.E, w.d_ff, inp.group_off, inp.k_g, dtype=w.dtype)
+    if tiles is not None:
+        lay.set_tiles(tiles)
     Xd = dev(inp.X) if X is None else X
     br = None if L.br is None else torch.from_numpy(L.br).cuda()
     Y, idx, gate, S = lay.forward(Xd, dev(L.Wr), br, dev(L.Wg), dev(L.Wu), dev(L.Wd))

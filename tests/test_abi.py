@@ -76,6 +76,13 @@ def test_host_validation_without_device(lib):
         with pytest.raises(ec.ECError) as e:
             ec.ec_ctx_set_workspace(ctx, 0x1001, 1 << 40)
         assert e.value.status == ec.EC_ERR_WORKSPACE
+        # tile policies: the three named ones, nothing else
+        for policy in (ec.EC_TILES_256, ec.EC_TILES_512, ec.EC_TILES_AUTO):
+            ec.ec_ctx_set_tiles(ctx, policy)
+        for policy in (-1, 3):
+            with pytest.raises(ec.ECError) as e:
+                ec.ec_ctx_set_tiles(ctx, policy)
+            assert e.value.status == ec.EC_ERR_INVALID_ARG
     finally:
         ec.ec_ctx_destroy(ctx)
 

@@ -57,17 +57,22 @@ def _check(bufs):
             assert torch.isfinite(b.t.float()).all(), name
 
 
-@pytest.mark.parametrize("dtype", ["f32", "bf16"])
-def test_expert_choice_writes_stay_inside_buffers(dtype):
+# (dtype, d, d_ff, tile policy): fp32 SIMT path; bf16 with 256-column tiles (d = 192 leaves a
+# ragged column tile); bf16 with 256 x 512 tiles (d and 2 d_ff multiples of 512)
+EC_SHAPES = [("f32", 68, 36, 0), ("bf16", 192, 128, 1), ("bf16", 512, 256, 2)]
+
+
+@pytest.mark.parametrize("dtype,d,d_ff,tiles", EC_SHAPES, ids=["f32", "bf16", "bf16_wide"])
+def test_expert_choice_writes_stay_inside_buffers(dtype, d, d_ff, tiles):
     from paper_2604_01622_gb300.layer import ECMoELayer
     base = I.WORKLOADS["tiny_f32"] if dtype == "f32" else I.WORKLOADS["ec_d2048_e64"]
-    w = I.scaled(base, G=3, L=200, d=192 if dtype == "bf16" else 68, E=12,
-                 d_ff=128 if dtype == "bf16" else 36, k_base=40, router_bias=True, layers=1)
+    w = I.scaled(base, G=3, L=200, d=d, E=12, d_ff=d_ff, k_base=40, router_bias=True, layers=1)
     inp = I.make_inputs(w)
     group_off = np.array([0, 137, 137 + 263, 600], np.int32)   # ragged, N = 600
     k_g = np.array([40, 0, 70], np.int32)
     L = inp.layers[0]
     lay = ECMoELayer(w.N, w.d, w.E, w.d_ff, group_off, k_g, dtype=dtype)
+    lay.set_tiles(tiles)
     ws = _guard_workspace(lay)
     dt = lay.tdtype
     M = lay.M
@@ -88,14 +93,16 @@ def test_expert_choice_writes_stay_inside_buffers(dtype):
     lay.close()
 
 
-def test_token_choice_writes_stay_inside_buffers():
+@pytest.mark.parametrize("d,d_ff,tiles", [(128, 192, 1), (512, 256, 2)], ids=["narrow", "wide"])
+def test_token_choice_writes_stay_inside_buffers(d, d_ff, tiles):
     from paper_2604_01622_gb300.layer import TCMoELayer
-    w = I.Workload("guard_tc", G=1, L=700, d=128, E=12, d_ff=192, k_base=0, dtype="bf16",
+    w = I.Workload("guard_tc", G=1, L=700, d=d, E=12, d_ff=d_ff, k_base=0, dtype="bf16",
                    seed=21, router_bias=True)
     inp = I.make_inputs(w)
     L = inp.layers[0]
     k, cap = 3, 150
     lay = TCMoELayer(w.N, w.d, w.E, w.d_ff, k, cap)
+    lay.set_tiles(tiles)
     ws = _guard_workspace(lay)
     out = {"Y": Guarded((w.N, w.d), torch.bfloat16), "choice": Guarded((w.N, k), torch.int32),
            "gate": Guarded((w.N, k), torch.float32), "kept": Guarded((w.N, k), torch.int32),

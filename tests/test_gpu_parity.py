@@ -25,9 +25,9 @@ def _oracle_full(inp, layer, idx):
     return fwd, bwd
 
 
-def _check_layer(inp, layer=0):
+def _check_layer(inp, layer=0, tiles=None):
     w = inp.w
-    lay, out = gpu_layer(inp, layer)
+    lay, out = gpu_layer(inp, layer, tiles=tiles)
     S_gpu = host(out["S"]).T                              # [N][E] fp32 values as float64
     idx_gpu = out["idx"].cpu().numpy()
     # selection: bit-exact on the GPU's own scores
@@ -164,6 +164,32 @@ def test_bf16_ragged_groups_and_capacity_edges():
     inp.group_off = np.array([0, 0, 150, 151, 333], np.int32)
     inp.k_g = np.array([0, 150, 1, 17], np.int32)
     _check_layer(inp)
+
+
+def _wide_case():
+    # d = 512 and 2 d_ff = 512: with EC_TILES_512 every GEMM but dU takes 256 x 512 tiles (two
+    # 256-column accumulator halves handed over separately); M = 3 * 70 = 210 rows leaves a
+    # ragged row tile, and the short K loops (4 k-slices in the down GEMM, 8 in the others)
+    # hold the half-1 MMAs at both ends of a tile at once
+    w = I.scaled(I.WORKLOADS["ec_d2048_e64"], G=3, L=256, d=512, E=6, d_ff=256, k_base=70,
+                 seed=17, router_bias=True, layers=1)
+    return I.make_inputs(w)
+
+
+def test_bf16_wide_tiles_match_oracle():
+    from paper_2604_01622_gb300 import EC_TILES_512
+    _check_layer(_wide_case(), tiles=EC_TILES_512)
+
+
+def test_bf16_tile_policies_agree_bit_for_bit():
+    """256 x 256 and 256 x 512 tiles issue the same N = 256 MMAs over K in the same order and
+    the same epilogue arithmetic per element, so every output is bit-identical."""
+    from paper_2604_01622_gb300 import EC_TILES_256, EC_TILES_512
+    inp = _wide_case()
+    _, a = gpu_layer(inp, tiles=EC_TILES_256)
+    _, b = gpu_layer(inp, tiles=EC_TILES_512)
+    for k in ("Y", "idx", "gate", "dX", "dWr", "dbr", "dWg", "dWu", "dWd"):
+        assert torch.equal(a[k], b[k]), k
 
 
 def test_bf16_few_tokens_minimum_widths():

@@ -21,13 +21,15 @@ BOUND = 2e-2
 GRADS = ("Y", "dX", "dWr", "dWg", "dWu", "dWd")
 
 
-def _run(inp, k, capacity, residual=False):
+def _run(inp, k, capacity, residual=False, tiles=None):
     from paper_2604_01622_gb300.layer import TCMoELayer
     w = inp.w
     L = inp.layers[0]
     lay = TCMoELayer(w.N, w.d, w.E, w.d_ff, k, capacity)
     if residual:
         lay.set_residual(True)
+    if tiles is not None:
+        lay.set_tiles(tiles)
     br = None if L.br is None else torch.from_numpy(L.br).cuda()
     Y, choice, gate, kept, load, S = lay.forward(dev(inp.X), dev(L.Wr), br, dev(L.Wg),
                                                  dev(L.Wu), dev(L.Wd))
@@ -68,7 +70,10 @@ CASES = [
     ("e100_k5", dict(L=384, E=100, d=64, d_ff=64), 5, None),
     # one expert: every token's single choice, normalised gate 1, no router gradient
     ("e1_k1", dict(E=1, L=300), 1, None),
+    # d and 2 d_ff multiples of 512, tile policy EC_TILES_512: the GEMMs take 256 x 512 tiles
+    ("wide_tiles", dict(L=300, d=512, d_ff=256, E=6, router_bias=True), 2, 1.0),
 ]
+TILES = {"wide_tiles": 2}
 
 
 def _workload(over):
@@ -84,7 +89,7 @@ def test_tc_layer_parity(name, over, k, cf):
     inp = I.make_inputs(w)
     L = inp.layers[0]
     cap = tc_capacity(cf, k, w.N, w.E)
-    lay, out = _run(inp, k, cap)
+    lay, out = _run(inp, k, cap, tiles=TILES.get(name))
     S_gpu, choice, kept = _check_selection(out, k, cap, w.E)
     Wr, Wg, Wu, Wd = L.Wr.f64(), L.Wg.f64(), L.Wu.f64(), L.Wd.f64()
     fwd = TC.tc_forward(inp.X.f64(), Wr, L.br, Wg, Wu, Wd, k, forced=(choice, kept))
