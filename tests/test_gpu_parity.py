@@ -181,6 +181,15 @@ def test_bf16_wide_tiles_match_oracle():
     _check_layer(_wide_case(), tiles=EC_TILES_512)
 
 
+def test_bf16_wide_tiles_single_k_slice():
+    """M = 40 rows per expert: the weight-gradient GEMMs' K loop is one 64-row slice, shorter
+    than the 3-slice tail whose half-1 MMAs wait for half 0, so every k-slice is held."""
+    from paper_2604_01622_gb300 import EC_TILES_512
+    w = I.scaled(I.WORKLOADS["ec_d2048_e64"], G=2, L=64, d=512, E=5, d_ff=256, k_base=20,
+                 seed=18, layers=1)
+    _check_layer(I.make_inputs(w), tiles=EC_TILES_512)
+
+
 def test_bf16_tile_policies_agree_bit_for_bit():
     """256 x 256 and 256 x 512 tiles issue the same N = 256 MMAs over K in the same order and
     the same epilogue arithmetic per element, so every output is bit-identical."""

@@ -110,10 +110,13 @@ def test_tc_layer_parity(name, over, k, cf):
     lay.close()
 
 
-def test_tc_capacity_zero_drops_everything():
-    w = _workload(dict())
+@pytest.mark.parametrize("wide", [False, True], ids=["narrow", "wide"])
+def test_tc_capacity_zero_drops_everything(wide):
+    """Capacity 0: no expert keeps a row, so every GEMM tile has an empty K loop or no rows
+    (with 256 x 512 tiles: both accumulator halves are still handed over per tile)."""
+    w = _workload(dict(d=512, d_ff=256) if wide else dict())
     inp = I.make_inputs(w)
-    lay, out = _run(inp, 2, 0)
+    lay, out = _run(inp, 2, 0, tiles=2 if wide else None)
     assert not out["kept"].any() and not out["load"].any()
     assert not out["Y"].any() and not out["dX"].any()
     for g in ("dWg", "dWu", "dWd", "dWr"):
