@@ -761,187 +761,187 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
       // The accumulator segments (one, or a wide tile's two halves, each released as soon
       // as it is drained): segment h holds tile columns [h*SEGW, (h+1)*SEGW).
       for (int h = 0; h < NH; ++h) {
-      const int a = WIDE ? h : (it & 1);
-      const uint32_t par = WIDE ? (uint32_t)(it & 1) : (uint32_t)((it >> 1) & 1);
-      if (!mbar_wait(&tfull[a], par, abort_flag, p.status)) { stop = true; break; }
-      tc_fence_after();
-      const uint32_t tacc = tmem_base + (uint32_t)(WIDE ? h * SEGW : a * BN) +
-                            ((uint32_t)(q * 32) << 16);
-      const int cb = h * SEGW;                   // first tile column of the segment
-      constexpr int NC32 = SEGW / 32 / NPART;    // 32-column chunks per warp
-      const int c32 = part * NC32;
-      if constexpr (EPI == EPI_STORE_BF16 || EPI == EPI_STORE_F32) {
+        const int a = WIDE ? h : (it & 1);
+        const uint32_t par = WIDE ? (uint32_t)(it & 1) : (uint32_t)((it >> 1) & 1);
+        if (!mbar_wait(&tfull[a], par, abort_flag, p.status)) { stop = true; break; }
+        tc_fence_after();
+        const uint32_t tacc = tmem_base + (uint32_t)(WIDE ? h * SEGW : a * BN) +
+                              ((uint32_t)(q * 32) << 16);
+        const int cb = h * SEGW;                   // first tile column of the segment
+        constexpr int NC32 = SEGW / 32 / NPART;    // 32-column chunks per warp
+        const int c32 = part * NC32;
+        if constexpr (EPI == EPI_STORE_BF16 || EPI == EPI_STORE_F32) {
 #pragma unroll 1
-        for (int c = c32; c < c32 + NC32; ++c) {
-          tmem_ld32(tacc + c * 32, v);
-          tmem_wait_ld();
-          const int n = nt * BN + cb + c * 32;
-          if (st_any && n < p.N) {
+          for (int c = c32; c < c32 + NC32; ++c) {
+            tmem_ld32(tacc + c * 32, v);
+            tmem_wait_ld();
+            const int n = nt * BN + cb + c * 32;
+            if (st_any && n < p.N) {
 #pragma unroll
-            for (int i = 0; i < 32; ++i) f[i] = no_k ? 0.f : f32(v[i]);
-            if constexpr (EPI == EPI_STORE_BF16) put_bf16(&mO0, n, f);
-            else put_f32(&mO0, n, f);
-          }
-        }
-      } else if constexpr (EPI == EPI_STORE_F32_SPLIT) {
-#pragma unroll 1
-        for (int c = c32; c < c32 + NC32; ++c) {
-          tmem_ld32(tacc + c * 32, v);
-          tmem_wait_ld();
-          const int half = c >= SEGW / 64;
-          const int n = nt * (BN / 2) + cb / 2 + (c % (SEGW / 64)) * 32;
-          if (st_any && n < p.N) {
-#pragma unroll
-            for (int i = 0; i < 32; ++i) f[i] = no_k ? 0.f : f32(v[i]);
-            put_f32(half ? &mO1 : &mO0, n, f);
-          }
-        }
-      } else if constexpr (EPI == EPI_SWIGLU_FWD) {
-        uint32_t w[32];
-        constexpr int NC64 = SEGW / 64 / NPART;
-        const float gs = (p.gate && row_ok) ? __ldg(p.gate + grow) : 1.0f;
-#pragma unroll 1
-        for (int c = part * NC64; c < (part + 1) * NC64; ++c) {
-          tmem_ld32(tacc + c * 32, v);
-          tmem_ld32(tacc + SEGW / 2 + c * 32, w);
-          tmem_wait_ld();
-          const int n = nt * (BN / 2) + cb / 2 + c * 32;
-          if (st_any && n < p.N) {
-            float g[32];
-#pragma unroll
-            for (int i = 0; i < 32; ++i) {
-              f[i] = no_k ? 0.f : f32(v[i]);
-              g[i] = no_k ? 0.f : f32(w[i]);
-            }
-            put2_bf16(&mO0, &mO1, n, f, g);
-            const uint64_t gs2 = f2(gs, gs);
-#pragma unroll
-            for (int i = 0; i < 32; i += 2) {   // U = gs * silu(A) * B, two columns at a time
-              const uint64_t a2 = f2(f[i], f[i + 1]);
-              const uint64_t u2 =
-                  f2_mul(gs2, f2_mul(f2_mul(a2, f2_sigmoid(a2)), f2(g[i], g[i + 1])));
-              f2_split(u2, f[i], f[i + 1]);
-            }
-            put_bf16(&mO2, n, f);
-          }
-        }
-      } else if constexpr (EPI == EPI_SWIGLU_BWD) {
-        // A and B of the next chunk are requested before the current one is computed (not
-        // with variable rows, whose tile decode leaves too few registers for the second set)
-        constexpr bool PREFETCH = VARM != 1;
-        const bf16* pa = reinterpret_cast<const bf16*>(p.in0) + row_off + nt * BN;
-        const bf16* pb = reinterpret_cast<const bf16*>(p.in1) + row_off + nt * BN;
-        uint4 ra[4], rb[4], na[4], nb[4];
-#pragma unroll
-        for (int i = 0; i < 4; ++i) ra[i] = rb[i] = na[i] = nb[i] = make_uint4(0, 0, 0, 0);
-        auto fetch = [&](int c, uint4* xa, uint4* xb) {
-          const int n = nt * BN + c * 32;
-          if (row_ok && n < p.N) {
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-              xa[i] = __ldg(reinterpret_cast<const uint4*>(pa + c * 32) + i);
-              xb[i] = __ldg(reinterpret_cast<const uint4*>(pb + c * 32) + i);
+              for (int i = 0; i < 32; ++i) f[i] = no_k ? 0.f : f32(v[i]);
+              if constexpr (EPI == EPI_STORE_BF16) put_bf16(&mO0, n, f);
+              else put_f32(&mO0, n, f);
             }
           }
-        };
-        if (PREFETCH) fetch(c32, ra, rb);
-        const float gs = (p.gate && row_ok) ? __ldg(p.gate + grow) : 1.0f;
-        // <acc, silu(A) * B> over this warp's columns of the row: even and odd columns
-        uint64_t dot2 = f2(0.f, 0.f);
+        } else if constexpr (EPI == EPI_STORE_F32_SPLIT) {
 #pragma unroll 1
-        for (int c = c32; c < c32 + NC32; ++c) {
-          if (!PREFETCH) fetch(c, ra, rb);
-          else if (c + 1 < c32 + NC32) fetch(c + 1, na, nb);
-          tmem_ld32(tacc + c * 32, v);
-          tmem_wait_ld();
-          const int n = nt * BN + c * 32;
-          if (st_any && n < p.N) {
-            float av[32], bv[32];   // av ends up holding dB
-            if (no_k) {
+          for (int c = c32; c < c32 + NC32; ++c) {
+            tmem_ld32(tacc + c * 32, v);
+            tmem_wait_ld();
+            const int half = c >= SEGW / 64;
+            const int n = nt * (BN / 2) + cb / 2 + (c % (SEGW / 64)) * 32;
+            if (st_any && n < p.N) {
 #pragma unroll
-              for (int i = 0; i < 32; ++i) f[i] = av[i] = 0.f;
-            } else {
+              for (int i = 0; i < 32; ++i) f[i] = no_k ? 0.f : f32(v[i]);
+              put_f32(half ? &mO1 : &mO0, n, f);
+            }
+          }
+        } else if constexpr (EPI == EPI_SWIGLU_FWD) {
+          uint32_t w[32];
+          constexpr int NC64 = SEGW / 64 / NPART;
+          const float gs = (p.gate && row_ok) ? __ldg(p.gate + grow) : 1.0f;
+#pragma unroll 1
+          for (int c = part * NC64; c < (part + 1) * NC64; ++c) {
+            tmem_ld32(tacc + c * 32, v);
+            tmem_ld32(tacc + SEGW / 2 + c * 32, w);
+            tmem_wait_ld();
+            const int n = nt * (BN / 2) + cb / 2 + c * 32;
+            if (st_any && n < p.N) {
+              float g[32];
+#pragma unroll
+              for (int i = 0; i < 32; ++i) {
+                f[i] = no_k ? 0.f : f32(v[i]);
+                g[i] = no_k ? 0.f : f32(w[i]);
+              }
+              put2_bf16(&mO0, &mO1, n, f, g);
+              const uint64_t gs2 = f2(gs, gs);
+#pragma unroll
+              for (int i = 0; i < 32; i += 2) {   // U = gs * silu(A) * B, two columns at a time
+                const uint64_t a2 = f2(f[i], f[i + 1]);
+                const uint64_t u2 =
+                    f2_mul(gs2, f2_mul(f2_mul(a2, f2_sigmoid(a2)), f2(g[i], g[i + 1])));
+                f2_split(u2, f[i], f[i + 1]);
+              }
+              put_bf16(&mO2, n, f);
+            }
+          }
+        } else if constexpr (EPI == EPI_SWIGLU_BWD) {
+          // A and B of the next chunk are requested before the current one is computed (not
+          // with variable rows, whose tile decode leaves too few registers for the second set)
+          constexpr bool PREFETCH = VARM != 1;
+          const bf16* pa = reinterpret_cast<const bf16*>(p.in0) + row_off + nt * BN;
+          const bf16* pb = reinterpret_cast<const bf16*>(p.in1) + row_off + nt * BN;
+          uint4 ra[4], rb[4], na[4], nb[4];
+#pragma unroll
+          for (int i = 0; i < 4; ++i) ra[i] = rb[i] = na[i] = nb[i] = make_uint4(0, 0, 0, 0);
+          auto fetch = [&](int c, uint4* xa, uint4* xb) {
+            const int n = nt * BN + c * 32;
+            if (row_ok && n < p.N) {
 #pragma unroll
               for (int i = 0; i < 4; ++i) {
-                unpack16(ra[i], av + 8 * i, bf16());
-                unpack16(rb[i], bv + 8 * i, bf16());
-              }
-              // two columns at a time: dU = gs acc, sg = sigma(a), dA = dU b sg (1 + a (1 - sg)),
-              // dB = dU a sg, and the gate-gradient terms acc a sg b
-              const uint64_t gs2 = f2(gs, gs), one2 = f2(1.f, 1.f), mone2 = f2(-1.f, -1.f);
-#pragma unroll
-              for (int i = 0; i < 32; i += 2) {
-                const uint64_t a2 = f2(av[i], av[i + 1]);
-                const uint64_t b2 = f2(bv[i], bv[i + 1]);
-                const uint64_t c2 = f2(f32(v[i]), f32(v[i + 1]));
-                const uint64_t sg2 = f2_sigmoid(a2);
-                const uint64_t das2 = f2_mul(f2_mul(gs2, c2), sg2);
-                dot2 = f2_fma(c2, f2_mul(f2_mul(a2, sg2), b2), dot2);
-                const uint64_t q2 = f2_fma(a2, f2_fma(sg2, mone2, one2), one2);
-                f2_split(f2_mul(f2_mul(das2, b2), q2), f[i], f[i + 1]);
-                f2_split(f2_mul(das2, a2), av[i], av[i + 1]);
+                xa[i] = __ldg(reinterpret_cast<const uint4*>(pa + c * 32) + i);
+                xb[i] = __ldg(reinterpret_cast<const uint4*>(pb + c * 32) + i);
               }
             }
-            put2_bf16(&mO0, &mO1, n, f, av);
-          }
-          if (PREFETCH)
-#pragma unroll
-            for (int i = 0; i < 4; ++i) { ra[i] = na[i]; rb[i] = nb[i]; }
-        }
-        if (p.dgate_part && row_ok) {
-          float de, dd;
-          f2_split(dot2, de, dd);
-          p.dgate_part[(int64_t)(nt * NPART + part) * p.dgate_stride + grow] = de + dd;
-        }
-      } else if constexpr (EPI == EPI_ROUTER) {
-        const int E = p.n_valid;
-        float mx = -INFINITY;
+          };
+          if (PREFETCH) fetch(c32, ra, rb);
+          const float gs = (p.gate && row_ok) ? __ldg(p.gate + grow) : 1.0f;
+          // <acc, silu(A) * B> over this warp's columns of the row: even and odd columns
+          uint64_t dot2 = f2(0.f, 0.f);
 #pragma unroll 1
-        for (int c = 0; c < BN / 32; ++c) {
-          tmem_ld32(tacc + c * 32, v);
-          tmem_wait_ld();
+          for (int c = c32; c < c32 + NC32; ++c) {
+            if (!PREFETCH) fetch(c, ra, rb);
+            else if (c + 1 < c32 + NC32) fetch(c + 1, na, nb);
+            tmem_ld32(tacc + c * 32, v);
+            tmem_wait_ld();
+            const int n = nt * BN + c * 32;
+            if (st_any && n < p.N) {
+              float av[32], bv[32];   // av ends up holding dB
+              if (no_k) {
 #pragma unroll
-          for (int i = 0; i < 32; ++i) {
-            const int e = c * 32 + i;
-            if (e < E) mx = fmaxf(mx, f32(v[i]) + (p.bias ? p.bias[e] : 0.f));
+                for (int i = 0; i < 32; ++i) f[i] = av[i] = 0.f;
+              } else {
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                  unpack16(ra[i], av + 8 * i, bf16());
+                  unpack16(rb[i], bv + 8 * i, bf16());
+                }
+                // two columns at a time: dU = gs acc, sg = sigma(a), dA = dU b sg (1 + a (1 - sg)),
+                // dB = dU a sg, and the gate-gradient terms acc a sg b
+                const uint64_t gs2 = f2(gs, gs), one2 = f2(1.f, 1.f), mone2 = f2(-1.f, -1.f);
+#pragma unroll
+                for (int i = 0; i < 32; i += 2) {
+                  const uint64_t a2 = f2(av[i], av[i + 1]);
+                  const uint64_t b2 = f2(bv[i], bv[i + 1]);
+                  const uint64_t c2 = f2(f32(v[i]), f32(v[i + 1]));
+                  const uint64_t sg2 = f2_sigmoid(a2);
+                  const uint64_t das2 = f2_mul(f2_mul(gs2, c2), sg2);
+                  dot2 = f2_fma(c2, f2_mul(f2_mul(a2, sg2), b2), dot2);
+                  const uint64_t q2 = f2_fma(a2, f2_fma(sg2, mone2, one2), one2);
+                  f2_split(f2_mul(f2_mul(das2, b2), q2), f[i], f[i + 1]);
+                  f2_split(f2_mul(das2, a2), av[i], av[i + 1]);
+                }
+              }
+              put2_bf16(&mO0, &mO1, n, f, av);
+            }
+            if (PREFETCH)
+#pragma unroll
+              for (int i = 0; i < 4; ++i) { ra[i] = na[i]; rb[i] = nb[i]; }
           }
-        }
-        float sum = 0.f;
-#pragma unroll 1
-        for (int c = 0; c < BN / 32; ++c) {
-          tmem_ld32(tacc + c * 32, v);
-          tmem_wait_ld();
-#pragma unroll
-          for (int i = 0; i < 32; ++i) {
-            const int e = c * 32 + i;
-            if (e < E) sum += expf(f32(v[i]) + (p.bias ? p.bias[e] : 0.f) - mx);
+          if (p.dgate_part && row_ok) {
+            float de, dd;
+            f2_split(dot2, de, dd);
+            p.dgate_part[(int64_t)(nt * NPART + part) * p.dgate_stride + grow] = de + dd;
           }
-        }
-        const float inv = 1.0f / sum;
-        float* S = reinterpret_cast<float*>(p.out0);
-        float* ST = reinterpret_cast<float*>(p.out1);
+        } else if constexpr (EPI == EPI_ROUTER) {
+          const int E = p.n_valid;
+          float mx = -INFINITY;
 #pragma unroll 1
-        for (int c = 0; c < BN / 32; ++c) {
-          tmem_ld32(tacc + c * 32, v);
-          tmem_wait_ld();
+          for (int c = 0; c < BN / 32; ++c) {
+            tmem_ld32(tacc + c * 32, v);
+            tmem_wait_ld();
 #pragma unroll
-          for (int i = 0; i < 32; ++i) {
-            const int e = c * 32 + i;
-            if (e < E && row_ok) {
-              const float pr = expf(f32(v[i]) + (p.bias ? p.bias[e] : 0.f) - mx) * inv;
-              S[(int64_t)gm * E + e] = pr;
-              ST[(int64_t)e * p.M + gm] = pr;
+            for (int i = 0; i < 32; ++i) {
+              const int e = c * 32 + i;
+              if (e < E) mx = fmaxf(mx, f32(v[i]) + (p.bias ? p.bias[e] : 0.f));
+            }
+          }
+          float sum = 0.f;
+#pragma unroll 1
+          for (int c = 0; c < BN / 32; ++c) {
+            tmem_ld32(tacc + c * 32, v);
+            tmem_wait_ld();
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+              const int e = c * 32 + i;
+              if (e < E) sum += expf(f32(v[i]) + (p.bias ? p.bias[e] : 0.f) - mx);
+            }
+          }
+          const float inv = 1.0f / sum;
+          float* S = reinterpret_cast<float*>(p.out0);
+          float* ST = reinterpret_cast<float*>(p.out1);
+#pragma unroll 1
+          for (int c = 0; c < BN / 32; ++c) {
+            tmem_ld32(tacc + c * 32, v);
+            tmem_wait_ld();
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+              const int e = c * 32 + i;
+              if (e < E && row_ok) {
+                const float pr = expf(f32(v[i]) + (p.bias ? p.bias[e] : 0.f) - mx) * inv;
+                S[(int64_t)gm * E + e] = pr;
+                ST[(int64_t)e * p.M + gm] = pr;
+              }
             }
           }
         }
-      }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) {
-        // the segment is free again: tell the CTA that issues the MMAs
-        if constexpr (PAIR) mbar_arrive_cluster(mapa_shared(smem_u32(&tempty[a]), 0));
-        else mbar_arrive(&tempty[a]);
-      }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) {
+          // the segment is free again: tell the CTA that issues the MMAs
+          if constexpr (PAIR) mbar_arrive_cluster(mapa_shared(smem_u32(&tempty[a]), 0));
+          else mbar_arrive(&tempty[a]);
+        }
       }   // segments
     }
     // the TMA stores read the staging buffers until they complete
