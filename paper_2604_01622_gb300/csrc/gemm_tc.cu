@@ -332,6 +332,20 @@ __device__ __forceinline__ void stage_bf16(uint8_t* buf, int r, const float* v) 
                    pack_bf16x2(v[8 * j + 4], v[8 * j + 5]),
                    pack_bf16x2(v[8 * j + 6], v[8 * j + 7]));
 }
+// The same layouts from words already in their output format: 16 words of two bf16 columns
+// each, or 32 fp32 words, in column order.
+__device__ __forceinline__ void stage_bf16w(uint8_t* buf, int r, const uint32_t* w) {
+#pragma unroll
+  for (int j = 0; j < 4; ++j)
+    *reinterpret_cast<uint4*>(buf + r * 64 + ((j ^ ((r >> 1) & 3)) << 4)) =
+        make_uint4(w[4 * j], w[4 * j + 1], w[4 * j + 2], w[4 * j + 3]);
+}
+__device__ __forceinline__ void stage_f32w(uint8_t* buf, int r, const uint32_t* w) {
+#pragma unroll
+  for (int j = 0; j < 8; ++j)
+    *reinterpret_cast<uint4*>(buf + r * 128 + ((j ^ (r & 7)) << 4)) =
+        make_uint4(w[4 * j], w[4 * j + 1], w[4 * j + 2], w[4 * j + 3]);
+}
 __device__ __forceinline__ void fence_async_smem() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
@@ -757,6 +771,36 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
         __syncwarp();
         if (lane == 0) tma_store_3d(m, smem_u32(b), n, srow, sbat);
       };
+      // the same from words in the output format (wide tiles, whose segments are read into
+      // registers before they are stored)
+      auto put_bf16w = [&](const CUtensorMap* m, int n, const uint32_t* w) {
+        if (lane == 0) bulk_wait_read<1>();
+        __syncwarp();
+        uint8_t* b = sStage + (warp - 2) * STAGE_BUF + slot * 2048;
+        stage_bf16w(b, lane, w);
+        fence_async_smem();
+        __syncwarp();
+        if (lane == 0) tma_store_3d(m, smem_u32(b), n, srow, sbat);
+        slot ^= 1;
+      };
+      auto put_f32w = [&](const CUtensorMap* m, int n, const uint32_t* w) {
+        if (lane == 0) bulk_wait_read<0>();
+        __syncwarp();
+        uint8_t* b = sStage + (warp - 2) * STAGE_BUF;
+        stage_f32w(b, lane, w);
+        fence_async_smem();
+        __syncwarp();
+        if (lane == 0) tma_store_3d(m, smem_u32(b), n, srow, sbat);
+      };
+      // hand accumulator segment a back to the MMA issuer (its TMEM loads have completed)
+      auto release = [&](int a) {
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) {
+          if constexpr (PAIR) mbar_arrive_cluster(mapa_shared(smem_u32(&tempty[a]), 0));
+          else mbar_arrive(&tempty[a]);
+        }
+      };
 
       // The accumulator segments (one, or a wide tile's two halves, each released as soon
       // as it is drained): segment h holds tile columns [h*SEGW, (h+1)*SEGW).
@@ -770,7 +814,88 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
         const int cb = h * SEGW;                   // first tile column of the segment
         constexpr int NC32 = SEGW / 32 / NPART;    // 32-column chunks per warp
         const int c32 = part * NC32;
-        if constexpr (EPI == EPI_STORE_BF16 || EPI == EPI_STORE_F32) {
+        if constexpr (WIDE) {
+          // The segment's values go to registers first (packed to bf16 where the output is
+          // bf16), the segment is handed back to the MMA issuer, and only then are the chunks
+          // staged and stored: the next tile's MMAs wait for the TMEM reads alone.
+          if constexpr (EPI == EPI_STORE_BF16) {
+            uint32_t pk[NC32][16];
+#pragma unroll
+            for (int i = 0; i < NC32; ++i) {
+              tmem_ld32(tacc + (c32 + i) * 32, v);
+              tmem_wait_ld();
+              if (i == NC32 - 1) release(a);   // the segment's last TMEM read has completed
+#pragma unroll
+              for (int j = 0; j < 16; ++j)
+                pk[i][j] = no_k ? 0u : pack_bf16x2(f32(v[2 * j]), f32(v[2 * j + 1]));
+            }
+#pragma unroll
+            for (int i = 0; i < NC32; ++i) {
+              const int n = nt * BN + cb + (c32 + i) * 32;
+              if (st_any && n < p.N) put_bf16w(&mO0, n, pk[i]);
+            }
+          } else if constexpr (EPI == EPI_STORE_F32 || EPI == EPI_STORE_F32_SPLIT) {
+            uint32_t raw[NC32][32];
+#pragma unroll
+            for (int i = 0; i < NC32; ++i) tmem_ld32(tacc + (c32 + i) * 32, raw[i]);
+            tmem_wait_ld();
+            release(a);
+#pragma unroll
+            for (int i = 0; i < NC32; ++i) {
+              const int c = c32 + i;
+              if (no_k) {
+#pragma unroll
+                for (int j = 0; j < 32; ++j) raw[i][j] = 0u;
+              }
+              if constexpr (EPI == EPI_STORE_F32) {
+                const int n = nt * BN + cb + c * 32;
+                if (st_any && n < p.N) put_f32w(&mO0, n, raw[i]);
+              } else {
+                const int half = c >= SEGW / 64;
+                const int n = nt * (BN / 2) + cb / 2 + (c % (SEGW / 64)) * 32;
+                if (st_any && n < p.N) put_f32w(half ? &mO1 : &mO0, n, raw[i]);
+              }
+            }
+          } else if constexpr (EPI == EPI_SWIGLU_FWD) {
+            // column pairs (gate chunk, up chunk): a pair's A, B, U are packed while the next
+            // pair's TMEM reads are in flight and stored once the segment is released
+            constexpr int NC64 = SEGW / 64 / NPART;
+            uint32_t pa[16], pb[16], pu[16];
+            const float gs = (p.gate && row_ok) ? __ldg(p.gate + grow) : 1.0f;
+            const uint64_t gs2 = f2(gs, gs);
+            auto store_pair = [&](int c) {
+              const int n = nt * (BN / 2) + cb / 2 + c * 32;
+              if (st_any && n < p.N) {
+                put_bf16w(&mO0, n, pa);
+                put_bf16w(&mO1, n, pb);
+                put_bf16w(&mO2, n, pu);
+              }
+            };
+#pragma unroll
+            for (int i = 0; i < NC64; ++i) {
+              uint32_t w[32];
+              const int c = part * NC64 + i;
+              tmem_ld32(tacc + c * 32, v);
+              tmem_ld32(tacc + SEGW / 2 + c * 32, w);
+              tmem_wait_ld();
+              if (i == NC64 - 1) release(a);   // the segment's last TMEM read has completed
+              if (i > 0) store_pair(c - 1);
+#pragma unroll
+              for (int j = 0; j < 32; j += 2) {   // U = gs * silu(A) * B, two columns at a time
+                const float a0 = no_k ? 0.f : f32(v[j]), a1 = no_k ? 0.f : f32(v[j + 1]);
+                const float b0 = no_k ? 0.f : f32(w[j]), b1 = no_k ? 0.f : f32(w[j + 1]);
+                const uint64_t a2 = f2(a0, a1);
+                const uint64_t u2 = f2_mul(gs2, f2_mul(f2_mul(a2, f2_sigmoid(a2)), f2(b0, b1)));
+                float u0, u1;
+                f2_split(u2, u0, u1);
+                pa[j / 2] = pack_bf16x2(a0, a1);
+                pb[j / 2] = pack_bf16x2(b0, b1);
+                pu[j / 2] = pack_bf16x2(u0, u1);
+              }
+            }
+            store_pair(part * NC64 + NC64 - 1);
+          }
+        } else if constexpr (EPI == EPI_STORE_BF16 || EPI == EPI_STORE_F32) {
 #pragma unroll 1
           for (int c = c32; c < c32 + NC32; ++c) {
             tmem_ld32(tacc + c * 32, v);
@@ -935,13 +1060,8 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
             }
           }
         }
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) {
-          // the segment is free again: tell the CTA that issues the MMAs
-          if constexpr (PAIR) mbar_arrive_cluster(mapa_shared(smem_u32(&tempty[a]), 0));
-          else mbar_arrive(&tempty[a]);
-        }
+        // the accumulator is free again: tell the CTA that issues the MMAs
+        if constexpr (!WIDE) release(a);
       }   // segments
     }
     // the TMA stores read the staging buffers until they complete
