@@ -565,6 +565,7 @@ def run_reference(args):
            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
            "config": {"workload": w.name, "sequences": w.G, "seq_len": w.L, "tokens": w.N,
                       "d_model": w.d, "experts": w.E, "d_ff": w.d_ff, "k_per_seq": w.k_base,
+                      "layers": w.layers, "shared_experts": args.shared_experts,
                       "parallelism": "host cores",
                       **({"routing": "token_choice", "k": args.tc_k,
                           "capacity_factor": args.tc_cf} if tc else {})},
