@@ -140,33 +140,46 @@ class Clocks:
 class OracleSample:
     """A bounded sample of the workload for the float64 oracle (as it stands): whole
     sequences of the workload when `tokens` >= its sequence length, else one shorter
-    sequence with the capacity scaled to keep the workload's capacity factor."""
+    sequence with the capacity scaled to keep the workload's capacity factor. Shared
+    experts are included when configured; for a stack of layers one layer is timed and the
+    rate divided by the number of layers (the layers have equal shapes)."""
 
-    def __init__(self, tokens: int, w):
+    def __init__(self, tokens: int, w, shared_experts: int = 0, shared_dff: int = 0):
         from paper_2604_01622_gb300 import inputs as I
         if tokens >= w.L:
             G, L, k = max(1, tokens // w.L), w.L, w.k_base
         else:
             G, L, k = 1, tokens, max(1, w.k_base * tokens // w.L)
         self.tokens = G * L
+        self.layers = w.layers
         ws = I.scaled(w, G=G, L=L, k_base=k, timestep_capacity=False, layers=1)
         inp = I.make_inputs(ws)
         Ld = inp.layers[0]
         self.args = (inp.X.f64(), Ld.Wr.f64(), Ld.br, Ld.Wg.f64(), Ld.Wu.f64(), Ld.Wd.f64(),
                      inp.group_off, inp.k_g)
         self.dY = inp.dY.f64()
+        self.shared = None
+        if shared_experts:
+            sh = I.make_shared(ws, 0, shared_experts, shared_dff)
+            g, u, dn, f = sh.Wg.f64(), sh.Wu.f64(), sh.Wd.f64(), shared_dff
+            self.shared = [(g[:, i * f:(i + 1) * f], u[:, i * f:(i + 1) * f],
+                            dn[i * f:(i + 1) * f, :]) for i in range(shared_experts)]
         self.desc = (f"{G} sequence(s) x {L} tokens of the workload (k_g={k}, capacity factor "
-                     f"{w.E * k / L:g}, E={w.E}, d={w.d}, d_ff={w.d_ff}), oracle fwd+bwd")
+                     f"{w.E * k / L:g}, E={w.E}, d={w.d}, d_ff={w.d_ff}"
+                     + (f", {shared_experts} shared experts of d_ff {shared_dff}"
+                        if shared_experts else "")
+                     + (f"; one of the {w.layers} layers timed" if w.layers > 1 else "")
+                     + "), oracle fwd+bwd")
 
     def run(self):
-        """Returns (tokens/s, seconds)."""
+        """Returns (tokens/s through the whole stack, seconds of the timed layer)."""
         from oracle import ecmoe as O
         X, Wr, br, Wg, Wu, Wd, goff, kg = self.args
         t0 = time.perf_counter()
-        f = O.forward(X, Wr, br, Wg, Wu, Wd, goff, kg)
+        f = O.forward(X, Wr, br, Wg, Wu, Wd, goff, kg, shared=self.shared)
         O.backward(f, self.dY, Wr, Wg, Wu, Wd)
         dt = time.perf_counter() - t0
-        return self.tokens / dt, dt
+        return self.tokens / dt / self.layers, dt
 
 
 class TCOracleSample:
@@ -530,7 +543,7 @@ def run_ours(args):
     out["clocks"] = clk
     if rank == 0 and not args.no_cpu_baseline:
         smp = (TCOracleSample(args.tc_cpu_tokens, w, args.tc_k, args.tc_cf) if tc
-               else OracleSample(args.cpu_tokens, w))
+               else OracleSample(args.cpu_tokens, w, args.shared_experts, args.shared_dff))
         v, dt = smp.run()
         out["cpu_baseline"] = {"value": round(v, 2), "unit": UNIT, "cores": _cores(),
                                "kind": "oracle", "sample": smp.desc, "seconds": round(dt, 2)}
@@ -550,13 +563,14 @@ def run_reference(args):
     w = I.WORKLOADS[args.workload]
     tc = args.routing == "tc"
     smp = (TCOracleSample(args.tc_cpu_tokens, w, args.tc_k, args.tc_cf) if tc
-           else OracleSample(args.ref_tokens, w))
+           else OracleSample(args.ref_tokens, w, args.shared_experts, args.shared_dff))
     for _ in range(args.warmup):
         smp.run()
     total_t = 0.0
     for _ in range(args.steps):
         total_t += smp.run()[1]
     desc = smp.desc
+    total_t *= getattr(smp, "layers", 1)   # one of the stack's equal layers was timed
     v = args.steps * smp.tokens / total_t
     out = {"impl": "reference", "metric": METRIC_TC if tc else METRIC, "value": round(v, 2),
            "unit": UNIT,
