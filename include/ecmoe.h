@@ -89,9 +89,9 @@ ec_status ec_ctx_set_residual(ec_ctx* ctx, int32_t on);
  * output columns are a multiple of 512 and the GEMM's K loop is long enough (1024, or 2048
  * behind the gate/up epilogue) to hide the hand-over of their accumulator halves, else
  * 256 x 256. EC_TILES_256 always takes 256 x 256; EC_TILES_512 takes 256 x 512 wherever the
- * columns fill it. All three give results within the same bounds (the sums over K run in
- * the same order; only the tiling of the output differs). Returns EC_ERR_INVALID_ARG for
- * any other value. */
+ * columns fill it. All three give bit-identical results (the same N = 256 MMAs run over K
+ * in the same order, with the same epilogue arithmetic; only the tiling of the output
+ * differs). Returns EC_ERR_INVALID_ARG for any other value. */
 enum { EC_TILES_AUTO = 0, EC_TILES_256 = 1, EC_TILES_512 = 2 };
 ec_status ec_ctx_set_tiles(ec_ctx* ctx, int32_t policy);
 
