@@ -109,6 +109,14 @@ def test_f32_ragged_groups_and_capacity_edges(seed):
     _check_layer(inp)
 
 
+def test_f32_many_experts():
+    """500 experts (the fp32 path takes up to 512): the router softmax and the per-expert
+    selection over many columns, 96 tokens, 5 per expert."""
+    w = I.scaled(I.WORKLOADS["tiny_f32"], G=1, L=96, d=32, E=500, d_ff=16, k_base=5, seed=20,
+                 router_bias=True)
+    _check_layer(I.make_inputs(w))
+
+
 # ------------------------------------------------------------------ bf16 path (2e-2), small shapes
 SMALL_BF16 = {
     # d2048/e64-like: ragged M (2*80 = 160 rows: one full 128-row tile and a 32-row tail)
@@ -199,6 +207,15 @@ def test_bf16_tile_policies_agree_bit_for_bit():
     _, b = gpu_layer(inp, tiles=EC_TILES_512)
     for k in ("Y", "idx", "gate", "dX", "dWr", "dbr", "dWg", "dWu", "dWd"):
         assert torch.equal(a[k], b[k]), k
+
+
+@pytest.mark.parametrize("E", [160, 256])
+def test_bf16_many_experts_router_widths(E):
+    """160 and 256 experts take the router GEMM's 192- and 256-column tiles (softmax over
+    the valid columns of a zero-padded score tile); 256 is the largest expert count."""
+    w = I.scaled(I.WORKLOADS["ec_many_small_e128"], G=2, L=256, d=128, E=E, d_ff=64, k_base=8,
+                 seed=19, router_bias=True, layers=1)
+    _check_layer(I.make_inputs(w))
 
 
 def test_bf16_few_tokens_minimum_widths():

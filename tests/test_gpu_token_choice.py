@@ -70,6 +70,8 @@ CASES = [
     ("e100_k5", dict(L=384, E=100, d=64, d_ff=64), 5, None),
     # one expert: every token's single choice, normalised gate 1, no router gradient
     ("e1_k1", dict(E=1, L=300), 1, None),
+    # the largest routing: 256 experts, each token's 32 best (router tile of 256 columns)
+    ("e256_k32", dict(L=256, E=256, d=64, d_ff=64), 32, None),
     # d and 2 d_ff multiples of 512, tile policy EC_TILES_512: the GEMMs take 256 x 512 tiles
     ("wide_tiles", dict(L=300, d=512, d_ff=256, E=6, router_bias=True), 2, 1.0),
 ]
