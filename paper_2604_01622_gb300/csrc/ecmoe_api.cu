@@ -40,7 +40,7 @@ struct ec_ctx {
   // state saved by the forward pass
   bool residual = false;   // Y = X + EC(X), dX = dY + EC input gradient
   int Fs = 0;              // shared experts: total hidden width (0 = none)
-  size_t o_Ash = 0, o_Bsh = 0, o_Ush = 0, o_Osh = 0, o_dAsh = 0, o_dBsh = 0;
+  size_t o_Ash = 0, o_Bsh = 0, o_Ush = 0, o_Osh = 0, o_dAsh = 0, o_dBsh = 0, o_shpart = 0;
   const void *Wgs = nullptr, *Wus = nullptr, *Wds = nullptr;
   float *dWgs = nullptr, *dWus = nullptr, *dWds = nullptr;
   bool have_fwd = false;
@@ -116,6 +116,18 @@ size_t esize(const ec_ctx* c) { return c->dtype == EC_BF16 ? 2 : 4; }
 
 bool use_tc(const ec_ctx* c) { return c->dtype == EC_BF16; }
 
+// SM pairs of the current device (the tensor-core GEMMs run one 2-CTA cluster per pair)
+int sm_pairs(const ec_ctx*) {
+  static int pairs = 0;
+  if (!pairs) {
+    int dev = 0, n = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    pairs = n > 1 ? n / 2 : 1;
+  }
+  return pairs;
+}
+
 void layout(ec_ctx* c) {
   const size_t N = c->N, d = c->d, E = c->E, F = c->F, M = c->M_cap, G = c->G, es = esize(c);
   // expert rows: E x M for expert choice; token choice keeps each expert's rows in a region
@@ -164,6 +176,8 @@ void layout(ec_ctx* c) {
   c->o_Osh = take(Fs ? N * d * es : 0);
   c->o_dAsh = take(N * Fs * es);
   c->o_dBsh = take(N * Fs * es);
+  // the shared FFN's dWd as two split-K halves (tensor cores; see ffn_backward)
+  c->o_shpart = take(use_tc(c) && Fs ? 2 * Fs * d * 4 : 0);
   // fp32 scratch: SIMT GEMM outputs (fp32 path) and router logits / router dX part
   const size_t big = std::max(std::max(P * F, P * d), std::max(N * Fs, Fs ? N * d : 0));
   const size_t f32n = use_tc(c) ? N * E : std::max(big, N * E);
@@ -343,11 +357,16 @@ ec_status ffn_forward(ec_ctx* c, const FfnNames& nm, const T* H, const void* Wg,
 // On the tensor-core path with `gate`, dO holds the ungated rows dY[idx] and U the gated
 // ones (as ffn_forward wrote them): dU = gate * dO.Wd^T, dWd = U^T.dO, and the gate
 // gradients <dO.Wd^T, silu(A) B> land in dgate_part (c->dg_parts partials, stride E*M).
+// dwd_split: optional scratch of 2*F*d floats for the single-FFN case (E = 1, the shared
+// experts), whose dWd = U^T.dO has few output tiles for the whole GPU and a K loop over all
+// M rows: the rows are split into two halves computed as two batch entries at once and
+// summed in order afterwards.
 template <typename T>
 ec_status ffn_backward(ec_ctx* c, const FfnNames& nm, const T* dO, const T* H, const T* A,
                        const T* B, const T* U, const void* Wg, const void* Wu, const void* Wd,
                        T* dA, T* dB, T* dH, float* dWg, float* dWu, float* dWd, int E, int M, int F,
-                       cudaStream_t st, const float* gate = nullptr, float* dgate_part = nullptr) {
+                       cudaStream_t st, const float* gate = nullptr, float* dgate_part = nullptr,
+                       float* dwd_split = nullptr) {
   const int d = c->d;
   const int64_t P = (int64_t)E * M;
   if (P == 0) {
@@ -363,9 +382,21 @@ ec_status ffn_backward(ec_ctx* c, const FfnNames& nm, const T* dO, const T* H, c
                                  dgate_part, P));
     EC_KERNEL(nm.dgrad_h, 1,
               tc_expert_dgrad_h(dA, dB, Wg, Wu, dH, E, M, d, F, status, st, nullptr, c->tiles));
-    EC_KERNEL(nm.wgrad, 2,
-              tc_expert_wgrad(H, U, dO, dA, dB, dWg, dWu, dWd, E, M, d, F, status, st, nullptr,
-                              c->tiles));
+    if (dwd_split && E == 1 && M % 2 == 0 && M >= 2048 &&
+        2 * ((F + 255) / 256) * ((d + 511) / 512) <= sm_pairs(c)) {
+      EC_KERNEL(nm.wgrad, 1,
+                tc_expert_wgrad(H, U, dO, dA, dB, dWg, dWu, nullptr, 1, M, d, F, status, st,
+                                nullptr, c->tiles));
+      EC_KERNEL(nm.wgrad, 1,
+                tc_expert_wgrad(H, U, dO, nullptr, nullptr, nullptr, nullptr, dwd_split, 2, M / 2,
+                                d, F, status, st, nullptr, c->tiles));
+      EC_KERNEL(nm.wgrad, 1,
+                launch_reduce_splits(dwd_split, dWd, (int64_t)F * d, 2, st));
+    } else {
+      EC_KERNEL(nm.wgrad, 2,
+                tc_expert_wgrad(H, U, dO, dA, dB, dWg, dWu, dWd, E, M, d, F, status, st, nullptr,
+                                c->tiles));
+    }
   } else {
     float* dU32 = at<float>(c, c->o_f32a);
     float* dH32 = at<float>(c, c->o_f32b);
@@ -478,7 +509,8 @@ ec_status run_backward(ec_ctx* c, const void* dY, void* dX, float* dWr, float* d
     EC_TRY(ffn_backward<T>(c, kShared, dYt, static_cast<const T*>(c->X), at<T>(c, c->o_Ash),
                            at<T>(c, c->o_Bsh), at<T>(c, c->o_Ush), c->Wgs, c->Wus, c->Wds,
                            at<T>(c, c->o_dAsh), at<T>(c, c->o_dBsh), dh, dWgs, dWus, dWds, 1, N,
-                           Fs, st));
+                           Fs, st, nullptr, nullptr,
+                           use_tc(c) ? at<float>(c, c->o_shpart) : nullptr));
     dHsh = dh;
   }
   // router: dZ = S (dS - <dS,S>), dX = dZ Wr^T + sum dH, dWr = X^T dZ, dbr = sum dZ

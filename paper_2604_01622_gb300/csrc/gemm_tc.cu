@@ -1423,7 +1423,7 @@ cudaError_t tc_expert_wgrad(const void* H, const void* U, const void* dO, const 
     }
     return p;
   };
-  {
+  if (dWd) {
     // dWd[e] [F][d] = U[e]^T . dO[e]: A[m=f][k=t] = U[t][f] (MN-major), B[k=t][n=i] = dO[t][i]
     CUtensorMap ma, mb, mo;
     TC_TRY(act_map(&ma, U, F, E, M, vr, 64));
@@ -1448,7 +1448,7 @@ cudaError_t tc_expert_wgrad(const void* H, const void* U, const void* dO, const 
       TC_TRY((launch<256, true, true, false, false, EP, 6, 8, true>(ma, ma, mb, mb, mo, mo, mo, p,
                                                                   st)));
   }
-  {
+  if (dWg) {
     // [dWg | dWu][e] [d][F] = H[e]^T . [dA | dB][e]
     CUtensorMap ma, mb0, mb1, mo0, mo1;
     TC_TRY(act_map(&ma, H, d, E, M, vr, 64));

@@ -58,8 +58,9 @@ cudaError_t tc_expert_dgrad_h(const void* dA, const void* dB, const void* Wg, co
                               void* dH, int E, int M, int d, int F, int* status, cudaStream_t st,
                               const VarRows* vr = nullptr, int tiles = 0);
 
-// Weight gradients per expert, fp32: dWd = U^T.dO, dWg = H^T.dA, dWu = H^T.dB.
-// With `vr`, each expert sums over its own rows (an expert with none gets zeros).
+// Weight gradients per expert, fp32: dWd = U^T.dO, dWg = H^T.dA, dWu = H^T.dB (dWd NULL:
+// only dWg and dWu; dWg NULL: only dWd). With `vr`, each expert sums over its own rows (an
+// expert with none gets zeros).
 cudaError_t tc_expert_wgrad(const void* H, const void* U, const void* dO, const void* dA,
                             const void* dB, float* dWg, float* dWu, float* dWd, int E, int M,
                             int d, int F, int* status, cudaStream_t st,

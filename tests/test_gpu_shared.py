@@ -20,6 +20,9 @@ CASES = {
     "f32": (I.scaled(I.WORKLOADS["tiny_f32"], G=2, L=100, d=36, E=5, d_ff=20, k_base=9), 2, 12),
     "bf16": (I.scaled(I.WORKLOADS["ec_d2048_e64"], G=2, L=256, d=192, E=8, d_ff=128,
                       k_base=40), 2, 64),
+    # 2048 tokens: the shared FFN's dWd runs as two split-K halves summed afterwards
+    "bf16_split_k": (I.scaled(I.WORKLOADS["ec_d2048_e64"], G=2, L=1024, d=256, E=8, d_ff=128,
+                              k_base=64), 2, 128),
 }
 
 
