@@ -1018,6 +1018,57 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
             f2_split(dot2, de, dd);
             p.dgate_part[(int64_t)(nt * NPART + part) * p.dgate_stride + grow] = de + dd;
           }
+        } else if constexpr (EPI == EPI_ROUTER && BN <= 128) {
+          // up to 128 experts the row's logits stay in registers: one TMEM read, exp once,
+          // and the row of S written with 16-byte stores when E allows it
+          const int E = p.n_valid;
+          constexpr int NCH = BN / 32;
+          float ev[NCH][32];
+          float mx = -INFINITY;
+#pragma unroll
+          for (int c = 0; c < NCH; ++c) {
+            tmem_ld32(tacc + c * 32, v);
+            tmem_wait_ld();
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+              const int e = c * 32 + i;
+              ev[c][i] = e < E ? f32(v[i]) + (p.bias ? __ldg(p.bias + e) : 0.f) : -INFINITY;
+              mx = fmaxf(mx, ev[c][i]);
+            }
+          }
+          float sum = 0.f;
+#pragma unroll
+          for (int c = 0; c < NCH; ++c)
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+              ev[c][i] = c * 32 + i < E ? expf(ev[c][i] - mx) : 0.f;
+              sum += ev[c][i];
+            }
+          const float inv = 1.0f / sum;
+          float* S = reinterpret_cast<float*>(p.out0);
+          float* ST = reinterpret_cast<float*>(p.out1);
+          const bool vec = (E & 3) == 0;   // rows of S start on 16-byte boundaries
+#pragma unroll
+          for (int c = 0; c < NCH; ++c) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) ev[c][i] *= inv;
+            if (row_ok) {
+              float* srow = S + (int64_t)gm * E + c * 32;
+              if (vec && c * 32 + 32 <= E) {
+#pragma unroll
+                for (int j = 0; j < 8; ++j)
+                  reinterpret_cast<float4*>(srow)[j] =
+                      make_float4(ev[c][4 * j], ev[c][4 * j + 1], ev[c][4 * j + 2], ev[c][4 * j + 3]);
+              } else {
+#pragma unroll
+                for (int i = 0; i < 32; ++i)
+                  if (c * 32 + i < E) srow[i] = ev[c][i];
+              }
+#pragma unroll
+              for (int i = 0; i < 32; ++i)
+                if (c * 32 + i < E) ST[(int64_t)(c * 32 + i) * p.M + gm] = ev[c][i];
+            }
+          }
         } else if constexpr (EPI == EPI_ROUTER) {
           const int E = p.n_valid;
           float mx = -INFINITY;
