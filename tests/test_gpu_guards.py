@@ -121,3 +121,39 @@ def test_token_choice_writes_stay_inside_buffers(d, d_ff, tiles):
     _check({"workspace": ws, **out, **g})
     assert int(out["load"].t.max()) <= cap
     lay.close()
+
+
+def test_shared_experts_writes_stay_inside_buffers():
+    """Shared experts over 2048 tokens: their FFN buffers and the two split-K halves of their
+    dWd (summed afterwards) stay inside the workspace; the shared gradients inside theirs."""
+    from paper_2604_01622_gb300.layer import ECMoELayer
+    w = I.scaled(I.WORKLOADS["ec_d2048_e64"], G=2, L=1024, d=512, E=6, d_ff=256, k_base=96,
+                 router_bias=True, layers=1)
+    n_sh, f_sh = 2, 256
+    inp = I.make_inputs(w)
+    L = inp.layers[0]
+    sh = I.make_shared(w, 0, n_sh, f_sh)
+    lay = ECMoELayer(w.N, w.d, w.E, w.d_ff, inp.group_off, inp.k_g, dtype="bf16",
+                     d_ff_shared=n_sh * f_sh)
+    ws = _guard_workspace(lay)
+    M, Fs = lay.M, n_sh * f_sh
+    out = {"Y": Guarded((w.N, w.d), torch.bfloat16), "idx": Guarded((w.E, M), torch.int32),
+           "gate": Guarded((w.E, M), torch.float32), "S": Guarded((w.E, w.N), torch.float32)}
+    X, Wr, Wg, Wu, Wd = dev(inp.X), dev(L.Wr), dev(L.Wg), dev(L.Wu), dev(L.Wd)
+    Wgs, Wus, Wds = dev(sh.Wg), dev(sh.Wu), dev(sh.Wd)
+    br = torch.from_numpy(L.br).cuda()
+    s = torch.cuda.current_stream().cuda_stream
+    ec.ec_moe_forward_shared(lay.ctx, X.data_ptr(), Wr.data_ptr(), br.data_ptr(), Wg.data_ptr(),
+                             Wu.data_ptr(), Wd.data_ptr(), Wgs.data_ptr(), Wus.data_ptr(),
+                             Wds.data_ptr(), out["Y"].ptr, out["idx"].ptr, out["gate"].ptr,
+                             out["S"].ptr, s)
+    g = _grads(w, torch.bfloat16)
+    g.update({"dWg_s": Guarded((w.d, Fs), torch.float32), "dWu_s": Guarded((w.d, Fs), torch.float32),
+              "dWd_s": Guarded((Fs, w.d), torch.float32)})
+    dY = dev(inp.dY)
+    ec.ec_moe_backward_shared(lay.ctx, dY.data_ptr(), g["dX"].ptr, g["dWr"].ptr, g["dbr"].ptr,
+                              g["dWg"].ptr, g["dWu"].ptr, g["dWd"].ptr, g["dWg_s"].ptr,
+                              g["dWu_s"].ptr, g["dWd_s"].ptr, s)
+    lay.check()
+    _check({"workspace": ws, **out, **g})
+    lay.close()
