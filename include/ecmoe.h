@@ -84,14 +84,16 @@ ec_status ec_ctx_set_capacity(ec_ctx* ctx, const int32_t* k_g);
  * picks then get Y_t = X_t. Invalidates saved forward state. */
 ec_status ec_ctx_set_residual(ec_ctx* ctx, int32_t on);
 
-/* Tile shapes of the tensor-core expert GEMMs (bf16 path; the fp32 path ignores it).
- * EC_TILES_AUTO (default) picks per GEMM: 256 x 512 output tiles per SM pair where the
+/* Tile shapes of the tensor-core expert GEMMs (bf16 path; the fp32 path ignores it). An
+ * implementation choice with no counterpart in the paper (the expert FFNs of Sec. 2.2 are
+ * computed the same way under every policy). EC_TILES_AUTO (default) picks per GEMM: 256 x 512 output tiles per SM pair where the
  * output columns are a multiple of 512 and the GEMM's K loop is long enough (1024, or 2048
  * behind the gate/up epilogue) to hide the hand-over of their accumulator halves, else
  * 256 x 256. EC_TILES_256 always takes 256 x 256; EC_TILES_512 takes 256 x 512 wherever the
  * columns fill it. All three give bit-identical results (the same N = 256 MMAs run over K
  * in the same order, with the same epilogue arithmetic; only the tiling of the output
- * differs). Returns EC_ERR_INVALID_ARG for any other value. */
+ * differs). Takes effect from the next call on the context; returns EC_ERR_INVALID_ARG for
+ * any other value (the context keeps its policy). */
 enum { EC_TILES_AUTO = 0, EC_TILES_256 = 1, EC_TILES_512 = 2 };
 ec_status ec_ctx_set_tiles(ec_ctx* ctx, int32_t policy);
 
