@@ -40,7 +40,7 @@ UNIT = "tokens/s"
 # workload (dram__bytes_read.sum + dram__bytes_write.sum), keyed by the hash of the
 # kernel source it was taken on; a changed kernel reports null until re-captured.
 TILE_POLICY = {"auto": 0, "256": 1, "512": 2}   # EC_TILES_AUTO / EC_TILES_256 / EC_TILES_512
-TRAFFIC = {"7c367d5d470f": 2864281643}   # mean of the six expert-GEMM launches of one step
+TRAFFIC = {"155693575a18": 2864281643}   # mean of the six expert-GEMM launches of one step
 
 
 def _peaks():
@@ -490,7 +490,7 @@ def run_ours(args):
         "gather_dy": (N + P) * d * b,
         "softmax_bwd": 3 * N * E * 4,
         "dgate_reduce": (2 * math.ceil(w.d_ff / 256) + 1) * P * 4,
-        "dx_combine": P * d * b + N * d * 4 + N * d * b,
+        "dx_combine": P * d * b + 2 * N * d * b,   # dH rows; the router's dX part; dX
     }
     mem_bytes = {k: v for k, v in mem_bytes.items() if k in per}   # kernels this path launches
     mem_ms = sum(sum(per[k]) for k in mem_bytes) / args.steps

@@ -183,7 +183,7 @@ void layout(ec_ctx* c) {
   const size_t f32n = use_tc(c) ? N * E : std::max(big, N * E);
   c->o_f32a = take(f32n * 4);
   c->o_f32b = take((use_tc(c) ? 0 : big) * 4);
-  c->o_dXr = take(N * d * 4);
+  c->o_dXr = take(N * d * es);   // the router's part of dX, in the layer dtype
   c->o_colsum = take((size_t)colsum_scratch_floats((int)N, (int)E) * 4);
   // split-K partials of dWr = X^T dZ (tensor cores: equal token blocks, so N % splits == 0)
   if (use_tc(c)) {
@@ -514,7 +514,7 @@ ec_status run_backward(ec_ctx* c, const void* dY, void* dX, float* dWr, float* d
     dHsh = dh;
   }
   // router: dZ = S (dS - <dS,S>), dX = dZ Wr^T + sum dH, dWr = X^T dZ, dbr = sum dZ
-  float* dXr = at<float>(c, c->o_dXr);
+  T* dXr = at<T>(c, c->o_dXr);
   float* part = at<float>(c, c->o_part);
   const T* res = c->residual ? dYt : nullptr;
   if (use_tc(c)) {
@@ -535,7 +535,9 @@ ec_status run_backward(ec_ctx* c, const void* dY, void* dX, float* dWr, float* d
     EC_KERNEL("softmax_bwd", nz,
               launch_softmax_bwd(at<float>(c, c->o_S), slot, dgate, dZ, nullptr, N, E, E, M, st));
     EC_KERNEL("router_dgrad_gemm", nz,
-              launch_simt_gemm(sg(dZ, 0, E, 1, c->Wr, 0, 1, E, dXr, 0, d, N, d, E, 1), EType::F32,
+              launch_simt_gemm(sg(dZ, 0, E, 1, c->Wr, 0, 1, E, reinterpret_cast<float*>(dXr), 0, d,
+                                  N, d, E, 1),
+                               EType::F32,
                                et(c), st));
     EC_KERNEL("dx_combine", nz,
               launch_dx_combine<T>(dH, slot, dXr, res, dHsh, static_cast<T*>(dX), N, E, M, d, st));
@@ -635,7 +637,7 @@ ec_status run_tc_backward(ec_ctx* c, const void* dY, void* dX, float* dWr, float
                             0, d, F, status, st, &vr, c->tiles));
   float* dZ = at<float>(c, c->o_dZ);
   bf16* dZb = at<bf16>(c, c->o_dZb);
-  float* dXr = at<float>(c, c->o_dXr);
+  bf16* dXr = at<bf16>(c, c->o_dXr);
   float* part = at<float>(c, c->o_part);
   float* dgsum = at<float>(c, c->o_dgsum);
   EC_KERNEL("dgate_reduce", 1, launch_reduce_splits(row_dgate, dgsum, c->P_tc, c->dg_parts, st));

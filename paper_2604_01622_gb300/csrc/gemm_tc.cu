@@ -1530,7 +1530,7 @@ cudaError_t tc_expert_wgrad(const void* H, const void* U, const void* dO, const 
   return cudaSuccess;
 }
 
-cudaError_t tc_router_dgrad(const void* dZb, const void* Wr_pad, float* dXr, int N, int d, int Ep,
+cudaError_t tc_router_dgrad(const void* dZb, const void* Wr_pad, void* dXr, int N, int d, int Ep,
                             int* status, cudaStream_t st) {
   if (N == 0) return cudaSuccess;
   // dXr [N][d] = (dZ_hi + dZ_lo) [N][Ep] . Wr^T as one K loop over both planes;
@@ -1541,13 +1541,14 @@ cudaError_t tc_router_dgrad(const void* dZb, const void* Wr_pad, float* dXr, int
   TC_TRY(make_map(&ma1, hi + (size_t)N * Ep, Ep, N, 1, BM));
   TC_TRY(make_map(&mb, Wr_pad, Ep, d, 1, 256));
   CUtensorMap mo;
-  TC_TRY(make_out_map(&mo, dXr, true, d, N, 1));
+  TC_TRY(make_out_map(&mo, dXr, false, d, N, 1));
   Args p = base_args(1, N, d, 2 * Ep, 256, status);
   p.k_blocks0 = Ep / BK;
   p.out0 = dXr;
   p.ld = d;
   p.bstride = 0;
-  return launch<256, false, false, false, true, EPI_STORE_F32, 4>(ma0, ma1, mb, mb, mo, mo, mo, p, st);
+  return launch<256, false, false, false, true, EPI_STORE_BF16, 4>(ma0, ma1, mb, mb, mo, mo, mo, p,
+                                                                   st);
 }
 
 cudaError_t tc_router_wgrad(const void* X, const void* dZb, float* part, int N, int d, int Ep,

@@ -68,8 +68,8 @@ cudaError_t tc_expert_wgrad(const void* H, const void* U, const void* dO, const 
 
 // Router backward on the tensor cores. dZb [2][N][Ep] bf16: hi and lo planes of the
 // zero-padded softmax gradient (dZ ~ hi + lo); Wr_pad [d][Ep] bf16 (the padded router
-// weights of the forward pass). dXr [N][d] fp32 = dZ . Wr^T.
-cudaError_t tc_router_dgrad(const void* dZb, const void* Wr_pad, float* dXr, int N, int d, int Ep,
+// weights of the forward pass). dXr [N][d] bf16 = dZ . Wr^T (summed in fp32, rounded once).
+cudaError_t tc_router_dgrad(const void* dZb, const void* Wr_pad, void* dXr, int N, int d, int Ep,
                             int* status, cudaStream_t st);
 // part [2][splits][d][Ep] fp32: X^T . dZ_plane over `splits` equal blocks of tokens
 // (N % splits == 0); dWr is the sum of all 2*splits partials.

@@ -65,9 +65,10 @@ cudaError_t launch_softmax_bwd(const float* S, const int* slot, const float* dga
                                __nv_bfloat16* dZb, int N, int E, int Ep, int M, cudaStream_t st);
 cudaError_t launch_reduce_partials(const float* part, float* out, int rows, int cols, int ld,
                                    int splits, cudaStream_t st);
-// dX_t = dXr_t + R_t + R2_t (each if given) + sum of the token's dH rows.
+// dX_t = dXr_t + R_t + R2_t (each if given) + sum of the token's dH rows, summed in fp32;
+// dXr (the router's part of the input gradient) is in the layer's dtype.
 template <typename T>
-cudaError_t launch_dx_combine(const T* dH, const int* slot, const float* dXr, const T* R,
+cudaError_t launch_dx_combine(const T* dH, const int* slot, const T* dXr, const T* R,
                               const T* R2, T* dX, int N, int E, int M, int d, cudaStream_t st);
 // out[e] = sum over the N rows of Z [N][E]; scratch: colsum_scratch_floats(N, E) floats.
 // Two kernels.

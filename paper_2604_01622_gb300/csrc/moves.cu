@@ -312,7 +312,7 @@ cudaError_t launch_reduce_partials(const float* part, float* out, int rows, int 
 // ------------------------------------------------------------------ dX_t = dXr_t + sum dH rows
 template <typename T>
 __global__ void dx_combine_kernel(const T* __restrict__ dH, const int* __restrict__ slot,
-                                  const float* __restrict__ dXr, const T* __restrict__ R,
+                                  const T* __restrict__ dXr, const T* __restrict__ R,
                                   const T* __restrict__ R2, T* __restrict__ dX, int N, int E,
                                   int M, int d) {
   extern __shared__ int sh[];
@@ -333,12 +333,7 @@ __global__ void dx_combine_kernel(const T* __restrict__ dH, const int* __restric
     float acc0[VN], acc1[VN];
     auto init = [&](int v, float* acc) {
       if (dXr) {
-        const float4* r = reinterpret_cast<const float4*>(dXr + (size_t)t * d + (size_t)v * VN);
-#pragma unroll
-        for (int j = 0; j < VN / 4; ++j) {
-          const float4 q = r[j];
-          acc[4 * j] = q.x; acc[4 * j + 1] = q.y; acc[4 * j + 2] = q.z; acc[4 * j + 3] = q.w;
-        }
+        unpack16(__ldg(reinterpret_cast<const uint4*>(dXr + (size_t)t * d) + v), acc, T());
       } else {
 #pragma unroll
         for (int j = 0; j < VN; ++j) acc[j] = 0.f;
@@ -388,7 +383,7 @@ __global__ void dx_combine_kernel(const T* __restrict__ dH, const int* __restric
 }
 
 template <typename T>
-cudaError_t launch_dx_combine(const T* dH, const int* slot, const float* dXr, const T* R,
+cudaError_t launch_dx_combine(const T* dH, const int* slot, const T* dXr, const T* R,
                               const T* R2, T* dX, int N, int E, int M, int d, cudaStream_t st) {
   if (N == 0) return cudaSuccess;
   const size_t smem = (size_t)2 * E * sizeof(int);
@@ -532,7 +527,7 @@ cudaError_t launch_reduce_splits(const float* part, float* out, int64_t n, int s
                                          T*, int, int, int, int, cudaStream_t);                   \
   template cudaError_t launch_bwd_gather_scale<T>(const T*, const T*, const int*, const float*,   \
                                                   T*, float*, int64_t, int, cudaStream_t);        \
-  template cudaError_t launch_dx_combine<T>(const T*, const int*, const float*, const T*,         \
+  template cudaError_t launch_dx_combine<T>(const T*, const int*, const T*, const T*,             \
                                             const T*, T*, int, int, int, int, cudaStream_t);      \
   template cudaError_t launch_swiglu_fwd_ew<T>(const float*, const float*, T*, T*, T*, int64_t,   \
                                                cudaStream_t);                                     \
