@@ -26,7 +26,28 @@ FULL = ["ec_d2048_e64", "ec_timestep_d2048_e64", "ec_many_small_e128", "ec_wide_
 @pytest.mark.parametrize("name", FULL)
 def test_full_size_sampled_parity(name):
     w = I.scaled(I.WORKLOADS[name], layers=1)
-    inp = I.make_inputs(w)
+    _check_sampled(I.make_inputs(w))
+
+
+def test_large_batch_past_32_bit_offsets():
+    """8 sequences of 32768 tokens, 4096 per expert and sequence: 2.1 M expert rows, so the
+    gathered rows H and dY[idx] hold 4.4 G elements each, past 32-bit element offsets (and
+    about 55 GB are in use on the GPU). The bench workload's 32768 tokens are repeated in
+    every sequence; selection is per sequence, so each sequence picks the same positions,
+    and the samples include tokens of the last sequence (rows above 2^31 elements)."""
+    base = I.scaled(I.WORKLOADS["ec_d2048_e64"], layers=1)
+    inp0 = I.make_inputs(base)
+    G, L = 8, base.N
+    w = I.scaled(base, G=G, L=L, k_base=4096)
+    X = I.Tensor(np.tile(inp0.X.data, (G, 1)), inp0.X.dtype)
+    dY = I.Tensor(np.tile(inp0.dY.data, (G, 1)), inp0.dY.dtype)
+    inp = I.Inputs(w, X, dY, (np.arange(G + 1) * L).astype(np.int32),
+                   np.full(G, 4096, np.int32), inp0.layers)
+    _check_sampled(inp, extra_tokens=[w.N - 1, w.N - 4097, (G - 1) * L + 123])
+
+
+def _check_sampled(inp, extra_tokens=()):
+    w = inp.w
     L = inp.layers[0]
     lay, out = gpu_layer(inp)
     bound = tol(w)
@@ -42,7 +63,7 @@ def test_full_size_sampled_parity(name):
     rng = np.random.default_rng(2024)
     picked = np.zeros(w.N, bool)
     picked[idx.ravel()] = True
-    toks = list(rng.choice(np.nonzero(picked)[0], 24, replace=False))
+    toks = list(rng.choice(np.nonzero(picked)[0], 24, replace=False)) + list(extra_tokens)
     if (~picked).any():
         toks += list(rng.choice(np.nonzero(~picked)[0], min(4, int((~picked).sum())), replace=False))
     toks = [int(t) for t in toks]
