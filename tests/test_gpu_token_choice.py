@@ -159,14 +159,32 @@ def test_tc_full_size_sampled(cf):
     from paper_2604_01622_gb300.layer import tc_capacity
     w = I.scaled(I.WORKLOADS["ec_d2048_e64"], layers=1)
     inp = I.make_inputs(w)
+    _check_full(inp, 8, tc_capacity(cf, 8, w.N, w.E))
+
+
+def test_tc_large_batch_past_32_bit_offsets():
+    """262144 tokens (the bench workload's 32768 repeated 8 times), top-8 dropless: about
+    2.1 M padded expert rows, so the gathered rows hold 4.4 G elements, past 32-bit element
+    offsets; samples include the last tokens."""
+    base = I.scaled(I.WORKLOADS["ec_d2048_e64"], layers=1)
+    inp0 = I.make_inputs(base)
+    G = 8
+    w = I.scaled(base, G=G * base.G)
+    X = I.Tensor(np.tile(inp0.X.data, (G, 1)), inp0.X.dtype)
+    dY = I.Tensor(np.tile(inp0.dY.data, (G, 1)), inp0.dY.dtype)
+    inp = I.Inputs(w, X, dY, (np.arange(w.G + 1) * w.L).astype(np.int32),
+                   np.zeros(w.G, np.int32), inp0.layers)
+    _check_full(inp, 8, -1, extra=[w.N - 1, w.N - 1000])
+
+
+def _check_full(inp, k, cap, extra=()):
+    w = inp.w
     L = inp.layers[0]
-    k = 8
-    cap = tc_capacity(cf, k, w.N, w.E)
     lay, out = _run(inp, k, cap)
     S_gpu, choice, kept = _check_selection(out, k, cap, w.E)
     Wr = L.Wr.f64()
     rng = np.random.default_rng(99)
-    toks = np.sort(rng.choice(w.N, 16, replace=False))
+    toks = np.union1d(rng.choice(w.N, 16, replace=False), np.array(extra, dtype=np.int64))
     part = ~kept.all(axis=1)
     if part.any():   # tokens with a dropped pair
         toks = np.union1d(toks, rng.choice(np.nonzero(part)[0], min(8, int(part.sum())),
