@@ -480,16 +480,23 @@ def run_ours(args):
     gemm_per_launch = flops_step / max(1, gemm_launches / args.steps)
     b = 2 if w.dtype == "bf16" else 4
     N, d, E = w.N, w.d, w.E
+    Ep = (E + 63) // 64 * 64
+    parts = 2 * math.ceil(w.d_ff / 256) if w.dtype == "bf16" else 1
+    fused_rb = E % 4 == 0 and E <= 128 and not tc   # one router-backward kernel
     mem_bytes = {
-        "router_gemm_softmax": N * d * b + 2 * N * E * 4,
-        "topk": 2 * N * E * 4 + 2 * P * 4,
+        # X, S and S^T; expert choice also sets the slot map [N][E] to -1 there
+        "router_gemm_softmax": N * d * b + 2 * N * E * 4 + (0 if tc else N * E * 4),
+        "topk": N * E * 4 + 3 * P * 4,      # S^T read; idx, gate and the selected slots
         "tc_route": 2 * N * E * 4 + 3 * P * 4,
         "gather": (N + P) * d * b,          # token-major: each X row read once, P rows written
         "combine": P * d * b + N * d * b,
         "bwd_gather_scale": 3 * P * d * b,
         "gather_dy": (N + P) * d * b,
-        "softmax_bwd": 3 * N * E * 4,
-        "dgate_reduce": (2 * math.ceil(w.d_ff / 256) + 1) * P * 4,
+        # slot map and S read, gate-gradient partials read, dZ planes (bf16) or dZ (fp32)
+        "softmax_bwd": (2 * N * E * 4 + parts * P * 4
+                        + (2 * N * Ep * 2 if w.dtype == "bf16" else N * E * 4)) if fused_rb
+                       else 3 * N * E * 4,
+        "dgate_reduce": (parts + 1) * P * 4,
         "dx_combine": P * d * b + 2 * N * d * b,   # dH rows; the router's dX part; dX
     }
     mem_bytes = {k: v for k, v in mem_bytes.items() if k in per}   # kernels this path launches

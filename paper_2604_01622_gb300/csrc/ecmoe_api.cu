@@ -184,7 +184,8 @@ void layout(ec_ctx* c) {
   c->o_f32a = take(f32n * 4);
   c->o_f32b = take((use_tc(c) ? 0 : big) * 4);
   c->o_dXr = take(N * d * es);   // the router's part of dX, in the layer dtype
-  c->o_colsum = take((size_t)colsum_scratch_floats((int)N, (int)E) * 4);
+  c->o_colsum = take((size_t)std::max(colsum_scratch_floats((int)N, (int)E),
+                                       router_bwd_scratch_floats((int)N, (int)E)) * 4);
   // split-K partials of dWr = X^T dZ (tensor cores: equal token blocks, so N % splits == 0)
   if (use_tc(c)) {
     c->wr_splits = 1;
@@ -276,23 +277,26 @@ ec_status run_route(ec_ctx* c, const void* X, const void* Wr, const float* br, c
   float* ST = at<float>(c, c->o_ST);
   float* S = at<float>(c, c->o_S);
   const int nz = N > 0;
+  // each of the three kernels that write S token-major also sets the slot map to -1, so the
+  // top-k kernel writes only the selected entries
+  int* slot = at<int>(c, c->o_slot);
   if (S_in) {
     EC_CUDA(cudaMemcpyAsync(ST, S_in, (size_t)E * N * 4, cudaMemcpyDeviceToDevice, st), "copy S_in");
-    EC_KERNEL("transpose_scores", nz, launch_transpose_scores(ST, S, N, E, st));
+    EC_KERNEL("transpose_scores", nz, launch_transpose_scores(ST, S, slot, N, E, st));
   } else if (use_tc(c)) {
     EC_KERNEL("router_gemm_softmax", 2 * nz,
-              tc_router_softmax(X, Wr, at<void>(c, c->o_wrpad), br, S, ST, N, d, E,
+              tc_router_softmax(X, Wr, at<void>(c, c->o_wrpad), br, S, ST, slot, N, d, E,
                                 at<int>(c, c->o_status), st));
   } else {
     float* Z = at<float>(c, c->o_f32a);
     EC_KERNEL("router_gemm", nz,
               launch_simt_gemm(sg(X, 0, d, 1, Wr, 0, E, 1, Z, 0, E, N, E, d, 1), et(c), et(c), st));
-    EC_KERNEL("router_softmax", nz, launch_softmax_rows(Z, br, S, ST, N, E, st));
+    EC_KERNEL("router_softmax", nz, launch_softmax_rows(Z, br, S, ST, slot, N, E, st));
   }
   EC_KERNEL("topk", 1,
             launch_topk(ST, N, E, c->G, at<int>(c, c->o_goff), at<int>(c, c->o_kg),
                         at<int>(c, c->o_koff), c->M, c->max_group, at<int>(c, c->o_idx),
-                        at<float>(c, c->o_gate), at<int>(c, c->o_slot), st));
+                        at<float>(c, c->o_gate), slot, st));
   return EC_OK;
 }
 
@@ -517,12 +521,24 @@ ec_status run_backward(ec_ctx* c, const void* dY, void* dX, float* dWr, float* d
   T* dXr = at<T>(c, c->o_dXr);
   float* part = at<float>(c, c->o_part);
   const T* res = c->residual ? dYt : nullptr;
+  // Up to 128 experts one kernel sums the gate-gradient partials, applies the softmax
+  // Jacobian and takes the bias gradient's column sums (plus one kernel that adds those up).
+  const float* S = at<float>(c, c->o_S);
+  const bool fused = router_bwd_fused(E, (int64_t)P);
+  float* colsum = at<float>(c, c->o_colsum);
+  const int rb_launches = nz * (1 + (dbr ? 1 : 0));
   if (use_tc(c)) {
     bf16* dZb = at<bf16>(c, c->o_dZb);
-    float* dgsum = at<float>(c, c->o_dgsum);
-    EC_KERNEL("dgate_reduce", pz, launch_reduce_splits(dgate, dgsum, P, c->dg_parts, st));
-    EC_KERNEL("softmax_bwd", nz,
-              launch_softmax_bwd(at<float>(c, c->o_S), slot, dgsum, dZ, dZb, N, E, c->Ep, M, st));
+    if (fused) {
+      EC_KERNEL("softmax_bwd", rb_launches,
+                launch_router_softmax_bwd(S, slot, dgate, c->dg_parts, nullptr, dZb, dbr, colsum,
+                                          N, E, c->Ep, M, st));
+    } else {
+      float* dgsum = at<float>(c, c->o_dgsum);
+      EC_KERNEL("dgate_reduce", pz, launch_reduce_splits(dgate, dgsum, P, c->dg_parts, st));
+      EC_KERNEL("softmax_bwd", nz,
+                launch_softmax_bwd(S, slot, dgsum, dZ, dZb, N, E, c->Ep, M, st));
+    }
     EC_KERNEL("router_dgrad_gemm", nz,
               tc_router_dgrad(dZb, at<void>(c, c->o_wrpad), dXr, N, d, c->Ep, status, st));
     EC_KERNEL("dx_combine", nz,
@@ -532,8 +548,12 @@ ec_status run_backward(ec_ctx* c, const void* dY, void* dX, float* dWr, float* d
     EC_KERNEL("router_wgrad_reduce", 1,
               launch_reduce_partials(part, dWr, d, E, c->Ep, 2 * c->wr_splits, st));
   } else {
-    EC_KERNEL("softmax_bwd", nz,
-              launch_softmax_bwd(at<float>(c, c->o_S), slot, dgate, dZ, nullptr, N, E, E, M, st));
+    if (fused)
+      EC_KERNEL("softmax_bwd", rb_launches,
+                launch_router_softmax_bwd(S, slot, dgate, 1, dZ, nullptr, dbr, colsum, N, E, E, M,
+                                          st));
+    else
+      EC_KERNEL("softmax_bwd", nz, launch_softmax_bwd(S, slot, dgate, dZ, nullptr, N, E, E, M, st));
     EC_KERNEL("router_dgrad_gemm", nz,
               launch_simt_gemm(sg(dZ, 0, E, 1, c->Wr, 0, 1, E, reinterpret_cast<float*>(dXr), 0, d,
                                   N, d, E, 1),
@@ -548,8 +568,7 @@ ec_status run_backward(ec_ctx* c, const void* dY, void* dX, float* dWr, float* d
     EC_KERNEL("router_wgrad_reduce", 1,
               launch_reduce_splits(part, dWr, (int64_t)d * E, c->wr_splits, st));
   }
-  if (dbr)
-    EC_KERNEL("router_dbias", 2, launch_colsum(dZ, dbr, N, E, at<float>(c, c->o_colsum), st));
+  if (dbr && !fused) EC_KERNEL("router_dbias", 2, launch_colsum(dZ, dbr, N, E, colsum, st));
   return EC_OK;
 }
 
@@ -582,8 +601,8 @@ ec_status run_tc_forward(ec_ctx* c, const void* X, const void* Wr, const float* 
   bf16* O = at<bf16>(c, c->o_O);
   if (!nz) return EC_OK;
   EC_KERNEL("router_gemm_softmax", 2,
-            tc_router_softmax(X, Wr, at<void>(c, c->o_wrpad), br, S, at<float>(c, c->o_ST), N, d,
-                              E, status, st));
+            tc_router_softmax(X, Wr, at<void>(c, c->o_wrpad), br, S, at<float>(c, c->o_ST),
+                              nullptr, N, d, E, status, st));
   EC_KERNEL("tc_route", 5,
             launch_tc_route(S, N, E, k, c->tc_cap, at<int>(c, c->o_choice),
                             at<float>(c, c->o_tgate), at<float>(c, c->o_Zs), count, tiles,

@@ -50,7 +50,7 @@ struct Args {
   const float* bias;
   int64_t ld;                   // output row stride (elements)
   int64_t bstride;              // output batch stride (elements)
-  int n_valid;                  // router: number of experts
+  int n_valid;                  // router: number of experts (out2: int map set to -1 beside S)
   int* status;
   // Variable rows per expert (token-choice routing): expert e owns padded rows
   // vm_tiles[e]*PADR .. vm_tiles[e+1]*PADR of the row-major activations, of which the first
@@ -1047,6 +1047,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
           const float inv = 1.0f / sum;
           float* S = reinterpret_cast<float*>(p.out0);
           float* ST = reinterpret_cast<float*>(p.out1);
+          int* slot = reinterpret_cast<int*>(p.out2);
           const bool vec = (E & 3) == 0;   // rows of S start on 16-byte boundaries
 #pragma unroll
           for (int c = 0; c < NCH; ++c) {
@@ -1054,15 +1055,23 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
             for (int i = 0; i < 32; ++i) ev[c][i] *= inv;
             if (row_ok) {
               float* srow = S + (int64_t)gm * E + c * 32;
+              int* lrow = slot ? slot + (int64_t)gm * E + c * 32 : nullptr;
               if (vec && c * 32 + 32 <= E) {
 #pragma unroll
                 for (int j = 0; j < 8; ++j)
                   reinterpret_cast<float4*>(srow)[j] =
                       make_float4(ev[c][4 * j], ev[c][4 * j + 1], ev[c][4 * j + 2], ev[c][4 * j + 3]);
+                if (lrow)
+#pragma unroll
+                  for (int j = 0; j < 8; ++j)
+                    reinterpret_cast<int4*>(lrow)[j] = make_int4(-1, -1, -1, -1);
               } else {
 #pragma unroll
                 for (int i = 0; i < 32; ++i)
-                  if (c * 32 + i < E) srow[i] = ev[c][i];
+                  if (c * 32 + i < E) {
+                    srow[i] = ev[c][i];
+                    if (lrow) lrow[i] = -1;
+                  }
               }
 #pragma unroll
               for (int i = 0; i < 32; ++i)
@@ -1096,6 +1105,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
           const float inv = 1.0f / sum;
           float* S = reinterpret_cast<float*>(p.out0);
           float* ST = reinterpret_cast<float*>(p.out1);
+          int* slot = reinterpret_cast<int*>(p.out2);
 #pragma unroll 1
           for (int c = 0; c < BN / 32; ++c) {
             tmem_ld32(tacc + c * 32, v);
@@ -1107,6 +1117,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
                 const float pr = expf(f32(v[i]) + (p.bias ? p.bias[e] : 0.f) - mx) * inv;
                 S[(int64_t)gm * E + e] = pr;
                 ST[(int64_t)e * p.M + gm] = pr;
+                if (slot) slot[(int64_t)gm * E + e] = -1;
               }
             }
           }
@@ -1287,8 +1298,8 @@ __global__ void wait_probe_kernel(int* status, unsigned long long limit) {
   } while (0)
 
 cudaError_t tc_router_softmax(const void* X, const void* Wr, void* Wr_pad, const float* br,
-                              float* S, float* ST, int N, int d, int E, int* status,
-                              cudaStream_t st) {
+                              float* S, float* ST, int* slot_init, int N, int d, int E,
+                              int* status, cudaStream_t st) {
   if (N == 0) return cudaSuccess;
   const int Ep = (E + 63) / 64 * 64;
   pad_router_weights<<<256, 256, 0, st>>>(static_cast<const bf16*>(Wr), static_cast<bf16*>(Wr_pad),
@@ -1300,6 +1311,7 @@ cudaError_t tc_router_softmax(const void* X, const void* Wr, void* Wr_pad, const
   Args p = base_args(1, N, Ep, d, Ep, status);
   p.out0 = S;
   p.out1 = ST;
+  p.out2 = slot_init;
   p.bias = br;
   p.n_valid = E;
   switch (Ep) {

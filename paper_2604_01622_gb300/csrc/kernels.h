@@ -7,13 +7,16 @@
 namespace ecmoe {
 
 // ---------------------------------------------------------------- router + selection
-// Row softmax of fp32 logits Z [N][E] (+ br) -> S [N][E] and S^T [E][N].
-cudaError_t launch_softmax_rows(const float* Z, const float* br, float* S, float* ST, int N, int E,
-                                cudaStream_t st);
-// Transpose scores [E][N] -> [N][E] (used when the caller supplies S).
-cudaError_t launch_transpose_scores(const float* ST, float* S, int N, int E, cudaStream_t st);
-// Expert-choice top-k per (expert, group) over S^T [E][N]; writes idx/gate [E][M] and the
-// token->slot map slot [N][E] (m or -1).
+// Row softmax of fp32 logits Z [N][E] (+ br) -> S [N][E] and S^T [E][N]; sets the slot map
+// slot [N][E] to -1 (the state launch_topk expects).
+cudaError_t launch_softmax_rows(const float* Z, const float* br, float* S, float* ST, int* slot,
+                                int N, int E, cudaStream_t st);
+// Transpose scores [E][N] -> [N][E] (used when the caller supplies S); sets slot [N][E] to -1.
+cudaError_t launch_transpose_scores(const float* ST, float* S, int* slot, int N, int E,
+                                    cudaStream_t st);
+// Expert-choice top-k per (expert, group) over S^T [E][N]; writes idx/gate [E][M] and, for
+// the selected pairs only, the token->slot map slot [N][E] (= m). The other entries of slot
+// must already hold -1.
 cudaError_t launch_topk(const float* ST, int N, int E, int G, const int* group_off, const int* k_g,
                         const int* k_off, int M, int max_group, int* idx, float* gate, int* slot,
                         cudaStream_t st);
@@ -61,8 +64,22 @@ cudaError_t launch_combine(const T* O, const float* gate, const int* slot, const
 template <typename T>
 cudaError_t launch_bwd_gather_scale(const T* dY, const T* O, const int* idx, const float* gate,
                                     T* dO, float* dgate, int64_t P, int d, cudaStream_t st);
+// Router softmax Jacobian: dS[t][e] = dgate of the pair (t chosen by e) else 0,
+// dZ = S (dS - <dS, S>_row). dgate [E*M] summed beforehand; writes dZ [N][E] and, with dZb,
+// the bf16 hi/lo planes [2][N][Ep] (any E <= 512).
 cudaError_t launch_softmax_bwd(const float* S, const int* slot, const float* dgate, float* dZ,
                                __nv_bfloat16* dZb, int N, int E, int Ep, int M, cudaStream_t st);
+// The same, fused with the sum of the gate-gradient partials dg_part [parts][E*M] (in part
+// order) and, with dbr, with the router bias gradient dbr[e] = sum_t dZ[t][e] (per-CTA
+// column sums in scratch, then summed in a fixed order: deterministic). dZ and dZb are each
+// optional. For E % 4 == 0, E <= 128 and E*M < 2^31 (router_bwd_fused); one kernel, two
+// with dbr. scratch: router_bwd_scratch_floats(N, E) floats.
+bool router_bwd_fused(int E, int64_t P);
+int64_t router_bwd_scratch_floats(int N, int E);
+cudaError_t launch_router_softmax_bwd(const float* S, const int* slot, const float* dg_part,
+                                      int parts, float* dZ, __nv_bfloat16* dZb, float* dbr,
+                                      float* scratch, int N, int E, int Ep, int M,
+                                      cudaStream_t st);
 cudaError_t launch_reduce_partials(const float* part, float* out, int rows, int cols, int ld,
                                    int splits, cudaStream_t st);
 // dX_t = dXr_t + R_t + R2_t (each if given) + sum of the token's dH rows, summed in fp32;

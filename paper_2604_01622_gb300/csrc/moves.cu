@@ -288,6 +288,202 @@ cudaError_t launch_softmax_bwd(const float* S, const int* slot, const float* dga
   return cudaGetLastError();
 }
 
+// Fused form. A group of LPT lanes owns a token (LPT = 16 up to 64 experts, 32 up to 128),
+// each lane one 4-expert vector (16-byte loads of slot and S); a warp takes 32/LPT tokens at a
+// time and kRbIter of them back to back, all loads issued first. The gate gradients of the
+// selected pairs are gathered cooperatively: the warp lists its selected pairs in shared
+// memory (ballot order), each lane sums the partials of list entries lane, lane+32, ... (two
+// at a time, partials in order, as reduce_splits_kernel does), and every lane reads its own
+// sums back. The column sums of dZ for the bias gradient are taken per CTA in a fixed order.
+constexpr int kRbWarps = 8, kRbIter = 4;
+
+template <int LPT, bool WDZ, bool BIAS>
+__global__ void __launch_bounds__(kRbWarps * 32, 4)
+router_softmax_bwd_kernel(const float* __restrict__ S, const int* __restrict__ slot,
+                          const float* __restrict__ dg_part, int parts, int64_t P,
+                          float* __restrict__ dZ, bf16* __restrict__ dZb,
+                          float* __restrict__ bpart, int N, int E, int Ep, int M) {
+  constexpr int TPW = 32 / LPT;                   // tokens per warp per step
+  constexpr int TPB = kRbWarps * TPW * kRbIter;   // tokens per CTA
+  constexpr int NC = kRbIter * 4;                 // (token, expert) candidates per lane
+  __shared__ int s_list[kRbWarps][32 * NC];
+  __shared__ float s_col[BIAS ? kRbWarps * TPW : 1][BIAS ? 4 * LPT : 1];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int sub = lane / LPT, v = lane % LPT;     // token of the warp, expert vector
+  const bool vok = v < (E >> 2);
+  const int t0 = blockIdx.x * TPB + (warp * TPW + sub) * kRbIter;
+  int4 sl[kRbIter];
+  float4 sv[kRbIter];
+#pragma unroll
+  for (int it = 0; it < kRbIter; ++it) {
+    const int t = t0 + it;
+    sl[it] = make_int4(-1, -1, -1, -1);
+    sv[it] = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (t < N && vok) {
+      sl[it] = reinterpret_cast<const int4*>(slot + (size_t)t * E)[v];
+      sv[it] = reinterpret_cast<const float4*>(S + (size_t)t * E)[v];
+    }
+  }
+  // list of the warp's selected pairs (offset of the pair in a partial plane)
+  int* list = s_list[warp];
+  int pos[NC];
+  int cnt = 0;
+  const unsigned below = (1u << lane) - 1u;
+#pragma unroll
+  for (int it = 0; it < kRbIter; ++it) {
+    const int m[4] = {sl[it].x, sl[it].y, sl[it].z, sl[it].w};
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const bool sel = m[j] >= 0;
+      const unsigned b = __ballot_sync(0xffffffffu, sel);
+      const int p = cnt + __popc(b & below);
+      pos[it * 4 + j] = sel ? p : -1;
+      if (sel) list[p] = (4 * v + j) * M + m[j];
+      cnt += __popc(b);
+    }
+  }
+  __syncwarp();
+  for (int i = lane; i < cnt; i += 64) {
+    const int i2 = i + 32;
+    const int o1 = list[i];
+    const int o2 = i2 < cnt ? list[i2] : o1;
+    float s1 = 0.f, s2 = 0.f;
+    for (int k0 = 0; k0 < parts; k0 += 8) {
+      float x1[8], x2[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const bool ok = k0 + j < parts;
+        x1[j] = ok ? dg_part[(size_t)(k0 + j) * P + o1] : 0.f;
+        x2[j] = ok ? dg_part[(size_t)(k0 + j) * P + o2] : 0.f;
+      }
+#pragma unroll
+      for (int j = 0; j < 8; ++j)
+        if (k0 + j < parts) { s1 += x1[j]; s2 += x2[j]; }
+    }
+    reinterpret_cast<float*>(list)[i] = s1;
+    if (i2 < cnt) reinterpret_cast<float*>(list)[i2] = s2;
+  }
+  __syncwarp();
+  float csum[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+  for (int it = 0; it < kRbIter; ++it) {
+    float ds[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int p = pos[it * 4 + j];
+      ds[j] = p >= 0 ? reinterpret_cast<const float*>(list)[p] : 0.f;
+    }
+    float dot = 0.f;
+    dot = fmaf(ds[0], sv[it].x, dot);
+    dot = fmaf(ds[1], sv[it].y, dot);
+    dot = fmaf(ds[2], sv[it].z, dot);
+    dot = fmaf(ds[3], sv[it].w, dot);
+#pragma unroll
+    for (int o = LPT / 2; o > 0; o >>= 1) dot += __shfl_xor_sync(0xffffffffu, dot, o);
+    const int t = t0 + it;
+    if (t >= N || !vok) continue;
+    const float z[4] = {sv[it].x * (ds[0] - dot), sv[it].y * (ds[1] - dot),
+                        sv[it].z * (ds[2] - dot), sv[it].w * (ds[3] - dot)};
+    if (WDZ) reinterpret_cast<float4*>(dZ + (size_t)t * E)[v] = make_float4(z[0], z[1], z[2], z[3]);
+    if (dZb) {
+      uint32_t h[2], l[2];
+#pragma unroll
+      for (int j = 0; j < 2; ++j) {
+        const __nv_bfloat162 hh = __floats2bfloat162_rn(z[2 * j], z[2 * j + 1]);
+        const float2 hf = __bfloat1622float2(hh);
+        const __nv_bfloat162 ll = __floats2bfloat162_rn(z[2 * j] - hf.x, z[2 * j + 1] - hf.y);
+        h[j] = *reinterpret_cast<const uint32_t*>(&hh);
+        l[j] = *reinterpret_cast<const uint32_t*>(&ll);
+      }
+      reinterpret_cast<uint2*>(dZb + (size_t)t * Ep)[v] = make_uint2(h[0], h[1]);
+      reinterpret_cast<uint2*>(dZb + (size_t)N * Ep + (size_t)t * Ep)[v] = make_uint2(l[0], l[1]);
+    }
+    if (BIAS)
+#pragma unroll
+      for (int j = 0; j < 4; ++j) csum[j] += z[j];
+  }
+  if (dZb && Ep > E)   // zero padding columns E..Ep-1 of both planes
+    for (int it = 0; it < kRbIter; ++it) {
+      const int t = t0 + it;
+      if (t >= N) break;
+      for (int c = E + 4 * v; c < Ep; c += 4 * LPT) {
+        *reinterpret_cast<uint2*>(dZb + (size_t)t * Ep + c) = make_uint2(0u, 0u);
+        *reinterpret_cast<uint2*>(dZb + (size_t)N * Ep + (size_t)t * Ep + c) = make_uint2(0u, 0u);
+      }
+    }
+  if (BIAS) {
+    // CTA column sums, rows in order; partials stored column-major [E][gridDim.x]
+    const int row = warp * TPW + sub;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) s_col[row][4 * v + j] = csum[j];
+    __syncthreads();
+    for (int c = threadIdx.x; c < E; c += blockDim.x) {
+      float s = 0.f;
+      for (int r = 0; r < kRbWarps * TPW; ++r) s += s_col[r][c];
+      bpart[(size_t)c * gridDim.x + blockIdx.x] = s;
+    }
+  }
+}
+
+// out[c] = sum over b of part[c][b] (nblk partials per column): one warp per column, lanes
+// over strided partials, then a fixed butterfly.
+__global__ void colsum_rows_kernel(const float* __restrict__ part, int nblk, int E,
+                                   float* __restrict__ out) {
+  const int c = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+  if (c >= E) return;
+  float s = 0.f;
+  for (int b = lane; b < nblk; b += 32) s += part[(size_t)c * nblk + b];
+  s = warp_sum(s);
+  if (lane == 0) out[c] = s;
+}
+
+bool router_bwd_fused(int E, int64_t P) {
+  return E > 0 && E % 4 == 0 && E <= 128 && P <= INT32_MAX;   // pair offsets kept as int
+}
+
+static int router_bwd_tpb(int E) { return kRbWarps * (E <= 64 ? 2 : 1) * kRbIter; }
+
+int64_t router_bwd_scratch_floats(int N, int E) {
+  return (int64_t)E * ((N + router_bwd_tpb(E) - 1) / router_bwd_tpb(E));
+}
+
+template <int LPT, bool WDZ, bool BIAS>
+static void router_bwd_go(int nblk, const float* S, const int* slot, const float* dg_part,
+                          int parts, int64_t P, float* dZ, bf16* dZb, float* bpart, int N, int E,
+                          int Ep, int M, cudaStream_t st) {
+  router_softmax_bwd_kernel<LPT, WDZ, BIAS><<<nblk, kRbWarps * 32, 0, st>>>(
+      S, slot, dg_part, parts, P, dZ, dZb, bpart, N, E, Ep, M);
+}
+
+template <int LPT>
+static void router_bwd_pick(int nblk, const float* S, const int* slot, const float* dg_part,
+                            int parts, int64_t P, float* dZ, bf16* dZb, float* bpart, int N,
+                            int E, int Ep, int M, cudaStream_t st) {
+  if (dZ) {
+    if (bpart) router_bwd_go<LPT, true, true>(nblk, S, slot, dg_part, parts, P, dZ, dZb, bpart, N, E, Ep, M, st);
+    else router_bwd_go<LPT, true, false>(nblk, S, slot, dg_part, parts, P, dZ, dZb, bpart, N, E, Ep, M, st);
+  } else {
+    if (bpart) router_bwd_go<LPT, false, true>(nblk, S, slot, dg_part, parts, P, dZ, dZb, bpart, N, E, Ep, M, st);
+    else router_bwd_go<LPT, false, false>(nblk, S, slot, dg_part, parts, P, dZ, dZb, bpart, N, E, Ep, M, st);
+  }
+}
+
+cudaError_t launch_router_softmax_bwd(const float* S, const int* slot, const float* dg_part,
+                                      int parts, float* dZ, bf16* dZb, float* dbr,
+                                      float* scratch, int N, int E, int Ep, int M,
+                                      cudaStream_t st) {
+  const int64_t P = (int64_t)E * M;
+  if (!router_bwd_fused(E, P) || parts < 1 || (dZb && (Ep < E || Ep % 4)))
+    return cudaErrorInvalidValue;
+  if (N == 0) return dbr ? cudaMemsetAsync(dbr, 0, (size_t)E * sizeof(float), st) : cudaSuccess;
+  const int nblk = (N + router_bwd_tpb(E) - 1) / router_bwd_tpb(E);
+  float* bpart = dbr ? scratch : nullptr;
+  if (E <= 64) router_bwd_pick<16>(nblk, S, slot, dg_part, parts, P, dZ, dZb, bpart, N, E, Ep, M, st);
+  else router_bwd_pick<32>(nblk, S, slot, dg_part, parts, P, dZ, dZb, bpart, N, E, Ep, M, st);
+  if (dbr) colsum_rows_kernel<<<(E + 7) / 8, 256, 0, st>>>(bpart, nblk, E, dbr);
+  return cudaGetLastError();
+}
+
 // out[i][e] = sum_s part[s][i][e] for the first `cols` of `ld` columns.
 __global__ void reduce_partials_kernel(const float* __restrict__ part, float* __restrict__ out,
                                        int rows, int cols, int ld, int splits) {

@@ -4,8 +4,8 @@
 // with the largest S[t,e] (Sec. 2.2 TopC; capacity per group, Sec. 4.2). Ties go to the
 // lower token index and the kept tokens are written in ascending index. One CTA per
 // (e, g) runs an MSB-first radix select over order-preserving 32-bit keys of the fp32
-// scores to find the k-th largest key, then compacts the column in index order with two
-// block scans, which makes the result unique and independent of thread timing.
+// scores to find the k-th largest key, then compacts the column in index order with one
+// block scan, which makes the result unique and independent of thread timing.
 #include "common.cuh"
 #include "kernels.h"
 
@@ -13,9 +13,10 @@ namespace ecmoe {
 
 // ------------------------------------------------------------------ softmax over experts
 // 32 tokens per CTA; the S^T tile is staged in shared memory so both layouts are written
-// with coalesced stores.
+// with coalesced stores. The slot map [N][E] (same layout as S) is set to -1 beside S.
 __global__ void softmax_rows_kernel(const float* __restrict__ Z, const float* __restrict__ br,
-                                    float* __restrict__ S, float* __restrict__ ST, int N, int E) {
+                                    float* __restrict__ S, float* __restrict__ ST,
+                                    int* __restrict__ slot, int N, int E) {
   extern __shared__ float tile[];  // [32][E+1]
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
   const int t0 = blockIdx.x * 32;
@@ -43,6 +44,7 @@ __global__ void softmax_rows_kernel(const float* __restrict__ Z, const float* __
       float p = tile[r * (E + 1) + e] * inv;
       tile[r * (E + 1) + e] = p;
       S[(size_t)t * E + e] = p;
+      slot[(size_t)t * E + e] = -1;
     }
   }
   __syncthreads();
@@ -52,18 +54,19 @@ __global__ void softmax_rows_kernel(const float* __restrict__ Z, const float* __
   }
 }
 
-cudaError_t launch_softmax_rows(const float* Z, const float* br, float* S, float* ST, int N, int E,
-                                cudaStream_t st) {
+cudaError_t launch_softmax_rows(const float* Z, const float* br, float* S, float* ST, int* slot,
+                                int N, int E, cudaStream_t st) {
   if (N == 0) return cudaSuccess;
   size_t smem = (size_t)32 * (E + 1) * sizeof(float);
   if (smem > 48 * 1024)
     cudaFuncSetAttribute(softmax_rows_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  softmax_rows_kernel<<<(N + 31) / 32, 256, smem, st>>>(Z, br, S, ST, N, E);
+  softmax_rows_kernel<<<(N + 31) / 32, 256, smem, st>>>(Z, br, S, ST, slot, N, E);
   return cudaGetLastError();
 }
 
-__global__ void transpose_scores_kernel(const float* __restrict__ ST, float* __restrict__ S, int N,
-                                        int E) {
+// S = (S^T)^T through a 32 x 32 shared tile; the slot map is set to -1 beside S.
+__global__ void transpose_scores_kernel(const float* __restrict__ ST, float* __restrict__ S,
+                                        int* __restrict__ slot, int N, int E) {
   __shared__ float tile[32][33];
   const int t0 = blockIdx.x * 32, e0 = blockIdx.y * 32;
   const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;  // 256 threads: 8 rows per pass
@@ -74,14 +77,18 @@ __global__ void transpose_scores_kernel(const float* __restrict__ ST, float* __r
   __syncthreads();
   for (int r = ty; r < 32; r += 8) {
     int t = t0 + r, e = e0 + tx;
-    if (e < E && t < N) S[(size_t)t * E + e] = tile[tx][r];
+    if (e < E && t < N) {
+      S[(size_t)t * E + e] = tile[tx][r];
+      slot[(size_t)t * E + e] = -1;
+    }
   }
 }
 
-cudaError_t launch_transpose_scores(const float* ST, float* S, int N, int E, cudaStream_t st) {
+cudaError_t launch_transpose_scores(const float* ST, float* S, int* slot, int N, int E,
+                                    cudaStream_t st) {
   if (N == 0) return cudaSuccess;
   dim3 grid((N + 31) / 32, (E + 31) / 32);
-  transpose_scores_kernel<<<grid, 256, 0, st>>>(ST, S, N, E);
+  transpose_scores_kernel<<<grid, 256, 0, st>>>(ST, S, slot, N, E);
   return cudaGetLastError();
 }
 
@@ -93,93 +100,126 @@ __device__ __forceinline__ uint32_t score_key(float s) {
   return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
 }
 
-// Exclusive scan of one int per thread across the block (blockDim multiple of 32).
-__device__ __forceinline__ int block_excl_scan(int v, int* s_warp) {
+// Exclusive scan of two counts per thread (packed as hi:lo 32-bit halves) across the block.
+__device__ __forceinline__ unsigned long long block_excl_scan2(unsigned long long v,
+                                                               unsigned long long* s_warp) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
-  int incl = v;
+  unsigned long long incl = v;
 #pragma unroll
   for (int o = 1; o < 32; o <<= 1) {
-    int u = __shfl_up_sync(0xffffffffu, incl, o);
+    const unsigned long long u = __shfl_up_sync(0xffffffffu, incl, o);
     if (lane >= o) incl += u;
   }
   if (lane == 31) s_warp[warp] = incl;
   __syncthreads();
   if (warp == 0) {
-    int w = lane < nw ? s_warp[lane] : 0;
-    int wi = w;
+    const unsigned long long w = lane < nw ? s_warp[lane] : 0ull;
+    unsigned long long wi = w;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
-      int u = __shfl_up_sync(0xffffffffu, wi, o);
+      const unsigned long long u = __shfl_up_sync(0xffffffffu, wi, o);
       if (lane >= o) wi += u;
     }
     if (lane < nw) s_warp[lane] = wi - w;
   }
   __syncthreads();
-  int r = incl - v + s_warp[warp];
+  const unsigned long long r = incl - v + s_warp[warp];
   __syncthreads();
   return r;
 }
 
+// The k-th largest key is found by an MSB-first radix select over the offsets u = key - kmin
+// of the column (kmin, kmax its smallest and largest key), 8 bits per pass starting at the top
+// bit of kmax - kmin. Scores of one expert over a sequence span a narrow range, so digits of
+// the raw key would put most of the column into a few bins of the first pass (and serialise
+// its shared-memory atomics); digits of the offset spread it over the whole histogram. The
+// select stops early once the bin that holds the k-th key is taken whole. The selected set
+// is the one the (score desc, index asc) order defines, whatever the digit boundaries.
+//
+// The slot map is expected to hold -1 for every (token, expert) on entry (written by the
+// kernel that produced S); only the selected entries are written here.
 template <bool SMEM>
-__global__ void __launch_bounds__(512)
+__global__ void __launch_bounds__(512, 4)
 topk_kernel(const float* __restrict__ ST, int N, int E, const int* __restrict__ group_off,
             const int* __restrict__ k_g, const int* __restrict__ k_off, int M,
             int* __restrict__ idx, float* __restrict__ gate, int* __restrict__ slot) {
-  extern __shared__ uint32_t skeys[];
+  extern __shared__ uint4 skeys4[];
+  uint32_t* skeys = reinterpret_cast<uint32_t*>(skeys4);
   __shared__ int hist[256];
-  __shared__ int s_warp[32];
+  __shared__ unsigned long long s_scan[32];
+  __shared__ uint32_t s_mn[32], s_mx[32];
   __shared__ uint32_t s_prefix;
-  __shared__ int s_remaining;
+  __shared__ int s_remaining, s_done;
   const int e = blockIdx.x, g = blockIdx.y;
   const int tid = threadIdx.x, nthr = blockDim.x, lane = tid & 31, warp = tid >> 5;
+  const int nw = nthr >> 5;
   const int lo = group_off[g];
   const int L = group_off[g + 1] - lo;
   const int k = k_g[g];
   const int base = k_off[g];
   const float* col = ST + (size_t)e * N + lo;
 
-  if (SMEM) {
-    for (int i = tid; i < L; i += nthr) skeys[i] = score_key(col[i]);
-    __syncthreads();
+  uint32_t mn = 0xFFFFFFFFu, mx = 0u;
+  for (int i = tid; i < L; i += nthr) {
+    const uint32_t key = score_key(col[i]);
+    if (SMEM) skeys[i] = key;
+    mn = min(mn, key);
+    mx = max(mx, key);
   }
-  auto key_at = [&](int i) -> uint32_t { return SMEM ? skeys[i] : score_key(col[i]); };
+  mn = __reduce_min_sync(0xffffffffu, mn);
+  mx = __reduce_max_sync(0xffffffffu, mx);
+  if (lane == 0) { s_mn[warp] = mn; s_mx[warp] = mx; }
+  __syncthreads();
+  if (warp == 0) {
+    mn = __reduce_min_sync(0xffffffffu, lane < nw ? s_mn[lane] : 0xFFFFFFFFu);
+    mx = __reduce_max_sync(0xffffffffu, lane < nw ? s_mx[lane] : 0u);
+    if (lane == 0) { s_mn[0] = mn; s_mx[0] = mx; }
+  }
+  __syncthreads();
+  mn = s_mn[0];
+  mx = s_mx[0];
+  auto off_at = [&](int i) -> uint32_t { return (SMEM ? skeys[i] : score_key(col[i])) - mn; };
 
-  // Radix select of the k-th largest key, 8 bits per pass from the top.
-  uint32_t T = 0xFFFFFFFFu;
+  // threshold T (an offset) and how many keys equal to it are taken (in token order)
+  uint32_t T = 0u;
   int need_eq = 0;
   if (k > 0) {
-    uint32_t prefix = 0u, mask = 0u;
+    int hi = mx == mn ? 0 : 32 - __clz(mx - mn);   // every offset lies in [0, 2^hi)
+    uint32_t prefix = 0u, mask = hi == 32 ? 0u : ~((1u << hi) - 1u);
     int remaining = k;
-    for (int pass = 0; pass < 4; ++pass) {
-      const int shift = 24 - 8 * pass;
+    bool done = hi == 0;                           // all keys equal: the first k are taken
+    while (!done && hi > 0) {
+      const int shift = max(hi - 8, 0);
+      const uint32_t dmask = (1u << (hi - shift)) - 1u;
       for (int i = tid; i < 256; i += nthr) hist[i] = 0;
       __syncthreads();
       for (int i = tid; i < L; i += nthr) {
-        uint32_t key = key_at(i);
-        if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1);
+        const uint32_t u = off_at(i);
+        if ((u & mask) == prefix) atomicAdd(&hist[(u >> shift) & dmask], 1);
       }
       __syncthreads();
       if (warp == 0) {
         // lane l owns bins 255-8l .. 248-8l (descending); find the bin holding the
-        // remaining-th largest key
+        // remaining-th largest offset
         int c[8], local = 0;
 #pragma unroll
         for (int j = 0; j < 8; ++j) { c[j] = hist[255 - (lane * 8 + j)]; local += c[j]; }
         int incl = local;
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) {
-          int u = __shfl_up_sync(0xffffffffu, incl, o);
+          const int u = __shfl_up_sync(0xffffffffu, incl, o);
           if (lane >= o) incl += u;
         }
-        int excl = incl - local;
+        const int excl = incl - local;
         if (excl < remaining && remaining <= incl) {
           int run = excl;
 #pragma unroll
           for (int j = 0; j < 8; ++j) {
             if (run + c[j] >= remaining) {
-              uint32_t bin = 255u - (uint32_t)(lane * 8 + j);
+              const uint32_t bin = 255u - (uint32_t)(lane * 8 + j);
               s_prefix = prefix | (bin << shift);
               s_remaining = remaining - run;
+              s_done = run + c[j] == remaining;   // the whole bin is taken
               break;
             }
             run += c[j];
@@ -189,48 +229,68 @@ topk_kernel(const float* __restrict__ ST, int N, int E, const int* __restrict__ 
       __syncthreads();
       prefix = s_prefix;
       remaining = s_remaining;
-      mask |= 0xFFu << shift;
+      done = s_done;
+      mask |= dmask << shift;
+      hi = shift;
       __syncthreads();
     }
     T = prefix;
-    need_eq = remaining;
+    // a bin taken whole: every offset >= T is selected
+    need_eq = (done && hi > 0) ? 0x7FFFFFFF : remaining;
   }
   const bool any = k > 0;
 
-  // Compaction in token order: thread tid owns a contiguous chunk.
-  const int chunk = (L + nthr - 1) / nthr;
+  // Compaction in token order: thread tid owns a contiguous chunk (a multiple of 4 keys, read
+  // 16 bytes at a time from shared memory); one scan gives both the keys above T and the keys
+  // equal to T before the chunk.
+  const int chunk = ((L + nthr - 1) / nthr + 3) & ~3;
   const int i0 = min(L, tid * chunk), i1 = min(L, i0 + chunk);
-  int n_eq = 0;
-  if (any)
-    for (int i = i0; i < i1; ++i) n_eq += key_at(i) == T;
-  const int eq_before = block_excl_scan(n_eq, s_warp);
-  int n_sel = 0;
-  {
-    int r = eq_before;
-    for (int i = i0; i < i1; ++i) {
-      const uint32_t key = key_at(i);
-      const bool eq = any && key == T;
-      n_sel += any && (key > T || (eq && r < need_eq));
-      r += eq;
+  auto load4 = [&](int i, uint32_t (&u)[4]) {
+    if (SMEM && i + 4 <= i1) {
+      const uint4 q = skeys4[i >> 2];
+      u[0] = q.x - mn; u[1] = q.y - mn; u[2] = q.z - mn; u[3] = q.w - mn;
+    } else {
+#pragma unroll
+      for (int j = 0; j < 4; ++j) u[j] = i + j < i1 ? off_at(i + j) : 0u;
     }
-  }
-  const int sel_before = block_excl_scan(n_sel, s_warp);
-  int r = eq_before, pos = sel_before;
+  };
+  uint32_t n_gt = 0, n_eq = 0;
+  if (any)
+    for (int i = i0; i < i1; i += 4) {
+      uint32_t u[4];
+      load4(i, u);
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+        if (i + j < i1) { n_gt += u[j] > T; n_eq += u[j] == T; }
+    }
+  const unsigned long long before =
+      block_excl_scan2(((unsigned long long)n_gt << 32) | n_eq, s_scan);
+  int r = (int)(before & 0xFFFFFFFFu);                 // keys equal to T before this one
+  int pos = (int)(before >> 32) + min(r, need_eq);     // selected keys before this one
+  if (!any) return;
   int* idx_row = idx + (size_t)e * M + base;
   float* gate_row = gate + (size_t)e * M + base;
-  for (int i = i0; i < i1; ++i) {
-    const uint32_t key = key_at(i);
-    const bool eq = any && key == T;
-    const bool s = any && (key > T || (eq && r < need_eq));
-    r += eq;
-    const int t = lo + i;
-    if (s) {
-      idx_row[pos] = t;
-      gate_row[pos] = col[i];
-      slot[(size_t)t * E + e] = base + pos;
-      ++pos;
-    } else {
-      slot[(size_t)t * E + e] = -1;
+  for (int i = i0; i < i1; i += 4) {
+    uint32_t u[4];
+    load4(i, u);
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      if (i + j >= i1) break;
+      const bool eq = u[j] == T;
+      const bool s = u[j] > T || (eq && r < need_eq);
+      r += eq;
+      if (s) {
+        const int t = lo + i + j;
+        const uint32_t key = u[j] + mn;
+        // the gate is the score the key encodes (-0.0 and +0.0 share a key: read it back)
+        const float sv = key == 0x80000000u
+                             ? col[i + j]
+                             : __uint_as_float((key & 0x80000000u) ? (key & 0x7FFFFFFFu) : ~key);
+        idx_row[pos] = t;
+        gate_row[pos] = sv;
+        slot[(size_t)t * E + e] = base + pos;
+        ++pos;
+      }
     }
   }
 }
@@ -241,7 +301,7 @@ cudaError_t launch_topk(const float* ST, int N, int E, int G, const int* group_o
   if (G == 0 || E == 0) return cudaSuccess;
   dim3 grid(E, G);
   const int threads = max_group >= 4096 ? 512 : (max_group >= 1024 ? 256 : 128);
-  const size_t smem = (size_t)max_group * sizeof(uint32_t);
+  const size_t smem = ((size_t)max_group + 3) / 4 * 16;
   if (smem <= 200 * 1024) {
     if (smem > 48 * 1024)
       cudaFuncSetAttribute(topk_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,

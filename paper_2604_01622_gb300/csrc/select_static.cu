@@ -9,8 +9,9 @@
 //
 // The array is module memory: every GPU that loads this library holds it until the process
 // exits. All calls share it, and it keeps the last call's contents: the group tables are
-// rewritten by each call and the selection kernel writes every slot entry it reads, so
-// nothing has to start at zero. Two calls whose work overlaps on the GPU (different streams,
+// rewritten by each call, and the slot map (the selection kernel's token->slot output, which
+// this variant does not return) is only written, never read, so nothing has to start at
+// zero or -1. Two calls whose work overlaps on the GPU (different streams,
 // or different host threads) race on the array; order them.
 #include <mutex>
 

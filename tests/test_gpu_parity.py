@@ -78,6 +78,38 @@ def test_selection_bit_exact_on_given_scores(quant):
         assert np.array_equal(S_out.cpu().numpy(), S.T)
 
 
+def test_selection_degenerate_columns():
+    """Columns the radix select treats specially: all scores equal (no pass), two values,
+    one outlier stretching the range to both signs (offsets over 31 bits), subnormals and
+    signed zeros, a column whose k-th score is tied across a group boundary; k = 0, k = L."""
+    from paper_2604_01622_gb300.layer import ECMoELayer
+    rng = np.random.default_rng(9)
+    N, E = 2500, 8
+    S = np.empty((N, E), np.float32)
+    S[:, 0] = 0.25
+    S[:, 1] = np.where(rng.random(N) < 0.3, 0.5, 0.125)
+    S[:, 2] = (1.0 / 64) * (1 + 0.02 * rng.standard_normal(N))
+    S[7, 2] = 3.0e38
+    S[11, 2] = -3.0e38
+    S[:, 3] = rng.integers(1, 40, N).astype(np.float32) * np.float32(1e-45)
+    S[:, 4] = np.where(rng.random(N) < 0.5, np.float32(-0.0), np.float32(0.0))
+    S[:, 5] = np.round(rng.random(N) * 4) / 4
+    S[:, 6] = -rng.random(N)
+    S[:, 7] = rng.random(N)
+    group_off = np.array([0, 1000, 1001, 1800, N], np.int32)
+    for k_g in (np.array([300, 1, 0, 700], np.int32), np.array([1000, 0, 799, 1], np.int32),
+                np.array([999, 1, 1, 350], np.int32)):
+        lay = ECMoELayer(N, 64, E, 64, group_off, k_g, dtype="f32")
+        idx, gate, _ = lay.route(S_in=torch.from_numpy(np.ascontiguousarray(S.T)).cuda())
+        lay.check()
+        ref_idx, ref_gate = O.ec_select(S.astype(np.float64), group_off, k_g)
+        assert np.array_equal(idx.cpu().numpy(), ref_idx)
+        g = gate.cpu().numpy()
+        assert np.array_equal(g.astype(np.float64), ref_gate)
+        # gates carry the scores bit for bit (the sign of zero included)
+        assert np.array_equal(g.view(np.uint32), S.T[np.arange(E)[:, None], ref_idx].view(np.uint32))
+
+
 def test_selection_long_groups_beyond_shared_memory():
     """Groups longer than the shared-memory key buffer take the global-memory path."""
     from paper_2604_01622_gb300.layer import ECMoELayer
