@@ -36,7 +36,8 @@ enum Epi : int {
   EPI_STORE_BF16 = 2,    // plain bf16 store
   EPI_SWIGLU_BWD = 3,    // acc = dU; reads A, B; writes dA, dB bf16
   EPI_STORE_F32 = 4,     // plain fp32 store
-  EPI_STORE_F32_SPLIT = 5  // cols [0,BN/2) -> out0, [BN/2,BN) -> out1, fp32
+  EPI_STORE_F32_SPLIT = 5, // cols [0,BN/2) -> out0, [BN/2,BN) -> out1, fp32
+  EPI_ROUTER_ST = 6      // the router softmax with S and S^T leaving by TMA stores (BN <= 128)
 };
 
 struct Args {
@@ -270,13 +271,21 @@ __host__ __device__ constexpr uint32_t tmem_cols() {
 }
 
 // Epilogue staging: one 4 KB buffer per epilogue warp (a 32 x 32 fp32 chunk, or two 32 x 32
-// bf16 chunks), written by the warp and stored to global memory by TMA.
+// bf16 chunks), written by the warp and stored to global memory by TMA. The staged router
+// epilogue takes two per warp (a chunk of S and the same chunk of S^T) and keeps the bias
+// row (up to 128 fp32) behind them.
 constexpr uint32_t STAGE_BUF = 4096;
 
-template <int BN, int STAGES, bool PAIR, int EPW, bool STAGED>
+__host__ __device__ constexpr uint32_t stage_bytes(int EPI, int EPW) {
+  return EPI == EPI_ROUTER ? 0u
+         : EPI == EPI_ROUTER_ST ? EPW * 2 * STAGE_BUF + 512u
+                                : EPW * STAGE_BUF;
+}
+
+template <int BN, int STAGES, bool PAIR, int EPW, int EPI>
 __host__ __device__ constexpr uint32_t smem_bytes() {
   return 1024 /*align slack*/ + STAGES * (BM * BK * 2 + (PAIR ? BN / 2 : BN) * BK * 2) +
-         (STAGED ? EPW * STAGE_BUF : 0) + 256 /*barriers*/;
+         stage_bytes(EPI, EPW) + 256 /*barriers*/;
 }
 
 __device__ __forceinline__ float f32(uint32_t u) { return __uint_as_float(u); }
@@ -447,11 +456,14 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
   constexpr uint32_t IDESC = instr_desc<SEGW, A_MN, B_MN, TM>();
   static_assert(BN % 64 == 0 && (BN <= 256 || (WIDE && PAIR)), "BN");
   static_assert(!PAIR || BN % 128 == 0, "pair tiles split B in two 64-column multiples");
-  static_assert(!WIDE || (EPI != EPI_SWIGLU_BWD && EPI != EPI_ROUTER && STAGES > TAIL),
+  static_assert(!WIDE || (EPI != EPI_SWIGLU_BWD && EPI != EPI_ROUTER && EPI != EPI_ROUTER_ST &&
+                          STAGES > TAIL),
                 "wide tiles: plain, split-column and SwiGLU forward epilogues");
   static_assert(EPW == 4 || EPW == 8, "epilogue warps: one or two per TMEM lane quarter");
-  static_assert(EPI != EPI_ROUTER || EPW == 4, "the row softmax needs whole rows per thread");
-  // every epilogue except the router's writes through shared memory and TMA stores
+  static_assert((EPI != EPI_ROUTER && EPI != EPI_ROUTER_ST) || EPW == 4,
+                "the row softmax needs whole rows per thread");
+  static_assert(EPI != EPI_ROUTER_ST || (BN <= 128 && !PAIR), "staged router: up to 128 experts");
+  // every epilogue except the plain router's writes through shared memory and TMA stores
   constexpr bool STAGED = EPI != EPI_ROUTER;
 
   extern __shared__ uint8_t smem_raw[];
@@ -460,7 +472,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
   uint8_t* sA = smem;
   uint8_t* sB = smem + STAGES * A_BYTES;
   uint8_t* sStage = sB + STAGES * B_BYTES;   // 1024-aligned: A_BYTES, B_BYTES are multiples
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sStage + (STAGED ? EPW * STAGE_BUF : 0));
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sStage + stage_bytes(EPI, EPW));
   uint64_t* full = bars;
   uint64_t* empty = bars + STAGES;
   uint64_t* tfull = bars + 2 * STAGES;
@@ -495,7 +507,8 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
   }
   if (STAGED && warp >= 2 && lane == 0) {
     prefetch_map(&mO0);
-    if (EPI == EPI_SWIGLU_FWD || EPI == EPI_SWIGLU_BWD || EPI == EPI_STORE_F32_SPLIT)
+    if (EPI == EPI_SWIGLU_FWD || EPI == EPI_SWIGLU_BWD || EPI == EPI_STORE_F32_SPLIT ||
+        EPI == EPI_ROUTER_ST)
       prefetch_map(&mO1);
     if (EPI == EPI_SWIGLU_FWD) prefetch_map(&mO2);
   }
@@ -713,6 +726,13 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
     int slot = 0;   // staging half of the next bf16 chunk (warp-uniform)
     int it = 0;
     bool stop = false;
+    // staged router: the bias row goes to shared memory once (every row reads all of it)
+    float* s_bias = reinterpret_cast<float*>(sStage + EPW * 2 * STAGE_BUF);
+    if constexpr (EPI == EPI_ROUTER_ST) {
+      const int t = (int)threadIdx.x - 64;   // 0..127 over the four epilogue warps
+      if (t < p.n_valid) s_bias[t] = p.bias ? __ldg(p.bias + t) : 0.f;
+      asm volatile("bar.sync 1, 128;" ::: "memory");
+    }
     for (int tile = cid; tile < total && !stop; tile += nwalk, ++it) {
       const Tile T = tile_at<VARM, TM>(p, tile, tiles_per_b, rank);
       const int nt = T.nt;
@@ -1018,9 +1038,10 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
             f2_split(dot2, de, dd);
             p.dgate_part[(int64_t)(nt * NPART + part) * p.dgate_stride + grow] = de + dd;
           }
-        } else if constexpr (EPI == EPI_ROUTER && BN <= 128) {
-          // up to 128 experts the row's logits stay in registers: one TMEM read, exp once,
-          // and the row of S written with 16-byte stores when E allows it
+        } else if constexpr ((EPI == EPI_ROUTER || EPI == EPI_ROUTER_ST) && BN <= 128) {
+          // up to 128 experts the row's logits stay in registers: one TMEM read, exp once;
+          // the staged form stores S and S^T as 32 x 32 chunks by TMA, the plain one writes
+          // the row of S with 16-byte stores when E allows it
           const int E = p.n_valid;
           constexpr int NCH = BN / 32;
           float ev[NCH][32];
@@ -1032,7 +1053,13 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
 #pragma unroll
             for (int i = 0; i < 32; ++i) {
               const int e = c * 32 + i;
-              ev[c][i] = e < E ? f32(v[i]) + (p.bias ? __ldg(p.bias + e) : 0.f) : -INFINITY;
+              float bias = 0.f;
+              if constexpr (EPI == EPI_ROUTER_ST) {
+                if (e < E) bias = s_bias[e];
+              } else {
+                bias = p.bias && e < E ? __ldg(p.bias + e) : 0.f;
+              }
+              ev[c][i] = e < E ? f32(v[i]) + bias : -INFINITY;
               mx = fmaxf(mx, ev[c][i]);
             }
           }
@@ -1045,9 +1072,43 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
               sum += ev[c][i];
             }
           const float inv = 1.0f / sum;
+          int* smap = reinterpret_cast<int*>(p.out2);
+          if constexpr (EPI == EPI_ROUTER_ST) {
+            // chunk c: S rows of this warp's 32 tokens (128-byte swizzle, thread = row) and
+            // the same values as S^T rows of 32 experts (thread = column: each expert's row
+            // of 32 tokens is one 128-byte line of the buffer, so the stores are conflict-free)
+            uint8_t* bS = sStage + (warp - 2) * 2 * STAGE_BUF;
+            uint8_t* bT = bS + STAGE_BUF;
+#pragma unroll
+            for (int c = 0; c < NCH; ++c) {
+#pragma unroll
+              for (int i = 0; i < 32; ++i) ev[c][i] *= inv;
+              if (c * 32 >= E || !st_any) continue;
+              if (lane == 0) bulk_wait_read<0>();   // both buffers have been read
+              __syncwarp();
+              stage_f32(bS, lane, ev[c]);
+#pragma unroll
+              for (int i = 0; i < 32; ++i)
+                *reinterpret_cast<float*>(bT + i * 128 + ((((lane >> 2) ^ (i & 7)) << 4) |
+                                                          ((lane & 3) << 2))) = ev[c][i];
+              fence_async_smem();
+              __syncwarp();
+              if (lane == 0) {
+                tma_store_3d(&mO0, smem_u32(bS), c * 32, srow, 0);
+                tma_store_3d(&mO1, smem_u32(bT), srow, c * 32, 0);
+              }
+            }
+            // the slot map's rows of this warp's tokens: one contiguous block, -1 throughout
+            if (smap && st_any) {
+              const int nrow = min(32, T.valid - q * 32);
+              int4* blk = reinterpret_cast<int4*>(smap + (int64_t)srow * E);
+              const int n4 = nrow * (E >> 2);
+              for (int j = lane; j < n4; j += 32) blk[j] = make_int4(-1, -1, -1, -1);
+            }
+          } else {
           float* S = reinterpret_cast<float*>(p.out0);
           float* ST = reinterpret_cast<float*>(p.out1);
-          int* slot = reinterpret_cast<int*>(p.out2);
+          int* slot = smap;
           const bool vec = (E & 3) == 0;   // rows of S start on 16-byte boundaries
 #pragma unroll
           for (int c = 0; c < NCH; ++c) {
@@ -1077,6 +1138,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
               for (int i = 0; i < 32; ++i)
                 if (c * 32 + i < E) ST[(int64_t)(c * 32 + i) * p.M + gm] = ev[c][i];
             }
+          }
           }
         } else if constexpr (EPI == EPI_ROUTER) {
           const int E = p.n_valid;
@@ -1209,7 +1271,7 @@ cudaError_t launch(const CUtensorMap& a0, const CUtensorMap& a1, const CUtensorM
                    const CUtensorMap& b1, const CUtensorMap& o0, const CUtensorMap& o1,
                    const CUtensorMap& o2, Args p, cudaStream_t st) {
   auto kern = tc_gemm_kernel<BN, A_MN, B_MN, B_SPLIT, K_SPLIT, EPI, STAGES, EPW, PAIR, VARM>;
-  constexpr uint32_t smem = smem_bytes<BN, STAGES, PAIR, EPW, EPI != EPI_ROUTER>();
+  constexpr uint32_t smem = smem_bytes<BN, STAGES, PAIR, EPW, EPI>();
   static_assert(smem <= 232448, "dynamic shared memory above the 227 KB per-block limit");
   constexpr int threads = 64 + 32 * EPW;
   static bool attr = false;
@@ -1314,6 +1376,17 @@ cudaError_t tc_router_softmax(const void* X, const void* Wr, void* Wr_pad, const
   p.out2 = slot_init;
   p.bias = br;
   p.n_valid = E;
+  if (Ep <= 128 && E % 4 == 0 && N % 4 == 0) {
+    // S [N][E] and S^T [E][N] leave through TMA stores (row strides of 16-byte multiples)
+    CUtensorMap mo0, mo1;
+    TC_TRY(make_out_map(&mo0, S, true, E, N, 1));
+    TC_TRY(make_out_map(&mo1, ST, true, N, E, 1));
+    if (Ep == 64)
+      return launch<64, false, true, false, false, EPI_ROUTER_ST, 8, 4>(ma, ma, mb, mb, mo0, mo1, ma,
+                                                                         p, st);
+    return launch<128, false, true, false, false, EPI_ROUTER_ST, 6, 4>(ma, ma, mb, mb, mo0, mo1, ma,
+                                                                        p, st);
+  }
   switch (Ep) {
     // the router epilogue writes S and S^T itself: the output maps are unused
     case 64:
