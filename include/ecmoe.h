@@ -73,10 +73,23 @@ ec_status ec_ctx_create(ec_ctx** out, int32_t N, int32_t d, int32_t E, int32_t d
 void ec_ctx_destroy(ec_ctx* ctx);
 
 /* Replace the per-group capacities (Sec. 4.2: a new k_g per denoising step).
- * sum(k_g) must not exceed the M the context was created with (the workspace is sized
- * for it). Copies k_g to the device with a synchronous copy; call outside stream capture.
- * Invalidates saved forward state. */
+ * k_g: host array of G int32. sum(k_g) must not exceed the M the context was created with
+ * (the workspace is sized for it); the context's M becomes sum(k_g). Synchronous: waits for
+ * the whole device (no earlier kernel on any stream may still read the group tables), then
+ * copies k_g to the device; call outside stream capture. Invalidates saved forward state. */
 ec_status ec_ctx_set_capacity(ec_ctx* ctx, const int32_t* k_g);
+
+/* The same update without a host round trip (Sec. 4.2: capacity that changes with the
+ * masking ratio of every sequence, step after step). k_g_dev: device array of G int32,
+ * read on `stream` by one small kernel, so a schedule computed on the device (or uploaded
+ * ahead for many steps) takes effect in stream order with no copy and no synchronisation.
+ * The new capacities must keep the context's current M: 0 <= k_g[g] <= L_g and
+ * sum(k_g) == ec_rows_per_expert(ctx) (the FLOPs-matched schedules of Sec. 4.2 keep the
+ * total; use ec_ctx_set_capacity to change it). The check runs on the device: if it fails,
+ * the previous capacities stay in force and the next ec_check_device returns EC_ERR_SHAPE.
+ * Needs the workspace; invalidates saved forward state. ec_ctx_set_workspace re-uploads the
+ * capacities last given on the host. */
+ec_status ec_ctx_set_capacity_async(ec_ctx* ctx, const int32_t* k_g_dev, void* stream);
 
 /* Residual form for stacked layers x_{l+1} = x_l + EC(x_l) (off by default): with it on,
  * ec_moe_forward writes Y = X + EC(X) and ec_moe_backward writes dX = dY + (the input
@@ -179,6 +192,12 @@ ec_status ec_moe_backward_shared(ec_ctx* ctx, const void* dY, void* dX, float* d
  * same context whose inputs are still alive. */
 ec_status ec_tc_ctx_create(ec_ctx** out, int32_t N, int32_t d, int32_t E, int32_t d_ff,
                            int32_t k, int32_t capacity, int32_t dtype);
+
+/* Token-choice expert capacity for a capacity factor (Sec. 2.2): ceil(CF k N / E), evaluated
+ * left to right in double precision, for the `capacity` argument of ec_tc_ctx_create.
+ * Returns -1 (dropless, no cap) for capacity_factor <= 0 or NaN, -2 for k < 1, N < 0,
+ * E < 1 or a result that does not fit. Host only. */
+int64_t ec_tc_capacity(double capacity_factor, int32_t k, int32_t N, int32_t E);
 ec_status ec_tc_forward(ec_ctx* ctx, const void* X, const void* Wr, const float* br,
                         const void* Wg, const void* Wu, const void* Wd, void* Y, int32_t* choice,
                         float* gate, int32_t* kept, int32_t* load, float* S_out, void* stream);
@@ -186,7 +205,8 @@ ec_status ec_tc_backward(ec_ctx* ctx, const void* dY, void* dX, float* dWr, floa
                          float* dWg, float* dWu, float* dWd, void* stream);
 
 /* Synchronise `stream`, read and clear the device status word. Returns EC_ERR_TIMEOUT if a
- * kernel gave up on a bounded wait since the last check, EC_ERR_CUDA on a CUDA error. */
+ * kernel gave up on a bounded wait since the last check, EC_ERR_SHAPE if a capacity update
+ * from device memory (ec_ctx_set_capacity_async) was rejected, EC_ERR_CUDA on a CUDA error. */
 ec_status ec_check_device(ec_ctx* ctx, void* stream);
 
 /* Per-kernel timing. With profiling on, every kernel launch of the following calls is
@@ -249,8 +269,12 @@ ec_status ec_selftest_bounded_wait(ec_ctx* ctx, uint64_t limit_ns, void* stream)
  *   gate [E][M] float (device, M = sum k_g) receive the same selection as ec_route with S_in.
  * Returns EC_ERR_UNSUPPORTED if N*E > EC_STATIC_SELECT_MAX_SCORES or
  * G > EC_STATIC_SELECT_MAX_GROUPS, EC_ERR_SHAPE / EC_ERR_INVALID_ARG on bad arguments,
- * EC_ERR_CUDA if a CUDA call fails. Asynchronous on `stream` (the host tables are copied
- * before the call returns). The first call on each device looks up the array's device
+ * EC_ERR_CUDA if a CUDA call fails. Asynchronous on `stream`. The call copies group_off and
+ * k_g into its own host array before it enqueues anything, so the caller may reuse or free
+ * them (pinned or pageable) as soon as it returns. It returns EC_ERR_UNSUPPORTED, having
+ * enqueued nothing, while `stream` is being captured: the group tables are copied from host
+ * memory that lives only for the duration of the call. The first call in each CUDA context
+ * (a device's primary context, and again after cudaDeviceReset) looks up the array's device
  * address; make that first call before any stream capture. All calls share the array:
  * calls that overlap on the GPU (other streams, other threads) race and must be ordered. */
 #define EC_STATIC_SELECT_MAX_SCORES 4194304
@@ -261,6 +285,12 @@ ec_status ec_select_static(const float* S, int32_t N, int32_t E, int32_t G,
 
 /* Message of the last failed call on this context ("" if none). Owned by the context. */
 const char* ec_last_error(const ec_ctx* ctx);
+
+/* The same message copied into a caller buffer: at most n-1 bytes and a terminating NUL
+ * (nothing is written when n is 0). Returns the status of the last failed call on the
+ * context (EC_OK if none has failed), or EC_ERR_INVALID_ARG for a NULL context, or a NULL
+ * buffer with n > 0. Device-side failures reach the message through ec_check_device. */
+ec_status ec_get_last_error(const ec_ctx* ctx, char* buf, size_t n);
 
 /* Static name of a status code. */
 const char* ec_status_string(ec_status s);

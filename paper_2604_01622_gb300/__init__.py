@@ -29,6 +29,7 @@ EXPORTS = (
     "ec_selftest_bounded_wait", "ec_ctx_set_residual", "ec_capacity_schedule",
     "ec_ctx_set_shared", "ec_moe_forward_shared", "ec_moe_backward_shared",
     "ec_tc_ctx_create", "ec_tc_forward", "ec_tc_backward", "ec_ctx_set_tiles",
+    "ec_ctx_set_capacity_async", "ec_get_last_error", "ec_tc_capacity",
 )
 EC_TILES_AUTO, EC_TILES_256, EC_TILES_512 = 0, 1, 2
 
@@ -59,6 +60,9 @@ def load():
         "ec_ctx_create": (i32, [ctypes.POINTER(vp), i32, i32, i32, i32, i32, P32, P32, i32]),
         "ec_ctx_destroy": (None, [vp]),
         "ec_ctx_set_capacity": (i32, [vp, P32]),
+        "ec_ctx_set_capacity_async": (i32, [vp, vp, vp]),
+        "ec_get_last_error": (i32, [vp, ctypes.c_char_p, sz]),
+        "ec_tc_capacity": (i64, [ctypes.c_double, i32, i32, i32]),
         "ec_rows_per_expert": (i64, [vp]),
         "ec_workspace_bytes": (sz, [vp]),
         "ec_ctx_set_workspace": (i32, [vp, vp, sz]),
@@ -126,6 +130,11 @@ def ec_ctx_destroy(ctx):
 def ec_ctx_set_capacity(ctx, k_g):
     k_arr, k_ptr = _i32(k_g)
     _check(ctx, load().ec_ctx_set_capacity(ctx, k_ptr))
+
+
+def ec_ctx_set_capacity_async(ctx, k_g_dev: int, stream):
+    """k_g from a device array (int32 [G]) on `stream`; sum(k_g) must keep the context's M."""
+    _check(ctx, load().ec_ctx_set_capacity_async(ctx, k_g_dev, stream))
 
 
 def ec_ctx_set_residual(ctx, on: bool):
@@ -248,3 +257,21 @@ def ec_capacity_schedule(scheduler, k_min, k_max, E, group_off, r, sigma=0.22):
 
 def ec_last_error(ctx) -> str:
     return load().ec_last_error(ctx).decode()
+
+
+def ec_get_last_error(ctx, n: int = 512):
+    """(status of the last failed call, its message truncated to n-1 bytes)."""
+    buf = ctypes.create_string_buffer(n) if n > 0 else None
+    st = load().ec_get_last_error(ctx, buf, n)
+    return int(st), (buf.value.decode() if buf is not None else "")
+
+
+def ec_tc_capacity(capacity_factor, k: int, N: int, E: int) -> int:
+    """Token-choice capacity ceil(CF k N / E) computed by the library; -1 (dropless) when
+    capacity_factor is None or <= 0."""
+    if capacity_factor is None:
+        return -1
+    v = int(load().ec_tc_capacity(float(capacity_factor), int(k), int(N), int(E)))
+    if v < -1:
+        raise ECError(EC_ERR_SHAPE, "ec_tc_capacity rejected its arguments")
+    return v

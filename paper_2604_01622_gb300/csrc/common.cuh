@@ -7,7 +7,9 @@
 namespace ecmoe {
 
 // Device status word codes (first word of the workspace).
-enum : int { DEV_OK = 0, DEV_TIMEOUT = 1 };
+// DEV_BAD_CAPACITY: a capacity update read from device memory was rejected (the previous
+// capacities stay in force).
+enum : int { DEV_OK = 0, DEV_TIMEOUT = 1, DEV_BAD_CAPACITY = 2 };
 
 // Element type tags.
 typedef __nv_bfloat16 bf16;

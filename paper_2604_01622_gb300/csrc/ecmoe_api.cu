@@ -4,6 +4,8 @@
 #include <string>
 #include <vector>
 #include <cstdio>
+#include <cmath>
+#include <algorithm>
 #include <cstring>
 #include <cstdarg>
 
@@ -52,6 +54,7 @@ struct ec_ctx {
   int tiles = EC_TILES_AUTO;   // expert-GEMM tile policy (ec_ctx_set_tiles)
   size_t o_choice = 0, o_tgate = 0, o_Zs = 0, o_count = 0, o_tiles = 0, o_kept = 0, o_tcscr = 0;
   std::string err;
+  ec_status err_status = EC_OK;   // status of the last failed call (ec_get_last_error)
 };
 
 namespace {
@@ -64,6 +67,7 @@ ec_status fail(ec_ctx* c, ec_status s, const char* fmt, ...) {
     vsnprintf(buf, sizeof buf, fmt, ap);
     va_end(ap);
     c->err = buf;
+    c->err_status = s;
   }
   return s;
 }
@@ -269,6 +273,12 @@ SimtGemmArgs sg(const void* A, int64_t a_bs, int64_t a_ms, int64_t a_ks, const v
 
 EType et(const ec_ctx* c) { return c->dtype == EC_BF16 ? EType::BF16 : EType::F32; }
 
+// The router weights as the tensor cores read them, [d][Ep] bf16: Wr itself when E is a
+// multiple of 64, else the zero-padded copy the forward pass made.
+const void* router_b(ec_ctx* c) {
+  return router_needs_pad(c->E) ? at<void>(c, c->o_wrpad) : c->Wr;
+}
+
 // ---------------------------------------------------------------- router + selection
 template <typename T>
 ec_status run_route(ec_ctx* c, const void* X, const void* Wr, const float* br, const float* S_in,
@@ -284,7 +294,7 @@ ec_status run_route(ec_ctx* c, const void* X, const void* Wr, const float* br, c
     EC_CUDA(cudaMemcpyAsync(ST, S_in, (size_t)E * N * 4, cudaMemcpyDeviceToDevice, st), "copy S_in");
     EC_KERNEL("transpose_scores", nz, launch_transpose_scores(ST, S, slot, N, E, st));
   } else if (use_tc(c)) {
-    EC_KERNEL("router_gemm_softmax", 2 * nz,
+    EC_KERNEL("router_gemm_softmax", (router_needs_pad(E) ? 2 : 1) * nz,
               tc_router_softmax(X, Wr, at<void>(c, c->o_wrpad), br, S, ST, slot, N, d, E,
                                 at<int>(c, c->o_status), st));
   } else {
@@ -540,7 +550,7 @@ ec_status run_backward(ec_ctx* c, const void* dY, void* dX, float* dWr, float* d
                 launch_softmax_bwd(S, slot, dgsum, dZ, dZb, N, E, c->Ep, M, st));
     }
     EC_KERNEL("router_dgrad_gemm", nz,
-              tc_router_dgrad(dZb, at<void>(c, c->o_wrpad), dXr, N, d, c->Ep, status, st));
+              tc_router_dgrad(dZb, router_b(c), dXr, N, d, c->Ep, status, st));
     EC_KERNEL("dx_combine", nz,
               launch_dx_combine<T>(dH, slot, dXr, res, dHsh, static_cast<T*>(dX), N, E, M, d, st));
     EC_KERNEL("router_wgrad_gemm", nz,
@@ -600,7 +610,7 @@ ec_status run_tc_forward(ec_ctx* c, const void* X, const void* Wr, const float* 
   bf16* U = at<bf16>(c, c->o_U);
   bf16* O = at<bf16>(c, c->o_O);
   if (!nz) return EC_OK;
-  EC_KERNEL("router_gemm_softmax", 2,
+  EC_KERNEL("router_gemm_softmax", router_needs_pad(E) ? 2 : 1,
             tc_router_softmax(X, Wr, at<void>(c, c->o_wrpad), br, S, at<float>(c, c->o_ST),
                               nullptr, N, d, E, status, st));
   EC_KERNEL("tc_route", 5,
@@ -665,7 +675,7 @@ ec_status run_tc_backward(ec_ctx* c, const void* dY, void* dX, float* dWr, float
                                   at<float>(c, c->o_tgate), at<float>(c, c->o_Zs), slot, dgsum, dZ,
                                   dZb, N, E, c->Ep, k, st));
   EC_KERNEL("router_dgrad_gemm", 1,
-            tc_router_dgrad(dZb, at<void>(c, c->o_wrpad), dXr, N, d, c->Ep, status, st));
+            tc_router_dgrad(dZb, router_b(c), dXr, N, d, c->Ep, status, st));
   EC_KERNEL("dx_combine", 1,
             launch_dx_combine<bf16>(dH, slot, dXr, c->residual ? dYt : nullptr, nullptr,
                                     static_cast<bf16*>(dX), N, E, 0, d, st));
@@ -727,7 +737,26 @@ ec_status ec_ctx_set_capacity(ec_ctx* c, const int32_t* k_g) {
   if (c && c->tc_k) return fail(c, EC_ERR_STATE, "token-choice context: use ec_tc_forward / ec_tc_backward");
   ec_status s = set_groups(c, nullptr, k_g, false);
   if (s != EC_OK) return s;
+  // the group tables are rewritten in place: no kernel of an earlier call, on any stream, may
+  // still be reading them
+  if (c->ws) EC_CUDA(cudaDeviceSynchronize(), "wait for the device before the capacity update");
   return upload_groups(c);
+}
+
+ec_status ec_ctx_set_capacity_async(ec_ctx* c, const int32_t* k_g_dev, void* stream) {
+  ec_status s = check_ready(c);
+  if (s != EC_OK) return s;
+  if (c->tc_k) return fail(c, EC_ERR_STATE, "token-choice context: use ec_tc_forward / ec_tc_backward");
+  if (!k_g_dev) return fail(c, EC_ERR_INVALID_ARG, "k_g is NULL");
+  if (reinterpret_cast<uintptr_t>(k_g_dev) & 3u)
+    return fail(c, EC_ERR_INVALID_ARG, "k_g must be 4-byte aligned");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  c->have_fwd = false;
+  EC_KERNEL("set_capacity", 1,
+            launch_set_capacity(k_g_dev, at<int>(c, c->o_goff), c->G, c->M, at<int>(c, c->o_kg),
+                                at<int>(c, c->o_koff), at<int>(c, c->o_status), st));
+  mark(c, "end", st);
+  return EC_OK;
 }
 
 int64_t ec_rows_per_expert(const ec_ctx* c) { return c ? c->M : -1; }
@@ -1008,11 +1037,34 @@ ec_status ec_check_device(ec_ctx* c, void* stream) {
   EC_CUDA(cudaMemcpy(&word, c->ws + c->o_status, 4, cudaMemcpyDeviceToHost), "read status");
   if (word != DEV_OK) {
     EC_CUDA(cudaMemset(c->ws + c->o_status, 0, 256), "clear status");
+    if (word == DEV_BAD_CAPACITY)
+      return fail(c, EC_ERR_SHAPE,
+                  "a capacity update from device memory was rejected (k_g outside [0, L_g] or "
+                  "sum(k_g) != %d); the previous capacities stayed in force", c->M);
     return fail(c, EC_ERR_TIMEOUT, "a kernel gave up on a bounded wait (device status %d)", word);
   }
   return EC_OK;
 }
 
 const char* ec_last_error(const ec_ctx* c) { return c ? c->err.c_str() : ""; }
+
+ec_status ec_get_last_error(const ec_ctx* c, char* buf, size_t n) {
+  if (!c || (!buf && n > 0)) return EC_ERR_INVALID_ARG;
+  if (n > 0) {
+    const size_t len = std::min(c->err.size(), n - 1);
+    std::memcpy(buf, c->err.data(), len);
+    buf[len] = '\0';
+  }
+  return c->err_status;
+}
+
+int64_t ec_tc_capacity(double capacity_factor, int32_t k, int32_t N, int32_t E) {
+  if (!(capacity_factor > 0.0)) return -1;   // dropless (also for NaN)
+  if (k < 1 || N < 0 || E < 1) return -2;
+  // Sec. 2.2: ceil(CF k N / E), evaluated left to right in double precision
+  const double v = capacity_factor * (double)k * (double)N / (double)E;
+  if (!(v < 9.0e18)) return -2;
+  return (int64_t)std::ceil(v);
+}
 
 }  // extern "C"

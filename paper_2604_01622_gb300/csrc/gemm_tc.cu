@@ -277,8 +277,10 @@ __host__ __device__ constexpr uint32_t tmem_cols() {
 constexpr uint32_t STAGE_BUF = 4096;
 
 __host__ __device__ constexpr uint32_t stage_bytes(int EPI, int EPW) {
+  // staged router: two buffers per warp, the bias row (128 floats) and the per-row partial
+  // maxima and sums the two warps of a lane quarter exchange (2 x 2 x 128 floats)
   return EPI == EPI_ROUTER ? 0u
-         : EPI == EPI_ROUTER_ST ? EPW * 2 * STAGE_BUF + 512u
+         : EPI == EPI_ROUTER_ST ? EPW * 2 * STAGE_BUF + 512u + (EPW > 4 ? 2048u : 0u)
                                 : EPW * STAGE_BUF;
 }
 
@@ -379,7 +381,10 @@ __device__ __forceinline__ void bulk_wait_all() {
 // ------------------------------------------------------------------ tile decode
 // VARM: 0 uniform batch of equal-M problems; 1 variable rows per expert (the M dimension,
 // rows are global padded rows, B is the expert's weights); 2 variable K per expert (weight
-// gradients: K runs over the expert's padded rows).
+// gradients: K runs over the expert's padded rows); 3 one problem whose rows are split
+// evenly over the CTAs in 32-row units (the router: every CTA streams its own contiguous
+// block of tokens, in tiles of up to 128 rows, so no SM is left with a second wave of whole
+// tiles while others idle).
 struct Tile {
   int b, mt, nt;
   int row0;      // first row of this CTA in the A / output row space
@@ -391,8 +396,25 @@ struct Tile {
 template <int VARM, int TM>
 __device__ __forceinline__ Tile tile_at(const Args& p, int tile, int tiles_per_b, uint32_t rank) {
   static_assert(VARM != 1 || TM == PADR, "variable-row tiles are one padding unit high");
+  static_assert(VARM != 3 || TM == BM, "row-split tiles are one CTA high");
   Tile t;
-  if constexpr (VARM == 1) {
+  if constexpr (VARM == 3) {
+    // CTA c owns the 32-row units [c U / G, (c+1) U / G) of the U = ceil(M / 32) units; its
+    // j-th tile (tile = c + j G) starts 128 j rows into that block. valid <= 0: the CTA has
+    // fewer tiles than the longest block (every role skips it).
+    const int G = (int)gridDim.x;
+    const int c = tile % G, j = tile / G;
+    const int64_t units = (p.M + 31) / 32;
+    const int r0 = (int)(32 * ((int64_t)c * units / G));
+    const int r1 = (int)min((int64_t)p.M, 32 * (((int64_t)c + 1) * units / G));
+    t.b = 0;
+    t.mt = j;
+    t.nt = 0;
+    t.row0 = r0 + j * BM;
+    t.valid = min(BM, r1 - t.row0);
+    t.kbl = p.k_blocks;
+    t.krow0 = 0;
+  } else if constexpr (VARM == 1) {
     const int mtile = tile / p.n_tiles;
     t.nt = tile - mtile * p.n_tiles;
     int lo = 0, hi = p.vm_E;   // last expert whose first block is at or before mtile
@@ -460,8 +482,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
                           STAGES > TAIL),
                 "wide tiles: plain, split-column and SwiGLU forward epilogues");
   static_assert(EPW == 4 || EPW == 8, "epilogue warps: one or two per TMEM lane quarter");
-  static_assert((EPI != EPI_ROUTER && EPI != EPI_ROUTER_ST) || EPW == 4,
-                "the row softmax needs whole rows per thread");
+  static_assert(EPI != EPI_ROUTER || EPW == 4, "the plain router keeps whole rows per thread");
   static_assert(EPI != EPI_ROUTER_ST || (BN <= 128 && !PAIR), "staged router: up to 128 experts");
   // every epilogue except the plain router's writes through shared memory and TMA stores
   constexpr bool STAGED = EPI != EPI_ROUTER;
@@ -533,6 +554,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
       bool ok = true;
       for (int tile = cid; tile < total && ok; tile += nwalk) {
         const Tile T = tile_at<VARM, TM>(p, tile, tiles_per_b, rank);
+        if (VARM == 3 && T.valid <= 0) continue;
         const int nt = T.nt;
         const int m0 = T.row0;
         const int ab = VARM ? 0 : T.b;          // batch coordinate of A
@@ -637,7 +659,9 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
         else mma_commit(bar);
       };
       for (int tile = cid; tile < total && ok; tile += nwalk, ++it) {
-        const int kbl = tile_at<VARM, TM>(p, tile, tiles_per_b, 0).kbl;
+        const Tile T0 = tile_at<VARM, TM>(p, tile, tiles_per_b, 0);
+        if (VARM == 3 && T0.valid <= 0) { --it; continue; }
+        const int kbl = T0.kbl;
         if constexpr (!WIDE) {
           const int a = it & 1;
           const uint32_t use = (uint32_t)(it >> 1);
@@ -729,12 +753,13 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
     // staged router: the bias row goes to shared memory once (every row reads all of it)
     float* s_bias = reinterpret_cast<float*>(sStage + EPW * 2 * STAGE_BUF);
     if constexpr (EPI == EPI_ROUTER_ST) {
-      const int t = (int)threadIdx.x - 64;   // 0..127 over the four epilogue warps
-      if (t < p.n_valid) s_bias[t] = p.bias ? __ldg(p.bias + t) : 0.f;
-      asm volatile("bar.sync 1, 128;" ::: "memory");
+      const int t = (int)threadIdx.x - 64;   // over the epilogue warps
+      if (t < 128) s_bias[t] = (p.bias && t < p.n_valid) ? __ldg(p.bias + t) : 0.f;
+      asm volatile("bar.sync 1, %0;" ::"n"(32 * EPW) : "memory");
     }
     for (int tile = cid; tile < total && !stop; tile += nwalk, ++it) {
       const Tile T = tile_at<VARM, TM>(p, tile, tiles_per_b, rank);
+      if (VARM == 3 && T.valid <= 0) { --it; continue; }
       const int nt = T.nt;
       const int gm = T.row0 + r;
       const bool row_ok = r < T.valid;
@@ -1041,18 +1066,21 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
         } else if constexpr ((EPI == EPI_ROUTER || EPI == EPI_ROUTER_ST) && BN <= 128) {
           // up to 128 experts the row's logits stay in registers: one TMEM read, exp once;
           // the staged form stores S and S^T as 32 x 32 chunks by TMA, the plain one writes
-          // the row of S with 16-byte stores when E allows it
+          // the row of S with 16-byte stores when E allows it. With two warps per lane quarter
+          // (staged form) each takes half of the row's chunks and the pair exchanges its
+          // partial maximum and sum through shared memory.
           const int E = p.n_valid;
-          constexpr int NCH = BN / 32;
+          constexpr int NCH = BN / 32 / NPART;     // chunks of 32 experts per warp
+          const int cb0 = part * NCH;              // first chunk of this warp
           float ev[NCH][32];
           float mx = -INFINITY;
 #pragma unroll
           for (int c = 0; c < NCH; ++c) {
-            tmem_ld32(tacc + c * 32, v);
+            tmem_ld32(tacc + (cb0 + c) * 32, v);
             tmem_wait_ld();
 #pragma unroll
             for (int i = 0; i < 32; ++i) {
-              const int e = c * 32 + i;
+              const int e = (cb0 + c) * 32 + i;
               float bias = 0.f;
               if constexpr (EPI == EPI_ROUTER_ST) {
                 if (e < E) bias = s_bias[e];
@@ -1063,14 +1091,27 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
               mx = fmaxf(mx, ev[c][i]);
             }
           }
+          float* s_xmax = s_bias + 128;            // [NPART][128] partial maxima
+          float* s_xsum = s_xmax + 256;            // [NPART][128] partial sums
+          if constexpr (NPART > 1) {
+            s_xmax[part * 128 + r] = mx;
+            asm volatile("bar.sync %0, 64;" ::"r"(2 + q) : "memory");
+            mx = fmaxf(mx, s_xmax[(1 - part) * 128 + r]);
+          }
           float sum = 0.f;
 #pragma unroll
           for (int c = 0; c < NCH; ++c)
 #pragma unroll
             for (int i = 0; i < 32; ++i) {
-              ev[c][i] = c * 32 + i < E ? expf(ev[c][i] - mx) : 0.f;
+              ev[c][i] = (cb0 + c) * 32 + i < E ? expf(ev[c][i] - mx) : 0.f;
               sum += ev[c][i];
             }
+          if constexpr (NPART > 1) {
+            s_xsum[part * 128 + r] = sum;
+            asm volatile("bar.sync %0, 64;" ::"r"(2 + q) : "memory");
+            // the same order in both warps: part 0's sum first
+            sum = part == 0 ? sum + s_xsum[128 + r] : s_xsum[r] + sum;
+          }
           const float inv = 1.0f / sum;
           int* smap = reinterpret_cast<int*>(p.out2);
           if constexpr (EPI == EPI_ROUTER_ST) {
@@ -1081,9 +1122,10 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
             uint8_t* bT = bS + STAGE_BUF;
 #pragma unroll
             for (int c = 0; c < NCH; ++c) {
+              const int cg = cb0 + c;
 #pragma unroll
               for (int i = 0; i < 32; ++i) ev[c][i] *= inv;
-              if (c * 32 >= E || !st_any) continue;
+              if (cg * 32 >= E || !st_any) continue;
               if (lane == 0) bulk_wait_read<0>();   // both buffers have been read
               __syncwarp();
               stage_f32(bS, lane, ev[c]);
@@ -1094,16 +1136,18 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
               fence_async_smem();
               __syncwarp();
               if (lane == 0) {
-                tma_store_3d(&mO0, smem_u32(bS), c * 32, srow, 0);
-                tma_store_3d(&mO1, smem_u32(bT), srow, c * 32, 0);
+                tma_store_3d(&mO0, smem_u32(bS), cg * 32, srow, 0);
+                tma_store_3d(&mO1, smem_u32(bT), srow, cg * 32, 0);
               }
             }
             // the slot map's rows of this warp's tokens: one contiguous block, -1 throughout
+            // (split between the warps of the lane quarter)
             if (smap && st_any) {
               const int nrow = min(32, T.valid - q * 32);
               int4* blk = reinterpret_cast<int4*>(smap + (int64_t)srow * E);
               const int n4 = nrow * (E >> 2);
-              for (int j = lane; j < n4; j += 32) blk[j] = make_int4(-1, -1, -1, -1);
+              for (int j = lane + part * 32; j < n4; j += 32 * NPART)
+                blk[j] = make_int4(-1, -1, -1, -1);
             }
           } else {
           float* S = reinterpret_cast<float*>(p.out0);
@@ -1302,6 +1346,19 @@ cudaError_t launch(const CUtensorMap& a0, const CUtensorMap& a1, const CUtensorM
   }
   // variable rows: p.M carries an upper bound of the padded rows, so `total` bounds the tiles
   if (PAIR) p.m_tiles = (p.M + 2 * BM - 1) / (2 * BM);
+  if constexpr (VARM == 3) {
+    // one CTA per SM (at most one per 32-row unit), each with the tiles of its row block
+    static_assert(!PAIR, "row split: single-CTA tiles");
+    const int64_t units = (p.M + 31) / 32;
+    if (units == 0 || p.k_blocks == 0) return cudaSuccess;
+    const int g = (int)(units < sm_count() ? units : sm_count());
+    const int64_t max_rows = 32 * ((units + g - 1) / g);
+    p.batch = 1;
+    p.n_tiles = 1;
+    p.m_tiles = g * (int)((max_rows + BM - 1) / BM);
+    kern<<<g, threads, smem, st>>>(a0, a1, b0, b1, o0, o1, o2, p);
+    return cudaGetLastError();
+  }
   const int total = p.batch * p.m_tiles * p.n_tiles;
   if (total == 0 || (VARM != 2 && p.k_blocks == 0)) return cudaSuccess;
   if (PAIR) {
@@ -1359,17 +1416,24 @@ __global__ void wait_probe_kernel(int* status, unsigned long long limit) {
     if (_e != cudaSuccess) return _e;    \
   } while (0)
 
+bool router_needs_pad(int E) { return E % 64 != 0; }
+
 cudaError_t tc_router_softmax(const void* X, const void* Wr, void* Wr_pad, const float* br,
                               float* S, float* ST, int* slot_init, int N, int d, int E,
                               int* status, cudaStream_t st) {
   if (N == 0) return cudaSuccess;
   const int Ep = (E + 63) / 64 * 64;
-  pad_router_weights<<<256, 256, 0, st>>>(static_cast<const bf16*>(Wr), static_cast<bf16*>(Wr_pad),
-                                          d, E, Ep);
-  TC_TRY(cudaGetLastError());
+  // Wr [d][E] already has the padded layout when E is a multiple of 64
+  const void* Wb = Wr;
+  if (router_needs_pad(E)) {
+    pad_router_weights<<<256, 256, 0, st>>>(static_cast<const bf16*>(Wr),
+                                            static_cast<bf16*>(Wr_pad), d, E, Ep);
+    TC_TRY(cudaGetLastError());
+    Wb = Wr_pad;
+  }
   CUtensorMap ma, mb;
   TC_TRY(make_map(&ma, X, d, N, 1, BM));
-  TC_TRY(make_map(&mb, Wr_pad, Ep, d, 1, 64));
+  TC_TRY(make_map(&mb, Wb, Ep, d, 1, 64));
   Args p = base_args(1, N, Ep, d, Ep, status);
   p.out0 = S;
   p.out1 = ST;
@@ -1381,11 +1445,13 @@ cudaError_t tc_router_softmax(const void* X, const void* Wr, void* Wr_pad, const
     CUtensorMap mo0, mo1;
     TC_TRY(make_out_map(&mo0, S, true, E, N, 1));
     TC_TRY(make_out_map(&mo1, ST, true, N, E, 1));
+    // rows split evenly over the SMs; the ring as deep as shared memory allows (the main
+    // loop streams X at the rate its bytes in flight allow), 4 epilogue warps
     if (Ep == 64)
-      return launch<64, false, true, false, false, EPI_ROUTER_ST, 8, 4>(ma, ma, mb, mb, mo0, mo1, ma,
-                                                                         p, st);
-    return launch<128, false, true, false, false, EPI_ROUTER_ST, 6, 4>(ma, ma, mb, mb, mo0, mo1, ma,
-                                                                        p, st);
+      return launch<64, false, true, false, false, EPI_ROUTER_ST, 8, 4, false, 3>(
+          ma, ma, mb, mb, mo0, mo1, ma, p, st);
+    return launch<128, false, true, false, false, EPI_ROUTER_ST, 6, 4, false, 3>(
+        ma, ma, mb, mb, mo0, mo1, ma, p, st);
   }
   switch (Ep) {
     // the router epilogue writes S and S^T itself: the output maps are unused

@@ -26,8 +26,11 @@ struct VarRows {
 
 // Router: Z = X.Wr (+br), S = row softmax over the E experts, written as S [N][E] and
 // S^T [E][N]. X [N][d] bf16, Wr [d][E] bf16. Wr_pad: device scratch of d*round_up(E,64)
-// bf16 (zero-padded copy of Wr made on the stream). slot_init (nullable): an int [N][E]
-// map set to -1 beside S (the expert-choice slot map before selection).
+// bf16 (zero-padded copy of Wr made on the stream when E is not a multiple of 64,
+// router_needs_pad; otherwise Wr itself is read and Wr_pad is untouched). slot_init
+// (nullable): an int [N][E] map set to -1 beside S (the expert-choice slot map before
+// selection).
+bool router_needs_pad(int E);
 cudaError_t tc_router_softmax(const void* X, const void* Wr, void* Wr_pad, const float* br,
                               float* S, float* ST, int* slot_init, int N, int d, int E,
                               int* status, cudaStream_t st);

@@ -21,6 +21,12 @@ cudaError_t launch_topk(const float* ST, int N, int E, int G, const int* group_o
                         const int* k_off, int M, int max_group, int* idx, float* gate, int* slot,
                         cudaStream_t st);
 
+// Capacity update from device memory (one CTA): if 0 <= k_new[g] <= L_g for every group and
+// sum k_new == M, writes k_g [G] and its prefix sums k_off [G+1]; otherwise leaves both and
+// records DEV_BAD_CAPACITY in the status word.
+cudaError_t launch_set_capacity(const int* k_new, const int* group_off, int G, int M, int* k_g,
+                                int* k_off, int* status, cudaStream_t st);
+
 // ---------------------------------------------------------------- token-choice routing
 // Row top-k of S [N][E] (k <= 32, E <= 512), per-expert counts capped at cap (cap < 0:
 // dropless), padded expert regions (tiles[e] in 256-row blocks), row->token map (-1 in

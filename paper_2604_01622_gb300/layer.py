@@ -7,15 +7,13 @@ from __future__ import annotations
 
 import torch
 
-import math
-
 from . import (EC_BF16, EC_F32, ec_check_device, ec_ctx_create, ec_ctx_destroy,
                ec_ctx_profile, ec_ctx_set_capacity, ec_ctx_set_profiling, ec_ctx_set_residual,
                ec_ctx_set_tiles,
                ec_ctx_set_shared, ec_ctx_set_workspace, ec_kernel_launches,
                ec_moe_backward, ec_moe_backward_shared, ec_moe_forward, ec_moe_forward_shared,
-               ec_route, ec_rows_per_expert, ec_tc_backward, ec_tc_ctx_create, ec_tc_forward,
-               ec_workspace_bytes)
+               ec_ctx_set_capacity_async, ec_route, ec_rows_per_expert, ec_tc_backward,
+               ec_tc_capacity, ec_tc_ctx_create, ec_tc_forward, ec_workspace_bytes)
 
 _DT = {"f32": (EC_F32, torch.float32), "bf16": (EC_BF16, torch.bfloat16)}
 
@@ -52,6 +50,10 @@ class ECMoELayer:
 
     def set_capacity(self, k_g):
         ec_ctx_set_capacity(self.ctx, k_g)
+
+    def set_capacity_async(self, k_g_dev, stream=None):
+        """k_g from an int32 device tensor [G] in stream order (sum must keep M)."""
+        ec_ctx_set_capacity_async(self.ctx, k_g_dev.data_ptr(), _stream(stream))
 
     def set_residual(self, on: bool):
         """Y = X + EC(X) and dX = dY + EC input gradient (stacked layers)."""
@@ -146,11 +148,9 @@ class ECMoELayer:
 
 
 def tc_capacity(cf, k, N, E) -> int:
-    """Token-choice expert capacity ceil(CF k N / E) (arXiv 2604.01622, Sec. 2.2); -1 (no cap,
-    dropless) when cf is None or <= 0."""
-    if cf is None or cf <= 0:
-        return -1
-    return int(math.ceil(cf * k * N / E))
+    """Token-choice expert capacity for a capacity factor (computed by the library's
+    ec_tc_capacity); -1 (no cap, dropless) when cf is None or <= 0."""
+    return ec_tc_capacity(cf, k, N, E)
 
 
 class TCMoELayer(ECMoELayer):

@@ -127,3 +127,48 @@ def test_token_choice_host_validation_without_device(lib):
         assert e.value.status == ec.EC_ERR_WORKSPACE
     finally:
         ec.ec_ctx_destroy(ctx)
+
+
+def test_get_last_error_copies_the_message(lib):
+    ctx = ec.ec_ctx_create(256, 64, 8, 128, 2, [0, 128, 256], [16, 16], ec.EC_F32)
+    try:
+        assert ec.ec_get_last_error(ctx) == (ec.EC_OK, "")
+        with pytest.raises(ec.ECError):
+            ec.ec_ctx_set_capacity(ctx, [200, 1])        # k_g above its group's 128 tokens
+        status, msg = ec.ec_get_last_error(ctx)
+        assert status == ec.EC_ERR_SHAPE and msg == ec.ec_last_error(ctx) and "k_g[0]" in msg
+        # truncated to n - 1 bytes plus the terminating NUL; n = 0 writes nothing
+        assert ec.ec_get_last_error(ctx, 6) == (ec.EC_ERR_SHAPE, msg[:5])
+        assert ec.ec_get_last_error(ctx, 0) == (ec.EC_ERR_SHAPE, "")
+        # a NULL buffer with room claimed is an argument error
+        assert lib.ec_get_last_error(ctx, None, 8) == ec.EC_ERR_INVALID_ARG
+    finally:
+        ec.ec_ctx_destroy(ctx)
+    assert lib.ec_get_last_error(None, None, 0) == ec.EC_ERR_INVALID_ARG
+
+
+def test_async_capacity_needs_a_workspace_and_an_aligned_array(lib):
+    ctx = ec.ec_ctx_create(256, 64, 8, 128, 2, [0, 128, 256], [16, 16], ec.EC_F32)
+    try:
+        with pytest.raises(ec.ECError) as e:
+            ec.ec_ctx_set_capacity_async(ctx, 0x1000, None)
+        assert e.value.status == ec.EC_ERR_WORKSPACE
+    finally:
+        ec.ec_ctx_destroy(ctx)
+    ctx = ec.ec_tc_ctx_create(1000, 64, 12, 128, 3, 250, ec.EC_BF16)
+    try:
+        with pytest.raises(ec.ECError):
+            ec.ec_ctx_set_capacity_async(ctx, 0x1000, None)
+    finally:
+        ec.ec_ctx_destroy(ctx)
+
+
+def test_tc_capacity_in_the_library_matches_the_oracle(lib):
+    from oracle import token_choice as T
+    for cf in (0.5, 1.0, 1.25, 1.5, 2.0, 1.0 / 3.0, 7.3):
+        for (k, N, E) in ((8, 32768, 64), (1, 1000, 12), (2, 333, 7), (32, 262144, 256)):
+            assert ec.ec_tc_capacity(cf, k, N, E) == T.tc_capacity(cf, k, N, E)
+    for cf in (None, 0, -1.0, float("nan")):
+        assert ec.ec_tc_capacity(cf, 8, 1024, 64) == -1
+    assert lib.ec_tc_capacity(1.0, 0, 1024, 64) == -2
+    assert lib.ec_tc_capacity(1.0, 8, 1024, 0) == -2
