@@ -296,6 +296,29 @@ def backward_expert(H, S_col, dY_rows, Wg_e, Wu_e, Wd_e):
     return H.T @ dA, H.T @ dB, u.T @ dO, dgate
 
 
+def router_backward_streamed(X, Wr, br, dY, idx, Wg, Wu, Wd):
+    """The router part of `backward` (dS, dZ, dWr, dbr) for a layer too large to hold the
+    per-expert activations: the same definitions, computed one expert at a time.
+
+    X, dY [N][d] float64; idx [E][M] the selection; Wg/Wu/Wd: callables e -> float64
+    matrix of expert e. For every selected pair (e, m), t = idx[e, m]:
+    dS[t, e] = <dY_t, FFN_e(x_t)>; then dZ = S * (dS - <dS, S>_row), dWr = X^T dZ,
+    dbr = sum_t dZ, with S the router scores of X.
+    """
+    X = np.asarray(X, np.float64)
+    dY = np.asarray(dY, np.float64)
+    idx = np.asarray(idx)
+    S = router_scores(X, Wr, br)
+    N, E = S.shape
+    dS = np.zeros((N, E))
+    for e in range(E):
+        rows = idx[e]
+        _, _, _, o = swiglu_ffn(X[rows], Wg(e), Wu(e), Wd(e))
+        dS[rows, e] = np.sum(dY[rows] * o, axis=1)
+    dZ = S * (dS - np.sum(dS * S, axis=1, keepdims=True))
+    return {"S": S, "dS": dS, "dZ": dZ, "dWr": X.T @ dZ, "dbr": dZ.sum(axis=0)}
+
+
 # ----------------------------------------------------------------------------
 # Stacked layers with residual adds, x_{l+1} = x_l + EC_l(x_l): how the four-layer
 # wide workload composes the layer (the transformer residual stream around each MoE
@@ -323,3 +346,34 @@ def stack_backward(fwds, layers, dOut):
         grads[l] = g
         d = d + g["dX"]
     return d, grads
+
+
+def stack_tokens(X_rows, dOut_rows, layers, pairs):
+    """Stack output and input gradient of sampled tokens, one token at a time.
+
+    With each layer's selection fixed, layer l's output for token t depends on x_{l,t} alone
+    (its gate is S[t, e] of that row), so x_{l+1,t} = x_{l,t} + Y_l(x_{l,t}) and
+    d_{l,t} = d_{l+1,t} + (input gradient of layer l at token t, given d_{l+1,t}) follow
+    `forward_tokens` / `backward_tokens` row by row.
+    X_rows, dOut_rows: token -> float64 row; layers: list of (Wr, br, Wg, Wu, Wd) with
+    Wg/Wu/Wd callables e -> float64 matrix; pairs: per layer, token -> [(e, m), ...].
+    Returns (xs, d0): xs[l][t] the input of layer l (xs[-1] the stack output), d0[t].
+    """
+    xs = [dict(X_rows)]
+    for l, (Wr, br, Wg, Wu, Wd) in enumerate(layers):
+        x = xs[-1]
+        toks = list(x)
+        S = router_scores(np.stack([x[t] for t in toks]), Wr, br)
+        srows = {t: S[i] for i, t in enumerate(toks)}
+        y = forward_tokens(x, srows, pairs[l], Wg, Wu, Wd)
+        xs.append({t: x[t] + y[t] for t in toks})
+    d = dict(dOut_rows)
+    for l in range(len(layers) - 1, -1, -1):
+        Wr, br, Wg, Wu, Wd = layers[l]
+        x = xs[l]
+        toks = list(x)
+        S = router_scores(np.stack([x[t] for t in toks]), Wr, br)
+        srows = {t: S[i] for i, t in enumerate(toks)}
+        dx = backward_tokens(x, srows, d, pairs[l], Wr, Wg, Wu, Wd)
+        d = {t: d[t] + dx[t] for t in toks}
+    return xs, d

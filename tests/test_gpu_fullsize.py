@@ -7,8 +7,10 @@ At full size the oracle cannot run the whole layer in float64 in seconds, so:
   * weight gradients are compared on a sampled expert, restricted to a slice of d_ff
     columns (a column slice of the gate/up weights and the matching rows of the down
     weights give exactly that slice of every weight gradient);
-  * dWr and dbr are checked through properties that hold at any size (softmax gradient
-    rows sum to zero), and unpicked tokens must give exact zeros.
+  * dWr and dbr are compared element by element with the oracle's router backward computed
+    one expert at a time over all pairs (the full layer's dS needs every pair's FFN output,
+    seconds of float64 work), besides the properties that hold at any size (softmax
+    gradient rows sum to zero); unpicked tokens must give exact zeros.
 Tolerance: relative max-norm 2e-2 over each sample (bf16 path).
 """
 import numpy as np
@@ -26,7 +28,7 @@ FULL = ["ec_d2048_e64", "ec_timestep_d2048_e64", "ec_many_small_e128", "ec_wide_
 @pytest.mark.parametrize("name", FULL)
 def test_full_size_sampled_parity(name):
     w = I.scaled(I.WORKLOADS[name], layers=1)
-    _check_sampled(I.make_inputs(w))
+    _check_sampled(I.make_inputs(w), full_router=True)
 
 
 def test_large_batch_past_32_bit_offsets():
@@ -46,7 +48,7 @@ def test_large_batch_past_32_bit_offsets():
     _check_sampled(inp, extra_tokens=[w.N - 1, w.N - 4097, (G - 1) * L + 123])
 
 
-def _check_sampled(inp, extra_tokens=()):
+def _check_sampled(inp, extra_tokens=(), full_router=False):
     w = inp.w
     L = inp.layers[0]
     lay, out = gpu_layer(inp)
@@ -106,4 +108,11 @@ def _check_sampled(inp, extra_tokens=()):
     if L.br is not None:
         dbr = host(out["dbr"])
         assert abs(dbr.sum()) <= 1e-3 * np.max(np.abs(dbr)) * w.E
+    # 5. router gradients in full, element by element
+    if full_router:
+        r = O.router_backward_streamed(inp.X.f64(), Wr, L.br, inp.dY.f64(), idx, Wg, Wu, Wd)
+        errs = {"dWr": relmax(dWr, r["dWr"])}
+        if L.br is not None:
+            errs["dbr"] = relmax(host(out["dbr"]), r["dbr"])
+        assert max(errs.values()) <= bound, errs
     lay.close()

@@ -4,6 +4,8 @@ Each case patches one step of the oracle with a plausible slip (a dropped
 term, a wrong sign, a swapped operand, a reversed tie rule) and runs the pin
 that should catch it; the pin must fail.
 """
+import math
+
 import numpy as np
 import pytest
 
@@ -81,3 +83,30 @@ def test_transposed_down_projection_gradient_is_caught(monkeypatch):
 
     monkeypatch.setattr(O, "backward", wrong)
     assert _fails(P.test_backward_matches_central_finite_differences)
+
+
+def _wrong_capacity(rule):
+    import math
+    from oracle import schedulers as SO
+
+    def group_capacity(name, r, k_min, k_max, E, group_off, sigma=0.22):
+        out = []
+        for g in range(len(r)):
+            L = int(group_off[g + 1]) - int(group_off[g])
+            k = SO.k_of_r(name, float(r[g]), k_min, k_max, sigma)
+            out.append(min(max(rule(k, L, E, int(group_off[-1])), 0), L))
+        return np.array(out, dtype=np.int32)
+    return group_capacity
+
+
+@pytest.mark.parametrize("rule", [
+    lambda k, L, E, N: math.floor(k * L + 0.5),          # the / E dropped
+    lambda k, L, E, N: math.floor(k * L / E),            # rounded down, not half up
+    lambda k, L, E, N: math.floor(k * N / E + 0.5),      # the whole batch as the pool
+])
+def test_wrong_group_capacity_is_caught(monkeypatch, rule):
+    from oracle import schedulers as SO
+    from tests import test_schedulers as TS
+    monkeypatch.setattr(SO, "group_capacity", _wrong_capacity(rule))
+    assert (_fails(TS.test_group_capacity_exact_where_no_rounding_is_in_play)
+            or _fails(TS.test_group_capacity_rounding_and_clipping))

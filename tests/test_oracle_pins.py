@@ -274,6 +274,42 @@ def test_sampled_forms_match_full_layer():
         np.testing.assert_allclose(dgate, g["dgate"][e], rtol=1e-11, atol=1e-12)
 
 
+@pytest.mark.parametrize("bias", [True, False])
+def test_streamed_router_backward_matches_full_backward(bias):
+    """The expert-at-a-time form used at full size gives the full backward's dS, dZ, dWr, dbr
+    (which finite differences and autograd pin)."""
+    X, Wr, br, Wg, Wu, Wd, groups, k = _tiny(17, bias=bias)
+    out = O.forward(X, Wr, br, Wg, Wu, Wd, groups, k)
+    dY = np.random.default_rng(18).standard_normal(X.shape)
+    g = O.backward(out, dY, Wr, Wg, Wu, Wd)
+    r = O.router_backward_streamed(X, Wr, br, dY, out["idx"], lambda e: Wg[e], lambda e: Wu[e],
+                                   lambda e: Wd[e])
+    for key in ("dS", "dZ", "dWr", "dbr"):
+        np.testing.assert_allclose(r[key], g[key], rtol=1e-11, atol=1e-13)
+
+
+def test_per_token_stack_matches_full_stack():
+    """Per-token composition through stacked layers equals the full stack on those rows."""
+    X, *_rest, groups, k = _tiny(23, N=40, d=8, E=4, d_ff=6, groups=(0, 17, 40), k=(5, 7))
+    layers = []
+    for l in range(3):
+        _, Wr, br, Wg, Wu, Wd, _, _ = _tiny(40 + l, N=40, d=8, E=4, d_ff=6, groups=(0, 17, 40),
+                                            bias=l != 1)
+        layers.append((Wr, br, Wg, Wu, Wd))
+    dOut = np.random.default_rng(24).standard_normal(X.shape)
+    xs, fwds = O.stack_forward(X, layers, groups, k)
+    d0, _ = O.stack_backward(fwds, layers, dOut)
+    toks = [0, 3, 16, 17, 29, 39]
+    pairs = [O.token_pairs(f["idx"], toks) for f in fwds]
+    fn = [(Wr, br, (lambda e, W=Wg: W[e]), (lambda e, W=Wu: W[e]), (lambda e, W=Wd: W[e]))
+          for (Wr, br, Wg, Wu, Wd) in layers]
+    xt, dt = O.stack_tokens({t: X[t] for t in toks}, {t: dOut[t] for t in toks}, fn, pairs)
+    for t in toks:
+        for l in range(len(layers) + 1):
+            np.testing.assert_allclose(xt[l][t], xs[l][t], rtol=1e-12, atol=1e-13)
+        np.testing.assert_allclose(dt[t], d0[t], rtol=1e-11, atol=1e-12)
+
+
 def test_residual_stack_backward_matches_finite_differences():
     rng = np.random.default_rng(21)
     X, *_rest, groups, k = _tiny(22, N=30, d=6, E=3, d_ff=5, groups=(0, 14, 30), k=(4, 6))
