@@ -136,6 +136,92 @@ class Clocks:
                 "reasons": sorted(reasons), "samples": len(sm)}
 
 
+class NvmlClocks:
+    """SM clock and clock-event reasons read through NVML every few milliseconds, so a timed
+    region of a tenth of a second still gets tens of samples (reads only; nothing is set)."""
+    BITS = {0x4: "sw_power_cap", 0x8: "hw_slowdown", 0x20: "sw_thermal_slowdown",
+            0x40: "hw_thermal_slowdown", 0x80: "hw_power_brake_slowdown"}
+
+    def __init__(self, index, period_s=0.004):
+        import ctypes
+        import threading
+        self.period = period_s
+        self.samples = []
+        self.lib = None
+        self.stop_flag = threading.Event()
+        self.thread = None
+        try:
+            lib = ctypes.CDLL("libnvidia-ml.so.1")
+            if lib.nvmlInit_v2() != 0:
+                return
+            h = ctypes.c_void_p()
+            if lib.nvmlDeviceGetHandleByIndex_v2(ctypes.c_uint(index), ctypes.byref(h)) != 0:
+                return
+            self.h = h
+            self.reasons_fn = getattr(lib, "nvmlDeviceGetCurrentClocksEventReasons", None) or \
+                getattr(lib, "nvmlDeviceGetCurrentClocksThrottleReasons")
+            mx = ctypes.c_uint()
+            self.max_mhz = (float(mx.value) if lib.nvmlDeviceGetMaxClockInfo(h, 1, ctypes.byref(mx)) == 0
+                            else None)
+            self.lib = lib
+        except (OSError, AttributeError):
+            self.lib = None
+
+    def _run(self):
+        import ctypes
+        mhz = ctypes.c_uint()
+        bits = ctypes.c_ulonglong()
+        while not self.stop_flag.is_set():
+            t = time.time()
+            ok = self.lib.nvmlDeviceGetClockInfo(self.h, 1, ctypes.byref(mhz)) == 0   # SM clock
+            ok = ok and self.reasons_fn(self.h, ctypes.byref(bits)) == 0
+            if ok:
+                self.samples.append((t, float(mhz.value), int(bits.value)))
+            time.sleep(self.period)
+
+    def start(self):
+        import threading
+        if self.lib is None:
+            return
+        self.stop_flag.clear()
+        self.thread = threading.Thread(target=self._run, daemon=True)
+        self.thread.start()
+
+    def stop(self):
+        if self.thread is not None:
+            self.stop_flag.set()
+            self.thread.join()
+            self.thread = None
+
+    def summary(self, window):
+        if self.lib is None:
+            return None
+        t0, t1 = window
+        sel = [(m, b) for (t, m, b) in self.samples if t0 <= t <= t1]
+        if not sel:
+            return None
+        mhz = sorted(m for m, _ in sel)
+        reasons = sorted({name for m, b in sel for bit, name in self.BITS.items() if b & bit})
+        return {"sm_mhz": mhz[len(mhz) // 2], "sm_max_mhz": self.max_mhz, "reasons": reasons,
+                "samples": len(sel)}
+
+
+def _clock_record(smi, nvml, window):
+    """nvidia-smi's record of the window (the profiling recipe's query), with NVML's denser
+    samples of the same window taking over the median and adding their reasons."""
+    rec = smi.summary(window)
+    nv = nvml.summary(window) if nvml is not None else None
+    if nv:
+        rec = dict(rec)
+        rec["nvidia_smi_samples"] = rec.get("samples")
+        rec["sm_mhz"] = nv["sm_mhz"]
+        rec["sm_max_mhz"] = nv["sm_max_mhz"] or rec.get("sm_max_mhz")
+        rec["reasons"] = sorted(set(rec.get("reasons", [])) | set(nv["reasons"]))
+        rec["samples"] = nv["samples"]
+        rec["source"] = "NVML every 4 ms (median SM clock, clock-event reasons) + nvidia-smi every 100 ms"
+    return rec
+
+
 # ------------------------------------------------------------------ CPU oracle sample
 class OracleSample:
     """A bounded sample of the workload for the float64 oracle (as it stands): whole
@@ -235,30 +321,62 @@ def _barrier(ws):
 
 
 # ------------------------------------------------------------------ our arm
-def run_ours(args):
+NOMINAL = {"bf16_tflops": 2250.0, "hbm_gbs": 7900.0,
+           "source": "GB300 nominal dense BF16 tensor rate and HBM3e bandwidth"}
+# the other workloads timed beside the headline one (single-GPU runs of the default line)
+EXTRA_WORKLOADS = ("tiny_f32", "ec_timestep_d2048_e64", "ec_many_small_e128",
+                   "ec_wide_d4096_e32_x4")
+
+
+def _mem_bytes(w, P, tc, splits_hint=None):
+    """Algorithmic bytes per launch of the memory-bound kernels (routing, gathers, combine,
+    router backward) of one layer: what each must read and write at least, with the gathers
+    counted token-major ((N + P) d b: each token row read once, P rows written)."""
+    b = 2 if w.dtype == "bf16" else 4
+    N, d, E = w.N, w.d, w.E
+    Ep = (E + 63) // 64 * 64
+    parts = 2 * math.ceil(w.d_ff / 256) if w.dtype == "bf16" else 1
+    fused_rb = E % 4 == 0 and E <= 128 and not tc   # one router-backward kernel
+    dz = 2 * N * Ep * 2 if w.dtype == "bf16" else N * E * 4     # dZ (bf16 hi + lo, or fp32)
+    return {
+        # X, S and S^T; expert choice also sets the slot map [N][E] to -1 there
+        "router_gemm_softmax": N * d * b + 2 * N * E * 4 + (0 if tc else N * E * 4),
+        "topk": N * E * 4 + 3 * P * 4,      # S^T read; idx, gate and the selected slots
+        "tc_route": 2 * N * E * 4 + 3 * P * 4,
+        "gather": (N + P) * d * b,          # token-major: each X row read once, P rows written
+        "combine": P * d * b + N * d * b,
+        "bwd_gather_scale": 3 * P * d * b,
+        "gather_dy": (N + P) * d * b,
+        # slot map and S read, gate-gradient partials read, dZ planes (bf16) or dZ (fp32)
+        "softmax_bwd": (2 * N * E * 4 + parts * P * 4 + dz) if fused_rb else 3 * N * E * 4,
+        "dgate_reduce": (parts + 1) * P * 4,
+        "router_dgrad_gemm": dz + N * d * b,        # dZ read, the router's dX part written
+        "dx_combine": P * d * b + 2 * N * d * b,   # dH rows; the router's dX part; dX
+        "router_wgrad_gemm": N * d * b + dz,       # X and dZ read (split-K partials aside)
+        "router_wgrad_reduce": d * E * 4,          # dWr written
+    }
+
+
+def _timestep_schedule(w, n, seed=12345):
+    """Per-step capacities of a timestep workload: each step draws a new masking ratio per
+    sequence and takes k_g by the workload's FLOPs-matched rule (the sum stays G k_base)."""
+    import numpy as np
+    from paper_2604_01622_gb300 import inputs as I
+    rng = np.random.default_rng(seed)
+    return np.stack([I.timestep_capacity(rng.random(w.G), w.k_base, w.L) for _ in range(n)])
+
+
+def measure(w, args, device, ws, local, headline):
+    """Build one workload's layers on the device and time fwd+bwd steps. Returns a dict of
+    the line's keys for it (the headline also gets the CUDA-graph leg and token coverage)."""
     import numpy as np
     import torch
-    ws, rank, local = _dist()
-    if ws > 1:
-        import torch.distributed as dist
-        dist.init_process_group("nccl", init_method="env://")
-    torch.cuda.set_device(local)
-    device = torch.device("cuda", local)
-
-    from paper_2604_01622_gb300 import build as B
-    if rank == 0 or ws == 1:
-        B.build()
-    _barrier(ws)
     from paper_2604_01622_gb300 import inputs as I
     from paper_2604_01622_gb300.layer import ECMoELayer, TCMoELayer, tc_capacity
-    w = I.WORKLOADS[args.workload]
     tc = args.routing == "tc"
     if tc and args.shared_experts:
         raise SystemExit("--routing tc has no shared experts")
-    if args.seqs:
-        w = I.scaled(w, G=args.seqs)
     inp = I.make_inputs(w)
-    Ld = inp.layers[0]
 
     def to_dev(t):
         if t.dtype == "bf16":
@@ -267,7 +385,8 @@ def run_ours(args):
 
     X, dY = to_dev(inp.X), to_dev(inp.dY)
     stack = []          # one context per layer; several layers stack with residual adds
-    Fs = args.shared_experts * args.shared_dff
+    Fs = args.shared_experts * args.shared_dff if headline else 0
+    tc_cap = None
     for li, Ld in enumerate(inp.layers):
         wts = (to_dev(Ld.Wr), None if Ld.br is None else torch.from_numpy(Ld.br).to(device),
                to_dev(Ld.Wg), to_dev(Ld.Wu), to_dev(Ld.Wd))
@@ -297,16 +416,30 @@ def run_ours(args):
                      dWu_s=torch.empty(w.d, Fs, dtype=torch.float32, device=device),
                      dWd_s=torch.empty(Fs, w.d, dtype=torch.float32, device=device))
         stack.append((lay_l, wts, [torch.empty_like(X)], g, shared))
-    lay, (Wr, br, Wg, Wu, Wd) = stack[0][0], stack[0][1]
+    lay = stack[0][0]
     Y = stack[-1][2][0]
     grads = stack[0][3]
     stream = torch.cuda.current_stream(device)
+    # Timestep workloads (Sec. 4.2): a new capacity per sequence every step, read by the
+    # layers from a device array uploaded once (ec_ctx_set_capacity_async), so the step has
+    # no host copy and no synchronisation for it.
+    dyn = w.timestep_capacity and not tc and not args.static_capacity
+    kg_dev = None
+    if dyn:
+        kg_dev = torch.from_numpy(_timestep_schedule(w, 16).astype(np.int32)).to(device)
+    step_no = [0]
 
     def run_stack(x, dy, y_last, dx_first, st=None):
         """Forward through every layer, then backward in reverse; returns nothing."""
+        kg = None
+        if dyn:
+            kg = kg_dev[step_no[0] % kg_dev.shape[0]]
+            step_no[0] += 1
         h = x
         for i, (l_, wts, ybuf, g, shared) in enumerate(stack):
             out = y_last if i == len(stack) - 1 else ybuf[0]
+            if kg is not None:
+                l_.set_capacity_async(kg, stream=st)
             l_.forward(h, *wts, Y=out, outputs=False, stream=st, shared=shared)
             h = out
         d = dy
@@ -329,8 +462,10 @@ def run_ours(args):
         l_[0].set_profiling(True)
     launches0 = sum(l_[0].launches for l_ in stack)
     clocks = Clocks(local)
+    nvml = NvmlClocks(local)
     clocks.start()
-    time.sleep(0.5)       # let the sampler come up before the timed region
+    nvml.start()
+    time.sleep(0.5)       # let the samplers come up before the timed region
     _barrier(ws)
     torch.cuda.synchronize(device)
     clocks.mark_begin()
@@ -352,31 +487,33 @@ def run_ours(args):
     ms = e0.elapsed_time(e1) / args.steps
     ms_max = _max_over_ranks(ms, ws, device)
 
-    # ---- the same step captured once in a CUDA graph and replayed (no per-kernel events):
-    # the launch-free form of the step
-    side = torch.cuda.Stream(device)
-    side.wait_stream(stream)
-    with torch.cuda.stream(side):
-        step()
-    stream.wait_stream(side)
-    graph = torch.cuda.CUDAGraph()
-    with torch.cuda.graph(graph):
-        step()
-    for _ in range(2):
-        graph.replay()
-    _barrier(ws)
-    torch.cuda.synchronize(device)
-    g0 = torch.cuda.Event(enable_timing=True)
-    g1 = torch.cuda.Event(enable_timing=True)
-    g0.record(stream)
-    for _ in range(args.steps):
-        graph.replay()
-    g1.record(stream)
-    torch.cuda.synchronize(device)
-    graph_ms = _max_over_ranks(g0.elapsed_time(g1) / args.steps, ws, device)
-    for l_ in stack:
-        l_[0].check()
-    del graph
+    graph_ms = None
+    if headline:
+        # ---- the same step captured once in a CUDA graph and replayed (no per-kernel
+        # events): the launch-free form of the step
+        side = torch.cuda.Stream(device)
+        side.wait_stream(stream)
+        with torch.cuda.stream(side):
+            step()
+        stream.wait_stream(side)
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph):
+            step()
+        for _ in range(2):
+            graph.replay()
+        _barrier(ws)
+        torch.cuda.synchronize(device)
+        g0 = torch.cuda.Event(enable_timing=True)
+        g1 = torch.cuda.Event(enable_timing=True)
+        g0.record(stream)
+        for _ in range(args.steps):
+            graph.replay()
+        g1.record(stream)
+        torch.cuda.synchronize(device)
+        graph_ms = _max_over_ranks(g0.elapsed_time(g1) / args.steps, ws, device)
+        for l_ in stack:
+            l_[0].check()
+        del graph
 
     # ---- end to end: every step copies its inputs in from pinned host memory and its
     # results (Y, dX) out, through the public API. Copies run on their own streams with
@@ -401,6 +538,7 @@ def run_ours(args):
     in_ready = [ev() for _ in range(NB)]
     computed = [ev() for _ in range(NB)]
     copied_out = [ev() for _ in range(NB)]
+
     def e2e_pass(n):
         """n pipelined steps; returns ms from the first input copy to the last output copy."""
         _barrier(ws)
@@ -436,15 +574,18 @@ def run_ours(args):
     e2e_t0 = time.time()
     e2e_total = e2e_pass(e_steps)
     e2e_window = (e2e_t0, time.time())
-    clk = clocks.stop(dev_window)
-    clk_e2e = clocks.summary(e2e_window)
+    nvml.stop()
+    clocks.stop(dev_window)
+    clk = _clock_record(clocks, nvml, dev_window)
+    clk_e2e = _clock_record(clocks, nvml, e2e_window)
     e2e_ms = _max_over_ranks(e2e_total / e_steps, ws, device)
     for l_ in stack:
         l_[0].check()
 
     # (after all timed work, so profiler launch counts of the timed steps are unaffected)
-    # expert rows per layer: E x sum(k_g) under expert choice; the kept (token, expert)
-    # pairs under token choice (read once from a forward with outputs)
+    # expert rows per layer: E x sum(k_g) under expert choice (the same every step, also
+    # with per-step capacities, whose sum is fixed); the kept (token, expert) pairs under
+    # token choice (read once from a forward with outputs)
     if tc:
         rows = []
         h = X
@@ -454,16 +595,20 @@ def run_ours(args):
             h = ybuf[0]
     else:
         rows = [w.E * int(inp.k_g.sum())] * w.layers
-    # token coverage of the first layer: tokens no expert picked (expert choice) or
-    # token-expert pairs dropped by the capacity (token choice)
-    if tc:
-        coverage = {"pairs_dropped_frac": round(1.0 - rows[0] / (w.N * args.tc_k), 6)}
-    else:
-        l0, wts0, ybuf0 = stack[0][0], stack[0][1], stack[0][2]
-        idx0 = l0.forward(X, *wts0, Y=ybuf0[0], outputs=True, shared=stack[0][4])[1]
-        picked = np.zeros(w.N, dtype=bool)
-        picked[idx0.cpu().numpy().ravel()] = True
-        coverage = {"tokens_unpicked_frac": round(1.0 - float(picked.mean()), 6)}
+    coverage = None
+    if headline:
+        # token coverage of the first layer: tokens no expert picked (expert choice) or
+        # token-expert pairs dropped by the capacity (token choice)
+        if tc:
+            coverage = {"pairs_dropped_frac": round(1.0 - rows[0] / (w.N * args.tc_k), 6)}
+        else:
+            l0, wts0, ybuf0 = stack[0][0], stack[0][1], stack[0][2]
+            if dyn:
+                l0.set_capacity(inp.k_g)
+            idx0 = l0.forward(X, *wts0, Y=ybuf0[0], outputs=True, shared=stack[0][4])[1]
+            picked = np.zeros(w.N, dtype=bool)
+            picked[idx0.cpu().numpy().ravel()] = True
+            coverage = {"tokens_unpicked_frac": round(1.0 - float(picked.mean()), 6)}
 
     # ---- roofline of the dominant kernel (the tcgen05 grouped GEMM)
     hbm, bf16_burst, bf16_sust, peak_src = _peaks()
@@ -476,33 +621,63 @@ def run_ours(args):
     gemm_ms_step = sum(sum(v) for v in gemm.values()) / args.steps
     P = sum(rows) / len(rows)
     flops_step = 18.0 * sum(rows) * w.d * w.d_ff
-    gemm_tflops = flops_step / (gemm_ms_step * 1e-3) / 1e12
+    gemm_tflops = flops_step / (gemm_ms_step * 1e-3) / 1e12 if gemm_ms_step > 0 else None
     gemm_per_launch = flops_step / max(1, gemm_launches / args.steps)
-    b = 2 if w.dtype == "bf16" else 4
-    N, d, E = w.N, w.d, w.E
-    Ep = (E + 63) // 64 * 64
-    parts = 2 * math.ceil(w.d_ff / 256) if w.dtype == "bf16" else 1
-    fused_rb = E % 4 == 0 and E <= 128 and not tc   # one router-backward kernel
-    mem_bytes = {
-        # X, S and S^T; expert choice also sets the slot map [N][E] to -1 there
-        "router_gemm_softmax": N * d * b + 2 * N * E * 4 + (0 if tc else N * E * 4),
-        "topk": N * E * 4 + 3 * P * 4,      # S^T read; idx, gate and the selected slots
-        "tc_route": 2 * N * E * 4 + 3 * P * 4,
-        "gather": (N + P) * d * b,          # token-major: each X row read once, P rows written
-        "combine": P * d * b + N * d * b,
-        "bwd_gather_scale": 3 * P * d * b,
-        "gather_dy": (N + P) * d * b,
-        # slot map and S read, gate-gradient partials read, dZ planes (bf16) or dZ (fp32)
-        "softmax_bwd": (2 * N * E * 4 + parts * P * 4
-                        + (2 * N * Ep * 2 if w.dtype == "bf16" else N * E * 4)) if fused_rb
-                       else 3 * N * E * 4,
-        "dgate_reduce": (parts + 1) * P * 4,
-        "dx_combine": P * d * b + 2 * N * d * b,   # dH rows; the router's dX part; dX
-    }
-    mem_bytes = {k: v for k, v in mem_bytes.items() if k in per}   # kernels this path launches
-    mem_ms = sum(sum(per[k]) for k in mem_bytes) / args.steps
+    kms = {k: round(sum(v) / args.steps, 4) for k, v in per.items()}
+    mem_bytes = {k: v for k, v in _mem_bytes(w, P, tc).items() if k in per}
+    # from the rounded per-kernel times of the line, so the figure can be recomputed from it
+    mem_ms = sum(kms[k] for k in mem_bytes)
     mem_gbs = (w.layers * sum(mem_bytes.values()) / (mem_ms * 1e-3) / 1e9 if mem_ms > 0
                else None)
+    r = {
+        "ms_per_step": round(ms_max, 4),
+        "value": round(ws * w.N / (ms_max * 1e-3), 1),
+        "e2e": {"value": round(ws * w.N / (e2e_ms * 1e-3), 1), "unit": UNIT,
+                "h2d_bytes_per_step": int(X.numel() * X.element_size() * 2),
+                "d2h_bytes_per_step": int(X.numel() * X.element_size() * 2),
+                "ms_per_step": round(e2e_ms, 4), "steps": e_steps,
+                "sm_mhz": clk_e2e.get("sm_mhz")},
+        "gemm_tflops": gemm_tflops, "gemm_per_launch": gemm_per_launch,
+        "expert_gemm_pct_bf16_peak": (None if gemm_tflops is None
+                                      else round(100 * gemm_tflops / bf16_burst, 2)),
+        "routing_hbm_gbs": None if mem_gbs is None else round(mem_gbs, 1),
+        "routing_hbm_frac": None if mem_gbs is None else round(mem_gbs / hbm, 4),
+        "routing_bytes_per_step": w.layers * sum(mem_bytes.values()),
+        "routing_kernels": sorted(mem_bytes),
+        "gpu_launches": int(launches),
+        "kernel_ms_per_step": kms,
+        "clocks": clk,
+        "graph_ms": graph_ms, "coverage": coverage, "rows": rows, "tc_cap": tc_cap,
+        "shared_ms": shared_ms, "Fs": Fs,
+        "dynamic_capacity": bool(dyn),
+    }
+    for l_ in stack:
+        l_[0].close()
+    return r
+
+
+def run_ours(args):
+    import gc
+    import torch
+    ws, rank, local = _dist()
+    if ws > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", init_method="env://")
+    torch.cuda.set_device(local)
+    device = torch.device("cuda", local)
+
+    from paper_2604_01622_gb300 import build as B
+    if rank == 0 or ws == 1:
+        B.build()
+    _barrier(ws)
+    from paper_2604_01622_gb300 import inputs as I
+    w = I.WORKLOADS[args.workload]
+    tc = args.routing == "tc"
+    if args.seqs:
+        w = I.scaled(w, G=args.seqs)
+    res = measure(w, args, device, ws, local, headline=True)
+    hbm, bf16_burst, bf16_sust, peak_src = _peaks()
+    gemm_tflops = res["gemm_tflops"]
     src = os.path.join(ROOT, "paper_2604_01622_gb300", "csrc", "gemm_tc.cu")
     tr = TRAFFIC.get(_src_hash(src))
     roofline = {
@@ -511,13 +686,15 @@ def run_ours(args):
         "peak": bf16_sust, "unit": "TFLOP/s", "frac": round(gemm_tflops / bf16_sust, 4),
         "peak_kind": f"bf16 sustained, {peak_src}",
         "frac_of_burst": round(gemm_tflops / bf16_burst, 4),
-        "flops_per_launch": gemm_per_launch,
+        "frac_of_nominal": round(gemm_tflops / NOMINAL["bf16_tflops"], 4),
+        "flops_per_launch": res["gemm_per_launch"],
         "traffic": tr,
     }
     out = {
-        "metric": METRIC_TC if tc else METRIC, "value": None, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
-        "warmup": args.warmup, "ms_per_step": round(ms_max, 4), "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
+        "metric": METRIC_TC if tc else METRIC, "value": res["value"], "unit": UNIT, "n_gpus": ws,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": res["ms_per_step"],
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": w.dtype,
+        "data": "synthetic",
         "config": {"workload": w.name, "sequences": w.G, "seq_len": w.L, "tokens": w.N,
                    "d_model": w.d, "experts": w.E, "d_ff": w.d_ff, "k_per_seq": w.k_base,
                    "layers": w.layers, "shared_experts": args.shared_experts,
@@ -525,37 +702,76 @@ def run_ours(args):
                    "parallelism": f"replicas{ws}" if ws > 1 else "single",
                    "l2": "inputs and activations larger than L2 (no flush)"},
     }
+    if res["dynamic_capacity"]:
+        out["config"]["capacity"] = ("per-sequence k_g redrawn every step from a device "
+                                     "array (ec_ctx_set_capacity_async), sum fixed")
     if tc:
-        out["config"].update(routing="token_choice", k=args.tc_k, capacity=tc_cap,
-                             capacity_factor=args.tc_cf, expert_rows=rows)
-    out["value"] = round(ws * w.N / (ms_max * 1e-3), 1)
-    out["expert_gemm_pct_bf16_peak"] = round(100 * gemm_tflops / bf16_burst, 2)
-    out["routing_hbm_gbs"] = None if mem_gbs is None else round(mem_gbs, 1)
-    out["routing_hbm_frac"] = None if mem_gbs is None else round(mem_gbs / hbm, 4)
-    out["e2e"] = {"value": round(ws * w.N / (e2e_ms * 1e-3), 1), "unit": UNIT,
-                  "h2d_bytes_per_step": int(X.numel() * X.element_size() * 2),
-                  "d2h_bytes_per_step": int(X.numel() * X.element_size() * 2),
-                  "ms_per_step": round(e2e_ms, 4), "steps": e_steps,
-                  "sm_mhz": clk_e2e.get("sm_mhz")}
+        out["config"].update(routing="token_choice", k=args.tc_k, capacity=res["tc_cap"],
+                             capacity_factor=args.tc_cf, expert_rows=res["rows"])
+    out["expert_gemm_pct_bf16_peak"] = res["expert_gemm_pct_bf16_peak"]
+    out["routing_hbm_gbs"] = res["routing_hbm_gbs"]
+    out["routing_hbm_frac"] = res["routing_hbm_frac"]
+    out["routing_hbm_frac_of_nominal"] = (None if res["routing_hbm_gbs"] is None else
+                                          round(res["routing_hbm_gbs"] / NOMINAL["hbm_gbs"], 4))
+    out["routing_bytes_per_step"] = res["routing_bytes_per_step"]
+    out["routing_kernels"] = res["routing_kernels"]
+    out["nominal_peaks"] = NOMINAL
+    out["e2e"] = res["e2e"]
     out["roofline"] = roofline
-    if Fs:
-        sh_flops = 18.0 * w.N * w.d * Fs * w.layers
+    if res["Fs"]:
+        sh_flops = 18.0 * w.N * w.d * res["Fs"] * w.layers
         out["shared_experts"] = {"experts": args.shared_experts, "d_ff_each": args.shared_dff,
-                                 "gemm_ms_per_step": round(shared_ms, 4),
-                                 "tflops": round(sh_flops / (shared_ms * 1e-3) / 1e12, 1)}
-    out["graph"] = {"ms_per_step": round(graph_ms, 4),
-                    "value": round(ws * w.N / (graph_ms * 1e-3), 1), "unit": UNIT,
+                                 "gemm_ms_per_step": round(res["shared_ms"], 4),
+                                 "tflops": round(sh_flops / (res["shared_ms"] * 1e-3) / 1e12, 1)}
+    out["graph"] = {"ms_per_step": round(res["graph_ms"], 4),
+                    "value": round(ws * w.N / (res["graph_ms"] * 1e-3), 1), "unit": UNIT,
                     "note": "same step captured in one CUDA graph, replayed; no per-kernel events"}
-    out["coverage"] = coverage
-    out["gpu_launches"] = int(launches)
-    out["kernel_ms_per_step"] = {k: round(sum(v) / args.steps, 4) for k, v in per.items()}
-    out["clocks"] = clk
+    out["coverage"] = res["coverage"]
+    out["gpu_launches"] = res["gpu_launches"]
+    out["kernel_ms_per_step"] = res["kernel_ms_per_step"]
+    out["clocks"] = res["clocks"]
+    # the other workloads, each in the same run (single GPU, default expert-choice line)
+    extra = [] if (ws > 1 or tc or args.shared_experts or args.seqs
+                   or args.workloads == "none") else \
+        [n for n in (EXTRA_WORKLOADS if args.workloads == "all" else args.workloads.split(","))
+         if n != w.name]
+    if extra:
+        out["workloads"] = {}
+    for name in extra:
+        del res
+        gc.collect()
+        torch.cuda.empty_cache()
+        wx = I.WORKLOADS[name]
+        res = measure(wx, args, device, ws, local, headline=False)
+        gt = res["gemm_tflops"]
+        out["workloads"][name] = {
+            "config": {"sequences": wx.G, "seq_len": wx.L, "tokens": wx.N, "d_model": wx.d,
+                       "experts": wx.E, "d_ff": wx.d_ff, "k_per_seq": wx.k_base,
+                       "layers": wx.layers, "dtype": wx.dtype,
+                       "capacity": ("per-sequence, redrawn every step (device array)"
+                                    if res["dynamic_capacity"] else "fixed")},
+            "ms_per_step": res["ms_per_step"], "tokens_per_s": res["value"],
+            "e2e_tokens_per_s": res["e2e"]["value"], "e2e_ms_per_step": res["e2e"]["ms_per_step"],
+            "expert_gemm_tflops": None if gt is None else round(gt, 1),
+            "expert_gemm_frac_of_burst": None if gt is None else round(gt / bf16_burst, 4),
+            "expert_gemm_frac_of_sustained": None if gt is None else round(gt / bf16_sust, 4),
+            "routing_hbm_gbs": res["routing_hbm_gbs"], "routing_hbm_frac": res["routing_hbm_frac"],
+            "gpu_launches": res["gpu_launches"],
+            "kernel_ms_per_step": res["kernel_ms_per_step"],
+            "clocks": res["clocks"],
+        }
     if rank == 0 and not args.no_cpu_baseline:
         smp = (TCOracleSample(args.tc_cpu_tokens, w, args.tc_k, args.tc_cf) if tc
                else OracleSample(args.cpu_tokens, w, args.shared_experts, args.shared_dff))
-        v, dt = smp.run()
-        out["cpu_baseline"] = {"value": round(v, 2), "unit": UNIT, "cores": _cores(),
-                               "kind": "oracle", "sample": smp.desc, "seconds": round(dt, 2)}
+        n, total, t_end = 0, 0.0, time.perf_counter() + args.cpu_seconds
+        while n == 0 or time.perf_counter() < t_end:
+            total += smp.run()[1]
+            n += 1
+        total *= getattr(smp, "layers", 1)   # one of the stack's equal layers was timed
+        out["cpu_baseline"] = {"value": round(n * smp.tokens / total, 2), "unit": UNIT,
+                               "cores": _cores(), "kind": "oracle",
+                               "sample": f"{smp.desc}, run {n} time(s)",
+                               "seconds": round(total, 2)}
     if rank == 0:
         print(json.dumps(out), flush=True)
     if ws > 1:
@@ -572,7 +788,7 @@ def run_reference(args):
     w = I.WORKLOADS[args.workload]
     tc = args.routing == "tc"
     smp = (TCOracleSample(args.tc_cpu_tokens, w, args.tc_k, args.tc_cf) if tc
-           else OracleSample(args.ref_tokens, w, args.shared_experts, args.shared_dff))
+           else OracleSample(args.cpu_tokens, w, args.shared_experts, args.shared_dff))
     for _ in range(args.warmup):
         smp.run()
     total_t = 0.0
@@ -621,10 +837,15 @@ def main():
     ap.add_argument("--tiles", choices=sorted(TILE_POLICY), default="auto",
                     help="expert-GEMM tile policy (bf16 path): auto, 256 or 512 columns")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--cpu-tokens", type=int, default=8192,
-                    help="tokens of the oracle's CPU baseline sample")
-    ap.add_argument("--ref-tokens", type=int, default=128,
-                    help="tokens per step of the reference (oracle) arm")
+    ap.add_argument("--cpu-tokens", type=int, default=4096,
+                    help="tokens of the oracle's sample (whole sequences of the workload): the "
+                         "cpu_baseline leg and every step of the reference arm")
+    ap.add_argument("--cpu-seconds", type=float, default=10.0,
+                    help="the cpu_baseline leg repeats its sample for at least this long")
+    ap.add_argument("--workloads", default="all",
+                    help="other workloads timed in the same run: all, none, or a comma list")
+    ap.add_argument("--static-capacity", action="store_true",
+                    help="timestep workloads keep their first capacities every step")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":
         ap.error("--warmup must be at least 3")

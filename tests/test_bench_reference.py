@@ -17,7 +17,7 @@ def _run(*args):
 
 
 def test_reference_line_keys():
-    d = _run("--workload", "tiny_f32", "--ref-tokens", "64")
+    d = _run("--workload", "tiny_f32", "--cpu-tokens", "64")
     assert d["impl"] == "reference" and d["unit"] == "tokens/s" and d["higher_is_better"]
     assert d["value"] > 0 and d["ms_per_step"] > 0 and d["n_gpus"] == 1
     assert d["config"]["workload"] == "tiny_f32"
@@ -29,8 +29,8 @@ def test_reference_line_keys():
 
 
 def test_reference_counts_shared_experts_and_layers():
-    plain = _run("--workload", "tiny_f32", "--ref-tokens", "64")
-    shared = _run("--workload", "tiny_f32", "--ref-tokens", "64", "--shared-experts", "2",
+    plain = _run("--workload", "tiny_f32", "--cpu-tokens", "64")
+    shared = _run("--workload", "tiny_f32", "--cpu-tokens", "64", "--shared-experts", "2",
                   "--shared-dff", "64")
     assert shared["config"]["shared_experts"] == 2
     assert "2 shared experts of d_ff 64" in shared["cpu_baseline"]["sample"]
