@@ -335,7 +335,7 @@ def _mem_bytes(w, P, tc, splits_hint=None):
     b = 2 if w.dtype == "bf16" else 4
     N, d, E = w.N, w.d, w.E
     Ep = (E + 63) // 64 * 64
-    parts = 2 * math.ceil(w.d_ff / 256) if w.dtype == "bf16" else 1
+    parts = math.ceil(w.d_ff / 256) if w.dtype == "bf16" else 1   # gate-gradient partials
     fused_rb = E % 4 == 0 and E <= 128 and not tc   # one router-backward kernel
     dz = 2 * N * Ep * 2 if w.dtype == "bf16" else N * E * 4     # dZ (bf16 hi + lo, or fp32)
     return {

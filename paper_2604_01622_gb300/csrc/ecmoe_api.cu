@@ -164,8 +164,8 @@ void layout(ec_ctx* c) {
   c->o_dO = take(P * d * es);
   c->o_dA = take(P * F * es);
   c->o_dB = take(P * F * es);
-  // bf16: the dU GEMM's epilogue leaves 2 partial gate gradients per 256-column tile
-  c->dg_parts = use_tc(c) ? 2 * ((c->F + 255) / 256) : 1;
+  // bf16: the dU GEMM's epilogue leaves one partial gate gradient per 256 columns of d_ff
+  c->dg_parts = use_tc(c) ? (c->F + 255) / 256 : 1;
   c->o_dgate = take(c->dg_parts * P * 4);
   c->o_dgsum = use_tc(c) ? take(P * 4) : c->o_dgate;
   c->o_dZ = take(N * E * 4);
@@ -393,7 +393,7 @@ ec_status ffn_backward(ec_ctx* c, const FfnNames& nm, const T* dO, const T* H, c
   if (use_tc(c)) {
     EC_KERNEL(nm.dgrad_up, 1,
               tc_expert_dgrad_up(dO, Wd, A, B, dA, dB, E, M, d, F, status, st, nullptr, gate,
-                                 dgate_part, P));
+                                 dgate_part, P, c->tiles));
     EC_KERNEL(nm.dgrad_h, 1,
               tc_expert_dgrad_h(dA, dB, Wg, Wu, dH, E, M, d, F, status, st, nullptr, c->tiles));
     if (dwd_split && E == 1 && M % 2 == 0 && M >= 2048 &&

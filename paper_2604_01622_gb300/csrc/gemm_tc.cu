@@ -272,16 +272,19 @@ __host__ __device__ constexpr uint32_t tmem_cols() {
 
 // Epilogue staging: one 4 KB buffer per epilogue warp (a 32 x 32 fp32 chunk, or two 32 x 32
 // bf16 chunks), written by the warp and stored to global memory by TMA. The staged router
-// epilogue takes two per warp (a chunk of S and the same chunk of S^T) and keeps the bias
-// row (up to 128 fp32) behind them.
+// epilogue passes a chunk of S and then the same chunk of S^T through it, and keeps the bias
+// row (up to 128 fp32) behind the buffers.
 constexpr uint32_t STAGE_BUF = 4096;
 
 __host__ __device__ constexpr uint32_t stage_bytes(int EPI, int EPW) {
   // staged router: two buffers per warp, the bias row (128 floats) and the per-row partial
   // maxima and sums the two warps of a lane quarter exchange (2 x 2 x 128 floats)
+  // SwiGLU backward: the staging buffers and two [128] float arrays in which the second warp
+  // of a lane quarter leaves its gate-gradient partial for the first
   return EPI == EPI_ROUTER ? 0u
-         : EPI == EPI_ROUTER_ST ? EPW * 2 * STAGE_BUF + 512u + (EPW > 4 ? 2048u : 0u)
-                                : EPW * STAGE_BUF;
+         : EPI == EPI_ROUTER_ST ? EPW * STAGE_BUF + 512u + (EPW > 4 ? 1024u : 0u)
+         : EPI == EPI_SWIGLU_BWD ? EPW * STAGE_BUF + 1024u
+                                 : EPW * STAGE_BUF;
 }
 
 template <int BN, int STAGES, bool PAIR, int EPW, int EPI>
@@ -478,9 +481,8 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
   constexpr uint32_t IDESC = instr_desc<SEGW, A_MN, B_MN, TM>();
   static_assert(BN % 64 == 0 && (BN <= 256 || (WIDE && PAIR)), "BN");
   static_assert(!PAIR || BN % 128 == 0, "pair tiles split B in two 64-column multiples");
-  static_assert(!WIDE || (EPI != EPI_SWIGLU_BWD && EPI != EPI_ROUTER && EPI != EPI_ROUTER_ST &&
-                          STAGES > TAIL),
-                "wide tiles: plain, split-column and SwiGLU forward epilogues");
+  static_assert(!WIDE || (EPI != EPI_ROUTER && EPI != EPI_ROUTER_ST && STAGES > TAIL),
+                "wide tiles: plain, split-column and SwiGLU epilogues");
   static_assert(EPW == 4 || EPW == 8, "epilogue warps: one or two per TMEM lane quarter");
   static_assert(EPI != EPI_ROUTER || EPW == 4, "the plain router keeps whole rows per thread");
   static_assert(EPI != EPI_ROUTER_ST || (BN <= 128 && !PAIR), "staged router: up to 128 experts");
@@ -751,7 +753,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
     int it = 0;
     bool stop = false;
     // staged router: the bias row goes to shared memory once (every row reads all of it)
-    float* s_bias = reinterpret_cast<float*>(sStage + EPW * 2 * STAGE_BUF);
+    float* s_bias = reinterpret_cast<float*>(sStage + EPW * STAGE_BUF);
     if constexpr (EPI == EPI_ROUTER_ST) {
       const int t = (int)threadIdx.x - 64;   // over the epilogue warps
       if (t < 128) s_bias[t] = (p.bias && t < p.n_valid) ? __ldg(p.bias + t) : 0.f;
@@ -847,6 +849,20 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
         }
       };
 
+      // Staged router: the slot map's rows of this warp's tokens are one contiguous block set
+      // to -1 throughout (split between the warps of the lane quarter); it does not depend on
+      // the accumulator, so it is written while the tile's main loop runs.
+      if constexpr (EPI == EPI_ROUTER_ST) {
+        int* smap = reinterpret_cast<int*>(p.out2);
+        if (smap && st_any) {
+          const int E = p.n_valid;
+          const int nrow = min(32, T.valid - q * 32);
+          int4* blk = reinterpret_cast<int4*>(smap + (int64_t)srow * E);
+          const int n4 = nrow * (E >> 2);
+          for (int j = lane + part * 32; j < n4; j += 32 * NPART)
+            blk[j] = make_int4(-1, -1, -1, -1);
+        }
+      }
       // The accumulator segments (one, or a wide tile's two halves, each released as soon
       // as it is drained): segment h holds tile columns [h*SEGW, (h+1)*SEGW).
       for (int h = 0; h < NH; ++h) {
@@ -859,7 +875,91 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
         const int cb = h * SEGW;                   // first tile column of the segment
         constexpr int NC32 = SEGW / 32 / NPART;    // 32-column chunks per warp
         const int c32 = part * NC32;
-        if constexpr (WIDE) {
+        if constexpr (EPI == EPI_SWIGLU_BWD) {
+          // Both tile forms, segment by segment (columns cb.. of the tile). A and B of the next
+          // chunk are requested before the current one is computed (not with variable rows,
+          // whose tile decode leaves too few registers for the second set). The segment goes
+          // back to the MMA issuer as soon as its last chunk has been read from TMEM.
+          constexpr bool PREFETCH = VARM != 1;
+          const bf16* pa = reinterpret_cast<const bf16*>(p.in0) + row_off + nt * BN + cb;
+          const bf16* pb = reinterpret_cast<const bf16*>(p.in1) + row_off + nt * BN + cb;
+          uint4 ra[4], rb[4], na[4], nb[4];
+#pragma unroll
+          for (int i = 0; i < 4; ++i) ra[i] = rb[i] = na[i] = nb[i] = make_uint4(0, 0, 0, 0);
+          auto fetch = [&](int c, uint4* xa, uint4* xb) {
+            const int n = nt * BN + cb + c * 32;
+            if (row_ok && n < p.N) {
+#pragma unroll
+              for (int i = 0; i < 4; ++i) {
+                xa[i] = __ldg(reinterpret_cast<const uint4*>(pa + c * 32) + i);
+                xb[i] = __ldg(reinterpret_cast<const uint4*>(pb + c * 32) + i);
+              }
+            }
+          };
+          if (PREFETCH) fetch(c32, ra, rb);
+          const float gs = (p.gate && row_ok) ? __ldg(p.gate + grow) : 1.0f;
+          // <acc, silu(A) * B> over this warp's columns of the row: even and odd columns
+          uint64_t dot2 = f2(0.f, 0.f);
+#pragma unroll 1
+          for (int c = c32; c < c32 + NC32; ++c) {
+            if (!PREFETCH) fetch(c, ra, rb);
+            else if (c + 1 < c32 + NC32) fetch(c + 1, na, nb);
+            tmem_ld32(tacc + c * 32, v);
+            tmem_wait_ld();
+            if (c == c32 + NC32 - 1) release(a);   // the segment's last TMEM read has completed
+            const int n = nt * BN + cb + c * 32;
+            if (st_any && n < p.N) {
+              float av[32], bv[32];   // av ends up holding dB
+              if (no_k) {
+#pragma unroll
+                for (int i = 0; i < 32; ++i) f[i] = av[i] = 0.f;
+              } else {
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                  unpack16(ra[i], av + 8 * i, bf16());
+                  unpack16(rb[i], bv + 8 * i, bf16());
+                }
+                // two columns at a time: dU = gs acc, sg = sigma(a), dA = dU b sg (1 + a (1 - sg)),
+                // dB = dU a sg, and the gate-gradient terms acc a sg b
+                const uint64_t gs2 = f2(gs, gs), one2 = f2(1.f, 1.f), mone2 = f2(-1.f, -1.f);
+#pragma unroll
+                for (int i = 0; i < 32; i += 2) {
+                  const uint64_t a2 = f2(av[i], av[i + 1]);
+                  const uint64_t b2 = f2(bv[i], bv[i + 1]);
+                  const uint64_t c2 = f2(f32(v[i]), f32(v[i + 1]));
+                  const uint64_t sg2 = f2_sigmoid(a2);
+                  const uint64_t das2 = f2_mul(f2_mul(gs2, c2), sg2);
+                  dot2 = f2_fma(c2, f2_mul(f2_mul(a2, sg2), b2), dot2);
+                  const uint64_t q2 = f2_fma(a2, f2_fma(sg2, mone2, one2), one2);
+                  f2_split(f2_mul(f2_mul(das2, b2), q2), f[i], f[i + 1]);
+                  f2_split(f2_mul(das2, a2), av[i], av[i + 1]);
+                }
+              }
+              put2_bf16(&mO0, &mO1, n, f, av);
+            }
+            if (PREFETCH)
+#pragma unroll
+              for (int i = 0; i < 4; ++i) { ra[i] = na[i]; rb[i] = nb[i]; }
+          }
+          // Partial j of a row covers output columns [256 j, 256 j + 256) (the same partials
+          // for both tile forms): the second warp of the lane quarter leaves its sum in shared
+          // memory and the first adds it to its own (in that order). The two buffers alternate
+          // between segments, so one barrier per segment keeps them apart.
+          if (p.dgate_part) {
+            float de, dd;
+            f2_split(dot2, de, dd);
+            float pd = de + dd;
+            if constexpr (NPART > 1) {
+              float* s_dg = reinterpret_cast<float*>(sStage + EPW * STAGE_BUF) +
+                            (((it * NH + h) & 1) << 7);
+              if (part == 1) s_dg[r] = pd;
+              asm volatile("bar.sync %0, 64;" ::"r"(2 + q) : "memory");
+              pd += s_dg[r];
+            }
+            if (part == 0 && row_ok)
+              p.dgate_part[(int64_t)(nt * NH + h) * p.dgate_stride + grow] = pd;
+          }
+        } else if constexpr (WIDE) {
           // The segment's values go to registers first (packed to bf16 where the output is
           // bf16), the segment is handed back to the MMA issuer, and only then are the chunks
           // staged and stored: the next tile's MMAs wait for the TMEM reads alone.
@@ -995,74 +1095,6 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
               put_bf16(&mO2, n, f);
             }
           }
-        } else if constexpr (EPI == EPI_SWIGLU_BWD) {
-          // A and B of the next chunk are requested before the current one is computed (not
-          // with variable rows, whose tile decode leaves too few registers for the second set)
-          constexpr bool PREFETCH = VARM != 1;
-          const bf16* pa = reinterpret_cast<const bf16*>(p.in0) + row_off + nt * BN;
-          const bf16* pb = reinterpret_cast<const bf16*>(p.in1) + row_off + nt * BN;
-          uint4 ra[4], rb[4], na[4], nb[4];
-#pragma unroll
-          for (int i = 0; i < 4; ++i) ra[i] = rb[i] = na[i] = nb[i] = make_uint4(0, 0, 0, 0);
-          auto fetch = [&](int c, uint4* xa, uint4* xb) {
-            const int n = nt * BN + c * 32;
-            if (row_ok && n < p.N) {
-#pragma unroll
-              for (int i = 0; i < 4; ++i) {
-                xa[i] = __ldg(reinterpret_cast<const uint4*>(pa + c * 32) + i);
-                xb[i] = __ldg(reinterpret_cast<const uint4*>(pb + c * 32) + i);
-              }
-            }
-          };
-          if (PREFETCH) fetch(c32, ra, rb);
-          const float gs = (p.gate && row_ok) ? __ldg(p.gate + grow) : 1.0f;
-          // <acc, silu(A) * B> over this warp's columns of the row: even and odd columns
-          uint64_t dot2 = f2(0.f, 0.f);
-#pragma unroll 1
-          for (int c = c32; c < c32 + NC32; ++c) {
-            if (!PREFETCH) fetch(c, ra, rb);
-            else if (c + 1 < c32 + NC32) fetch(c + 1, na, nb);
-            tmem_ld32(tacc + c * 32, v);
-            tmem_wait_ld();
-            const int n = nt * BN + c * 32;
-            if (st_any && n < p.N) {
-              float av[32], bv[32];   // av ends up holding dB
-              if (no_k) {
-#pragma unroll
-                for (int i = 0; i < 32; ++i) f[i] = av[i] = 0.f;
-              } else {
-#pragma unroll
-                for (int i = 0; i < 4; ++i) {
-                  unpack16(ra[i], av + 8 * i, bf16());
-                  unpack16(rb[i], bv + 8 * i, bf16());
-                }
-                // two columns at a time: dU = gs acc, sg = sigma(a), dA = dU b sg (1 + a (1 - sg)),
-                // dB = dU a sg, and the gate-gradient terms acc a sg b
-                const uint64_t gs2 = f2(gs, gs), one2 = f2(1.f, 1.f), mone2 = f2(-1.f, -1.f);
-#pragma unroll
-                for (int i = 0; i < 32; i += 2) {
-                  const uint64_t a2 = f2(av[i], av[i + 1]);
-                  const uint64_t b2 = f2(bv[i], bv[i + 1]);
-                  const uint64_t c2 = f2(f32(v[i]), f32(v[i + 1]));
-                  const uint64_t sg2 = f2_sigmoid(a2);
-                  const uint64_t das2 = f2_mul(f2_mul(gs2, c2), sg2);
-                  dot2 = f2_fma(c2, f2_mul(f2_mul(a2, sg2), b2), dot2);
-                  const uint64_t q2 = f2_fma(a2, f2_fma(sg2, mone2, one2), one2);
-                  f2_split(f2_mul(f2_mul(das2, b2), q2), f[i], f[i + 1]);
-                  f2_split(f2_mul(das2, a2), av[i], av[i + 1]);
-                }
-              }
-              put2_bf16(&mO0, &mO1, n, f, av);
-            }
-            if (PREFETCH)
-#pragma unroll
-              for (int i = 0; i < 4; ++i) { ra[i] = na[i]; rb[i] = nb[i]; }
-          }
-          if (p.dgate_part && row_ok) {
-            float de, dd;
-            f2_split(dot2, de, dd);
-            p.dgate_part[(int64_t)(nt * NPART + part) * p.dgate_stride + grow] = de + dd;
-          }
         } else if constexpr ((EPI == EPI_ROUTER || EPI == EPI_ROUTER_ST) && BN <= 128) {
           // up to 128 experts the row's logits stay in registers: one TMEM read, exp once;
           // the staged form stores S and S^T as 32 x 32 chunks by TMA, the plain one writes
@@ -1091,63 +1123,63 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
               mx = fmaxf(mx, ev[c][i]);
             }
           }
-          float* s_xmax = s_bias + 128;            // [NPART][128] partial maxima
-          float* s_xsum = s_xmax + 256;            // [NPART][128] partial sums
+          // [NPART][128]: slot `part` first holds this warp's maximum for the partner, then
+          // (written by the partner once it has read that maximum) the partner's sum
+          float* s_x = s_bias + 128;
           if constexpr (NPART > 1) {
-            s_xmax[part * 128 + r] = mx;
+            s_x[part * 128 + r] = mx;
             asm volatile("bar.sync %0, 64;" ::"r"(2 + q) : "memory");
-            mx = fmaxf(mx, s_xmax[(1 - part) * 128 + r]);
+            mx = fmaxf(mx, s_x[(1 - part) * 128 + r]);
           }
-          float sum = 0.f;
+          // exp through the hardware exp2 approximation (relative error ~1e-7, far below the
+          // bf16 inputs' rounding); four independent partial sums, added in a fixed order
+          float ps[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
           for (int c = 0; c < NCH; ++c)
 #pragma unroll
             for (int i = 0; i < 32; ++i) {
-              ev[c][i] = (cb0 + c) * 32 + i < E ? expf(ev[c][i] - mx) : 0.f;
-              sum += ev[c][i];
+              ev[c][i] = (cb0 + c) * 32 + i < E ? __expf(ev[c][i] - mx) : 0.f;
+              ps[i & 3] += ev[c][i];
             }
+          float sum = (ps[0] + ps[1]) + (ps[2] + ps[3]);
           if constexpr (NPART > 1) {
-            s_xsum[part * 128 + r] = sum;
+            s_x[(1 - part) * 128 + r] = sum;       // the partner's maximum was read above
             asm volatile("bar.sync %0, 64;" ::"r"(2 + q) : "memory");
             // the same order in both warps: part 0's sum first
-            sum = part == 0 ? sum + s_xsum[128 + r] : s_xsum[r] + sum;
+            const float os = s_x[part * 128 + r];
+            sum = part == 0 ? sum + os : os + sum;
           }
           const float inv = 1.0f / sum;
           int* smap = reinterpret_cast<int*>(p.out2);
           if constexpr (EPI == EPI_ROUTER_ST) {
-            // chunk c: S rows of this warp's 32 tokens (128-byte swizzle, thread = row) and
-            // the same values as S^T rows of 32 experts (thread = column: each expert's row
-            // of 32 tokens is one 128-byte line of the buffer, so the stores are conflict-free)
-            uint8_t* bS = sStage + (warp - 2) * 2 * STAGE_BUF;
-            uint8_t* bT = bS + STAGE_BUF;
+            // chunk c through the warp's staging buffer: first the S rows of its 32 tokens
+            // (128-byte swizzle, thread = row), then, once that store has read the buffer, the
+            // same values as S^T rows of 32 experts (thread = column: each expert's row of 32
+            // tokens is one 128-byte line of the buffer, so the stores are conflict-free)
+            uint8_t* bS = sStage + (warp - 2) * STAGE_BUF;
 #pragma unroll
             for (int c = 0; c < NCH; ++c) {
               const int cg = cb0 + c;
 #pragma unroll
               for (int i = 0; i < 32; ++i) ev[c][i] *= inv;
               if (cg * 32 >= E || !st_any) continue;
-              if (lane == 0) bulk_wait_read<0>();   // both buffers have been read
+              if (lane == 0) bulk_wait_read<0>();   // the buffer's last store has read it
               __syncwarp();
               stage_f32(bS, lane, ev[c]);
-#pragma unroll
-              for (int i = 0; i < 32; ++i)
-                *reinterpret_cast<float*>(bT + i * 128 + ((((lane >> 2) ^ (i & 7)) << 4) |
-                                                          ((lane & 3) << 2))) = ev[c][i];
               fence_async_smem();
               __syncwarp();
               if (lane == 0) {
                 tma_store_3d(&mO0, smem_u32(bS), cg * 32, srow, 0);
-                tma_store_3d(&mO1, smem_u32(bT), srow, cg * 32, 0);
+                bulk_wait_read<0>();
               }
-            }
-            // the slot map's rows of this warp's tokens: one contiguous block, -1 throughout
-            // (split between the warps of the lane quarter)
-            if (smap && st_any) {
-              const int nrow = min(32, T.valid - q * 32);
-              int4* blk = reinterpret_cast<int4*>(smap + (int64_t)srow * E);
-              const int n4 = nrow * (E >> 2);
-              for (int j = lane + part * 32; j < n4; j += 32 * NPART)
-                blk[j] = make_int4(-1, -1, -1, -1);
+              __syncwarp();
+#pragma unroll
+              for (int i = 0; i < 32; ++i)
+                *reinterpret_cast<float*>(bS + i * 128 + ((((lane >> 2) ^ (i & 7)) << 4) |
+                                                          ((lane & 3) << 2))) = ev[c][i];
+              fence_async_smem();
+              __syncwarp();
+              if (lane == 0) tma_store_3d(&mO1, smem_u32(bS), srow, cg * 32, 0);
             }
           } else {
           float* S = reinterpret_cast<float*>(p.out0);
@@ -1205,7 +1237,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
 #pragma unroll
             for (int i = 0; i < 32; ++i) {
               const int e = c * 32 + i;
-              if (e < E) sum += expf(f32(v[i]) + (p.bias ? p.bias[e] : 0.f) - mx);
+              if (e < E) sum += __expf(f32(v[i]) + (p.bias ? p.bias[e] : 0.f) - mx);
             }
           }
           const float inv = 1.0f / sum;
@@ -1220,7 +1252,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
             for (int i = 0; i < 32; ++i) {
               const int e = c * 32 + i;
               if (e < E && row_ok) {
-                const float pr = expf(f32(v[i]) + (p.bias ? p.bias[e] : 0.f) - mx) * inv;
+                const float pr = __expf(f32(v[i]) + (p.bias ? p.bias[e] : 0.f) - mx) * inv;
                 S[(int64_t)gm * E + e] = pr;
                 ST[(int64_t)e * p.M + gm] = pr;
                 if (slot) slot[(int64_t)gm * E + e] = -1;
@@ -1229,7 +1261,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ 
           }
         }
         // the accumulator is free again: tell the CTA that issues the MMAs
-        if constexpr (!WIDE) release(a);
+        if constexpr (!WIDE && EPI != EPI_SWIGLU_BWD) release(a);
       }   // segments
     }
     // the TMA stores read the staging buffers until they complete
@@ -1445,12 +1477,13 @@ cudaError_t tc_router_softmax(const void* X, const void* Wr, void* Wr_pad, const
     CUtensorMap mo0, mo1;
     TC_TRY(make_out_map(&mo0, S, true, E, N, 1));
     TC_TRY(make_out_map(&mo1, ST, true, N, E, 1));
-    // rows split evenly over the SMs; the ring as deep as shared memory allows (the main
-    // loop streams X at the rate its bytes in flight allow), 4 epilogue warps
+    // rows split evenly over the SMs; a 192 KB ring (the main loop streams X at the rate its
+    // bytes in flight allow); 8 epilogue warps, two per TMEM lane quarter, each taking half of
+    // a row's experts (the epilogue of a CTA's last tile is not hidden behind a main loop)
     if (Ep == 64)
-      return launch<64, false, true, false, false, EPI_ROUTER_ST, 8, 4, false, 3>(
+      return launch<64, false, true, false, false, EPI_ROUTER_ST, 8, 8, false, 3>(
           ma, ma, mb, mb, mo0, mo1, ma, p, st);
-    return launch<128, false, true, false, false, EPI_ROUTER_ST, 6, 4, false, 3>(
+    return launch<128, false, true, false, false, EPI_ROUTER_ST, 6, 8, false, 3>(
         ma, ma, mb, mb, mo0, mo1, ma, p, st);
   }
   switch (Ep) {
@@ -1565,13 +1598,19 @@ cudaError_t tc_expert_down(const void* U, const void* Wd, void* O, int E, int M,
 cudaError_t tc_expert_dgrad_up(const void* dO, const void* Wd, const void* A, const void* B,
                                void* dA, void* dB, int E, int M, int d, int F, int* status,
                                cudaStream_t st, const VarRows* vr, const float* gate,
-                               float* dgate_part, int64_t dgate_stride) {
+                               float* dgate_part, int64_t dgate_stride, int tiles) {
   CUtensorMap ma, mb, oa, ob;
   TC_TRY(act_map(&ma, dO, d, E, M, vr, BM));
   TC_TRY(make_map(&mb, Wd, d, F, E, 128));   // B[n=f][k=i] = Wd[f][i]: K-major, half per CTA
   TC_TRY(act_out_map(&oa, dA, F, E, M, vr));
   TC_TRY(act_out_map(&ob, dB, F, E, M, vr));
-  Args p = row_args(E, M, F, d, 256, status, vr);
+  // 256 x 512 pair tiles only when forced (tile policy 2), for uniform batches: the epilogue
+  // reads A and B per row, and draining an accumulator half that way takes longer than the
+  // few k-slices of MMAs that can cover it (measured on the bench workload: 1.10 ms against
+  // 0.83 ms with 256 x 256 tiles, whose double-buffered accumulators give the epilogue a
+  // whole tile of MMAs)
+  const bool wide = !vr && tiles == 2 && F % 512 == 0;
+  Args p = row_args(E, M, F, d, wide ? 512 : 256, status, vr);
   p.in0 = A;
   p.in1 = B;
   p.out0 = dA;
@@ -1581,6 +1620,9 @@ cudaError_t tc_expert_dgrad_up(const void* dO, const void* Wd, const void* A, co
   p.dgate_stride = dgate_stride;
   p.ld = F;
   p.bstride = (int64_t)M * F;
+  if (wide)
+    return launch<512, false, false, false, false, EPI_SWIGLU_BWD, kWideStages, 8, true, 0>(
+        ma, ma, mb, mb, oa, ob, ob, p, st);
   return launch_rows<256, false, false, false, false, EPI_SWIGLU_BWD>(ma, ma, mb, mb, oa, ob, ob, p,
                                                                       vr, st);
 }

@@ -22,7 +22,9 @@ struct VarRows {
 // Tile shapes of the expert GEMMs (the `tiles` argument below): 0 chooses per GEMM (256 x 512
 // pair tiles where the output columns fill them and the K loop is long enough to hide the
 // hand-over of their two accumulator halves, else 256 x 256), 1 always 256 x 256, 2 wide
-// tiles wherever the columns fill them. The dU GEMM always takes 256 x 256 tiles.
+// tiles wherever the columns fill them. The dU GEMM takes 256 x 512 tiles only under
+// policy 2 (and never with variable rows): its epilogue reads A and B per row and cannot
+// drain an accumulator half within the MMAs that cover it.
 
 // Router: Z = X.Wr (+br), S = row softmax over the E experts, written as S [N][E] and
 // S^T [E][N]. X [N][d] bf16, Wr [d][E] bf16. Wr_pad: device scratch of d*round_up(E,64)
@@ -49,13 +51,13 @@ cudaError_t tc_expert_down(const void* U, const void* Wd, void* O, int E, int M,
 
 // dU' = dO.Wd^T per expert, dU = g dU' (g the row's gate as in tc_expert_up, NULL: 1), then
 // dA = dU * B * silu'(A), dB = dU * silu(A) (bf16 out). With dgate_part, also the row's
-// gate gradient <dU', silu(A) * B> as 2*ceil(F/256) partial sums, partial j of row r at
-// dgate_part[j * dgate_stride + r].
+// gate gradient <dU', silu(A) * B> as ceil(F/256) partial sums (partial j over the columns
+// [256 j, 256 j + 256)), partial j of row r at dgate_part[j * dgate_stride + r].
 cudaError_t tc_expert_dgrad_up(const void* dO, const void* Wd, const void* A, const void* B,
                                void* dA, void* dB, int E, int M, int d, int F, int* status,
                                cudaStream_t st, const VarRows* vr = nullptr,
                                const float* gate = nullptr, float* dgate_part = nullptr,
-                               int64_t dgate_stride = 0);
+                               int64_t dgate_stride = 0, int tiles = 0);
 
 // dH = dA.Wg^T + dB.Wu^T per expert (one K loop over both halves). dH [E][M][d] bf16.
 cudaError_t tc_expert_dgrad_h(const void* dA, const void* dB, const void* Wg, const void* Wu,

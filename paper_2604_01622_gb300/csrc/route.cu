@@ -295,11 +295,165 @@ topk_kernel(const float* __restrict__ ST, int N, int E, const int* __restrict__ 
   }
 }
 
+// The same selection with the column in registers: thread i owns the KPT consecutive scores
+// [i KPT, i KPT + KPT) of the group (groups up to KPT * blockDim.x tokens), so every pass is an
+// unrolled loop over registers (no shared-memory copy of the keys), and the two histogram
+// buffers alternate between passes, so a pass needs two block barriers: one before the bin
+// search and one after it.
+template <int KPT, int NT, int MINB>
+__global__ void __launch_bounds__(NT, MINB)
+topk_reg_kernel(const float* __restrict__ ST, int N, int E, const int* __restrict__ group_off,
+                const int* __restrict__ k_g, const int* __restrict__ k_off, int M,
+                int* __restrict__ idx, float* __restrict__ gate, int* __restrict__ slot) {
+  __shared__ int hist[2][256];
+  __shared__ unsigned long long s_scan[32];
+  __shared__ uint32_t s_mn[32], s_mx[32];
+  __shared__ uint32_t s_prefix[2];
+  __shared__ int s_remaining[2], s_done[2];
+  const int e = blockIdx.x, g = blockIdx.y;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  constexpr int nw = NT / 32;
+  const int lo = group_off[g];
+  const int L = group_off[g + 1] - lo;
+  const int k = k_g[g];
+  const int base = k_off[g];
+  const float* col = ST + (size_t)e * N + lo;
+  const int i0 = tid * KPT;
+  const int nv = max(0, min(KPT, L - i0));        // keys this thread owns
+  uint32_t key[KPT];
+  if (nv == KPT && ((reinterpret_cast<uintptr_t>(col + i0) & 15u) == 0)) {
+#pragma unroll
+    for (int j = 0; j < KPT; j += 4) {
+      const float4 q = *reinterpret_cast<const float4*>(col + i0 + j);
+      key[j] = score_key(q.x); key[j + 1] = score_key(q.y);
+      key[j + 2] = score_key(q.z); key[j + 3] = score_key(q.w);
+    }
+  } else {
+#pragma unroll
+    for (int j = 0; j < KPT; ++j) key[j] = j < nv ? score_key(col[i0 + j]) : 0u;
+  }
+  uint32_t mn = 0xFFFFFFFFu, mx = 0u;
+#pragma unroll
+  for (int j = 0; j < KPT; ++j)
+    if (j < nv) { mn = min(mn, key[j]); mx = max(mx, key[j]); }
+  mn = __reduce_min_sync(0xffffffffu, mn);
+  mx = __reduce_max_sync(0xffffffffu, mx);
+  if (lane == 0) { s_mn[warp] = mn; s_mx[warp] = mx; }
+  for (int i = tid; i < 256; i += NT) hist[0][i] = 0;
+  __syncthreads();
+  mn = __reduce_min_sync(0xffffffffu, lane < nw ? s_mn[lane] : 0xFFFFFFFFu);
+  mx = __reduce_max_sync(0xffffffffu, lane < nw ? s_mx[lane] : 0u);
+  // keys become offsets from the column's smallest key (invalid slots are never read)
+#pragma unroll
+  for (int j = 0; j < KPT; ++j) key[j] -= mn;
+
+  uint32_t T = 0u;
+  int need_eq = 0;
+  if (k > 0) {
+    int hi = mx == mn ? 0 : 32 - __clz(mx - mn);   // every offset lies in [0, 2^hi)
+    uint32_t prefix = 0u, mask = hi == 32 ? 0u : ~((1u << hi) - 1u);
+    int remaining = k;
+    bool done = hi == 0;                           // all keys equal: the first k are taken
+    int b = 0;                                     // histogram buffer of this pass
+    while (!done && hi > 0) {
+      const int shift = max(hi - 8, 0);
+      const uint32_t dmask = (1u << (hi - shift)) - 1u;
+      // the other buffer was last read before the previous pass's second barrier
+      for (int i = tid; i < 256; i += NT) hist[b ^ 1][i] = 0;
+#pragma unroll
+      for (int j = 0; j < KPT; ++j)
+        if (j < nv && (key[j] & mask) == prefix) atomicAdd(&hist[b][(key[j] >> shift) & dmask], 1);
+      __syncthreads();
+      if (warp == 0) {
+        int c[8], local = 0;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) { c[j] = hist[b][255 - (lane * 8 + j)]; local += c[j]; }
+        int incl = local;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const int u = __shfl_up_sync(0xffffffffu, incl, o);
+          if (lane >= o) incl += u;
+        }
+        const int excl = incl - local;
+        if (excl < remaining && remaining <= incl) {
+          int run = excl;
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            if (run + c[j] >= remaining) {
+              const uint32_t bin = 255u - (uint32_t)(lane * 8 + j);
+              s_prefix[b] = prefix | (bin << shift);
+              s_remaining[b] = remaining - run;
+              s_done[b] = run + c[j] == remaining;   // the whole bin is taken
+              break;
+            }
+            run += c[j];
+          }
+        }
+      }
+      __syncthreads();
+      prefix = s_prefix[b];
+      remaining = s_remaining[b];
+      done = s_done[b];
+      mask |= dmask << shift;
+      hi = shift;
+      b ^= 1;
+    }
+    T = prefix;
+    need_eq = (done && hi > 0) ? 0x7FFFFFFF : remaining;
+  }
+  // compaction in token order: this thread's keys follow those of lower threads
+  uint32_t n_gt = 0, n_eq = 0;
+  if (k > 0)
+#pragma unroll
+    for (int j = 0; j < KPT; ++j)
+      if (j < nv) { n_gt += key[j] > T; n_eq += key[j] == T; }
+  const unsigned long long before =
+      block_excl_scan2(((unsigned long long)n_gt << 32) | n_eq, s_scan);
+  if (k == 0) return;
+  int r = (int)(before & 0xFFFFFFFFu);                 // keys equal to T before this one
+  int pos = (int)(before >> 32) + min(r, need_eq);     // selected keys before this one
+  int* idx_row = idx + (size_t)e * M + base;
+  float* gate_row = gate + (size_t)e * M + base;
+#pragma unroll
+  for (int j = 0; j < KPT; ++j) {
+    if (j >= nv) break;
+    const bool eq = key[j] == T;
+    const bool sel = key[j] > T || (eq && r < need_eq);
+    r += eq;
+    if (sel) {
+      const int t = lo + i0 + j;
+      const uint32_t kk = key[j] + mn;
+      // the gate is the score the key encodes (-0.0 and +0.0 share a key: read it back)
+      const float sv = kk == 0x80000000u
+                           ? col[i0 + j]
+                           : __uint_as_float((kk & 0x80000000u) ? (kk & 0x7FFFFFFFu) : ~kk);
+      idx_row[pos] = t;
+      gate_row[pos] = sv;
+      slot[(size_t)t * E + e] = base + pos;
+      ++pos;
+    }
+  }
+}
+
 cudaError_t launch_topk(const float* ST, int N, int E, int G, const int* group_off, const int* k_g,
                         const int* k_off, int M, int max_group, int* idx, float* gate, int* slot,
                         cudaStream_t st) {
   if (G == 0 || E == 0) return cudaSuccess;
   dim3 grid(E, G);
+  // columns up to 8192 scores: in registers, 16 per thread (128 threads for up to 2048, so
+  // that every column of a 16-sequence batch is resident at once; 256 up to 4096; 512)
+  if (max_group <= 8192) {
+    if (max_group <= 2048)
+      topk_reg_kernel<16, 128, 8><<<grid, 128, 0, st>>>(ST, N, E, group_off, k_g, k_off, M, idx,
+                                                        gate, slot);
+    else if (max_group <= 4096)
+      topk_reg_kernel<16, 256, 4><<<grid, 256, 0, st>>>(ST, N, E, group_off, k_g, k_off, M, idx,
+                                                        gate, slot);
+    else
+      topk_reg_kernel<16, 512, 2><<<grid, 512, 0, st>>>(ST, N, E, group_off, k_g, k_off, M, idx,
+                                                        gate, slot);
+    return cudaGetLastError();
+  }
   // measured per column (phase timestamps, 512 columns of 4096 and 2048 columns of 2048
   // scores): 256 threads beat 512 on 4096-score columns (13.0 vs 14.2 us for the launch), and
   // 128 threads let every column of 2048 scores be resident at once (19.8 vs 22.1 us)

@@ -241,6 +241,22 @@ def test_bf16_tile_policies_agree_bit_for_bit():
         assert torch.equal(a[k], b[k]), k
 
 
+def test_bf16_wide_dgrad_up_tiles_match_oracle_and_narrow_tiles():
+    """d_ff = 512: the dU GEMM (SwiGLU backward and gate-gradient partials in its epilogue)
+    takes 256 x 512 tiles too; M = 2 * 75 rows leaves a ragged row tile and d = 256 a K loop
+    of 4 k-slices. The partials cover the same column blocks in both tile forms, so the
+    results equal the 256 x 256 ones bit for bit."""
+    from paper_2604_01622_gb300 import EC_TILES_256, EC_TILES_512
+    w = I.scaled(I.WORKLOADS["ec_d2048_e64"], G=2, L=200, d=256, E=5, d_ff=512, k_base=75,
+                 seed=23, router_bias=True, layers=1)
+    inp = I.make_inputs(w)
+    _check_layer(inp, tiles=EC_TILES_512)
+    _, a = gpu_layer(inp, tiles=EC_TILES_256)
+    _, b = gpu_layer(inp, tiles=EC_TILES_512)
+    for k in ("Y", "dX", "dWr", "dbr", "dWg", "dWu", "dWd"):
+        assert torch.equal(a[k], b[k]), k
+
+
 @pytest.mark.parametrize("E", [160, 256])
 def test_bf16_many_experts_router_widths(E):
     """160 and 256 experts take the router GEMM's 192- and 256-column tiles (softmax over
