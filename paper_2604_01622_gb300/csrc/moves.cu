@@ -6,6 +6,8 @@
 // over experts in ascending order with no atomics, so results are deterministic.
 #include <algorithm>
 
+#include <type_traits>
+
 #include "common.cuh"
 #include "kernels.h"
 
@@ -485,23 +487,61 @@ cudaError_t launch_router_softmax_bwd(const float* S, const int* slot, const flo
 }
 
 // out[i][e] = sum_s part[s][i][e] for the first `cols` of `ld` columns.
+// Each output is the sum of its `splits` partials in split order; the partials of a batch of
+// eight splits are loaded before any of them is added, so eight loads are in flight per thread
+// (one at a time made the kernel wait on each load in turn). V = 4: four adjacent columns per
+// thread with 16-byte loads (cols and ld multiples of 4).
+template <int V>
 __global__ void reduce_partials_kernel(const float* __restrict__ part, float* __restrict__ out,
                                        int rows, int cols, int ld, int splits) {
-  const int64_t n = (int64_t)rows * cols;
+  typedef typename std::conditional<V == 4, float4, float>::type vec;
+  const int cv = cols / V;
+  const int64_t n = (int64_t)rows * cv;
+  const int64_t plane = (int64_t)rows * ld;
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
        i += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t r = i / cols, c = i % cols;
-    float s = 0.f;
-    for (int k = 0; k < splits; ++k) s += part[((int64_t)k * rows + r) * ld + c];
-    out[i] = s;
+    const int64_t r = i / cv, c = (i % cv) * V;
+    const float* src = part + r * ld + c;
+    float s[V];
+#pragma unroll
+    for (int j = 0; j < V; ++j) s[j] = 0.f;
+    int k = 0;
+    for (; k + 8 <= splits; k += 8) {
+      vec x[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) x[u] = *reinterpret_cast<const vec*>(src + (k + u) * plane);
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const float* xf = reinterpret_cast<const float*>(&x[u]);
+#pragma unroll
+        for (int j = 0; j < V; ++j) s[j] += xf[j];
+      }
+    }
+    for (; k < splits; ++k) {
+      const vec x = *reinterpret_cast<const vec*>(src + k * plane);
+      const float* xf = reinterpret_cast<const float*>(&x);
+#pragma unroll
+      for (int j = 0; j < V; ++j) s[j] += xf[j];
+    }
+    float* dst = out + r * cols + c;
+    if constexpr (V == 4) *reinterpret_cast<float4*>(dst) = make_float4(s[0], s[1], s[2], s[3]);
+    else dst[0] = s[0];
   }
 }
 
 cudaError_t launch_reduce_partials(const float* part, float* out, int rows, int cols, int ld,
                                    int splits, cudaStream_t st) {
   if (rows == 0 || cols == 0) return cudaSuccess;
-  reduce_partials_kernel<<<grid_for((int64_t)rows * cols, 152 * 16), 256, 0, st>>>(
-      part, out, rows, cols, ld, splits);
+  const bool v4 = cols % 4 == 0 && ld % 4 == 0 &&
+                  (reinterpret_cast<uintptr_t>(part) & 15u) == 0 &&
+                  (reinterpret_cast<uintptr_t>(out) & 15u) == 0;
+  const int64_t n = (int64_t)rows * cols / (v4 ? 4 : 1);
+  if (v4)
+    reduce_partials_kernel<4><<<grid_for(n, 152 * 16), 256, 0, st>>>(part, out, rows, cols, ld,
+                                                                       splits);
+  else
+    reduce_partials_kernel<1><<<grid_for(n, 152 * 16), 256, 0, st>>>(part, out, rows, cols, ld,
+                                                                       splits);
   return cudaGetLastError();
 }
 
@@ -701,8 +741,17 @@ __global__ void reduce_splits_kernel(const float* __restrict__ part, float* __re
                                      int64_t n, int splits) {
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
        i += (int64_t)gridDim.x * blockDim.x) {
+    // split order, eight loads in flight before they are added
     float s = 0.f;
-    for (int k = 0; k < splits; ++k) s += part[(size_t)k * n + i];
+    int k = 0;
+    for (; k + 8 <= splits; k += 8) {
+      float x[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) x[u] = part[(size_t)(k + u) * n + i];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) s += x[u];
+    }
+    for (; k < splits; ++k) s += part[(size_t)k * n + i];
     out[i] = s;
   }
 }
