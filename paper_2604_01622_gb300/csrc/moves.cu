@@ -488,9 +488,9 @@ cudaError_t launch_router_softmax_bwd(const float* S, const int* slot, const flo
 
 // out[i][e] = sum_s part[s][i][e] for the first `cols` of `ld` columns.
 // Each output is the sum of its `splits` partials in split order; the partials of a batch of
-// eight splits are loaded before any of them is added, so eight loads are in flight per thread
-// (one at a time made the kernel wait on each load in turn). V = 4: four adjacent columns per
-// thread with 16-byte loads (cols and ld multiples of 4).
+// sixteen splits are loaded before any of them is added, so sixteen loads are in flight per
+// thread (the outputs are few: 2048 x 64 for the router's dWr, 128 CTAs of 256 threads). V = 4:
+// four adjacent columns per thread with 16-byte loads (cols and ld multiples of 4).
 template <int V>
 __global__ void reduce_partials_kernel(const float* __restrict__ part, float* __restrict__ out,
                                        int rows, int cols, int ld, int splits) {
@@ -506,12 +506,12 @@ __global__ void reduce_partials_kernel(const float* __restrict__ part, float* __
 #pragma unroll
     for (int j = 0; j < V; ++j) s[j] = 0.f;
     int k = 0;
-    for (; k + 8 <= splits; k += 8) {
-      vec x[8];
+    for (; k + 16 <= splits; k += 16) {
+      vec x[16];
 #pragma unroll
-      for (int u = 0; u < 8; ++u) x[u] = *reinterpret_cast<const vec*>(src + (k + u) * plane);
+      for (int u = 0; u < 16; ++u) x[u] = *reinterpret_cast<const vec*>(src + (k + u) * plane);
 #pragma unroll
-      for (int u = 0; u < 8; ++u) {
+      for (int u = 0; u < 16; ++u) {
         const float* xf = reinterpret_cast<const float*>(&x[u]);
 #pragma unroll
         for (int j = 0; j < V; ++j) s[j] += xf[j];
