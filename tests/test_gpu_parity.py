@@ -257,6 +257,17 @@ def test_bf16_wide_dgrad_up_tiles_match_oracle_and_narrow_tiles():
         assert torch.equal(a[k], b[k]), k
 
 
+@pytest.mark.parametrize("G,L,E", [(3, 1700, 16), (1, 4868, 64), (2, 2050, 128)])
+def test_bf16_router_row_split_uneven(G, L, E):
+    """The router splits the tokens over the SMs in 32-row units: 160, 153 and 129 units
+    here over at most 152 CTAs, so some CTAs take one unit more than others, tiles of 32 to
+    128 rows occur, and the last unit is ragged (none of 5100, 4868, 4100 is a multiple of
+    32)."""
+    w = I.scaled(I.WORKLOADS["ec_many_small_e128"], G=G, L=L, d=128, E=E, d_ff=64,
+                 k_base=max(1, L // 8), seed=29, router_bias=True, layers=1)
+    _check_layer(I.make_inputs(w))
+
+
 @pytest.mark.parametrize("E", [160, 256])
 def test_bf16_many_experts_router_widths(E):
     """160 and 256 experts take the router GEMM's 192- and 256-column tiles (softmax over
