@@ -96,6 +96,91 @@ __global__ void tc_topk_rows_kernel(const float* __restrict__ S, int N, int E, i
   if (lane == 0) Z[t] = sum;
 }
 
+// The same selection for up to 64 experts (E a multiple of 4) and k <= 8, four threads per
+// token: thread j of the token holds scores 16 j .. 16 j + 15 and keeps its k best in a sorted
+// register list of packed words (order-preserving key above, 255 - expert below, so equal
+// scores order by lower expert index); k rounds take the largest head of the four lists. The
+// choices, gates (normalised by the sum taken in choice order) and Z match the warp-per-token
+// kernel exactly. The token's row of the slot map is set to -1 here as well.
+constexpr int kTopkFastE = 64, kTopkFastK = 8;
+
+__global__ void __launch_bounds__(256)
+tc_topk_rows4_kernel(const float* __restrict__ S, int N, int E, int k, int* __restrict__ choice,
+                     float* __restrict__ tgate, float* __restrict__ Z, int* __restrict__ slot) {
+  const int64_t gt = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const int t = (int)(gt >> 2), j = threadIdx.x & 3;
+  const bool ok = t < N;                  // the token's four threads agree
+  const int e0 = j * 16;
+  const int ne = ok ? max(0, min(16, E - e0)) : 0;
+  const float* row = S + (size_t)(ok ? t : 0) * E + e0;
+  float val[16];
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    float4 x = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (4 * q < ne) x = reinterpret_cast<const float4*>(row)[q];
+    val[4 * q] = x.x; val[4 * q + 1] = x.y; val[4 * q + 2] = x.z; val[4 * q + 3] = x.w;
+  }
+  if (ok) {
+    int4* sl = reinterpret_cast<int4*>(slot + (size_t)t * E + e0);
+#pragma unroll
+    for (int q = 0; q < 4; ++q)
+      if (4 * q < ne) sl[q] = make_int4(-1, -1, -1, -1);
+  }
+  // this thread's best k, descending; 0 is below every packed score
+  unsigned long long lst[kTopkFastK];
+  float lv[kTopkFastK];
+#pragma unroll
+  for (int i = 0; i < kTopkFastK; ++i) { lst[i] = 0ull; lv[i] = 0.f; }
+#pragma unroll
+  for (int q = 0; q < 16; ++q) {
+    if (q >= ne) break;
+    unsigned long long x = ((unsigned long long)score_key(val[q]) << 32) |
+                           (unsigned long long)(255 - (e0 + q));
+    float xv = val[q];
+#pragma unroll
+    for (int i = 0; i < kTopkFastK; ++i) {
+      if (x > lst[i]) {
+        const unsigned long long tx = lst[i];
+        const float tv = lv[i];
+        lst[i] = x; lv[i] = xv;
+        x = tx; xv = tv;
+      }
+    }
+  }
+  int my_e[2] = {0, 0};
+  float my_v[2] = {0.f, 0.f};
+  float sum = 0.f;
+  for (int r = 0; r < k; ++r) {
+    unsigned long long m = lst[0];
+    m = max(m, __shfl_xor_sync(0xffffffffu, m, 1));
+    m = max(m, __shfl_xor_sync(0xffffffffu, m, 2));
+    const bool mine = lst[0] == m;                  // exactly one thread of the token
+    float v = mine ? lv[0] : 0.f;
+    v += __shfl_xor_sync(0xffffffffu, v, 1);
+    v += __shfl_xor_sync(0xffffffffu, v, 2);
+    if (mine) {
+#pragma unroll
+      for (int i = 0; i + 1 < kTopkFastK; ++i) { lst[i] = lst[i + 1]; lv[i] = lv[i + 1]; }
+      lst[kTopkFastK - 1] = 0ull;
+    }
+    if ((r & 3) == j) {
+      my_e[r >> 2] = 255 - (int)(uint32_t)(m & 0xFFFFFFFFull);
+      my_v[r >> 2] = v;
+    }
+    sum += v;
+  }
+  if (!ok) return;
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    const int r = 4 * h + j;
+    if (r < k) {
+      choice[(size_t)t * k + r] = my_e[h];
+      tgate[(size_t)t * k + r] = my_v[h] / sum;
+    }
+  }
+  if (j == 0) Z[t] = sum;
+}
+
 // The position of token t in expert e's list is the number of tokens before t that chose
 // e: an exclusive scan, in token order, of the 0/1 column "chose e". It is done in three
 // levels: warp ballots within each 256-token block, warps within the block, blocks.
@@ -244,9 +329,15 @@ cudaError_t launch_tc_route(const float* S, int N, int E, int k, int cap, int* c
   int* hist = scratch;                          // [nblk][E]
   int* boff = scratch + (size_t)nblk * E;       // [nblk][E]
   int* total = boff + (size_t)nblk * E;         // [E]
-  cudaError_t err = cudaMemsetAsync(slot, 0xFF, (size_t)N * E * sizeof(int), st);   // -1
-  if (err != cudaSuccess) return err;
-  tc_topk_rows_kernel<<<(N + 7) / 8, 256, 0, st>>>(S, N, E, k, choice, tgate, Z);
+  if (E % 4 == 0 && E <= kTopkFastE && k <= kTopkFastK) {
+    // four threads per token; the slot map's -1 rows are written there too
+    tc_topk_rows4_kernel<<<(unsigned)(((int64_t)N * 4 + 255) / 256), 256, 0, st>>>(
+        S, N, E, k, choice, tgate, Z, slot);
+  } else {
+    cudaError_t err = cudaMemsetAsync(slot, 0xFF, (size_t)N * E * sizeof(int), st);   // -1
+    if (err != cudaSuccess) return err;
+    tc_topk_rows_kernel<<<(N + 7) / 8, 256, 0, st>>>(S, N, E, k, choice, tgate, Z);
+  }
   tc_rank_kernel<<<nblk, kRankBlock, 0, st>>>(choice, N, E, k, slot, hist);
   tc_block_scan_kernel<<<E, 256, 0, st>>>(hist, nblk, E, boff, total);
   tc_offsets_kernel<<<1, kMaxE, 0, st>>>(E, cap, total, count, tiles);
