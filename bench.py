@@ -330,30 +330,33 @@ EXTRA_WORKLOADS = ("tiny_f32", "ec_timestep_d2048_e64", "ec_many_small_e128",
                    "ec_wide_d4096_e32_x4")
 
 
-def _mem_bytes(w, P, tc, splits_hint=None):
+def _mem_bytes(w, P, tc, shared=False, splits_hint=None):
     """Algorithmic bytes per launch of the memory-bound kernels (routing, gathers, combine,
     router backward) of one layer: what each must read and write at least, with the gathers
-    counted token-major ((N + P) d b: each token row read once, P rows written)."""
+    counted token-major ((N + P) d b: each token row read once, P rows written). In a stack
+    (residual adds) the combine also reads X and the dX scatter the incoming gradient; with
+    shared experts they also read the shared FFN's output and its input gradient."""
     b = 2 if w.dtype == "bf16" else 4
     N, d, E = w.N, w.d, w.E
     Ep = (E + 63) // 64 * 64
     parts = math.ceil(w.d_ff / 256) if w.dtype == "bf16" else 1   # gate-gradient partials
     fused_rb = E % 4 == 0 and E <= 128 and not tc   # one router-backward kernel
     dz = 2 * N * Ep * 2 if w.dtype == "bf16" else N * E * 4     # dZ (bf16 hi + lo, or fp32)
+    extra = ((1 if w.layers > 1 else 0) + (1 if shared else 0)) * N * d * b
     return {
         # X, S and S^T; expert choice also sets the slot map [N][E] to -1 there
         "router_gemm_softmax": N * d * b + 2 * N * E * 4 + (0 if tc else N * E * 4),
         "topk": N * E * 4 + 3 * P * 4,      # S^T read; idx, gate and the selected slots
         "tc_route": 2 * N * E * 4 + 3 * P * 4,
         "gather": (N + P) * d * b,          # token-major: each X row read once, P rows written
-        "combine": P * d * b + N * d * b,
+        "combine": P * d * b + N * d * b + extra,
         "bwd_gather_scale": 3 * P * d * b,
         "gather_dy": (N + P) * d * b,
         # slot map and S read, gate-gradient partials read, dZ planes (bf16) or dZ (fp32)
         "softmax_bwd": (2 * N * E * 4 + parts * P * 4 + dz) if fused_rb else 3 * N * E * 4,
         "dgate_reduce": (parts + 1) * P * 4,
         "router_dgrad_gemm": dz + N * d * b,        # dZ read, the router's dX part written
-        "dx_combine": P * d * b + 2 * N * d * b,   # dH rows; the router's dX part; dX
+        "dx_combine": P * d * b + 2 * N * d * b + extra,   # dH rows; router's dX part; dX
         "router_wgrad_gemm": N * d * b + dz,       # X and dZ read (split-K partials aside)
         "router_wgrad_reduce": d * E * 4,          # dWr written
     }
@@ -626,7 +629,7 @@ def measure(w, args, device, ws, local, headline):
     gemm_tflops = flops_step / (gemm_ms_step * 1e-3) / 1e12 if gemm_ms_step > 0 else None
     gemm_per_launch = flops_step / max(1, gemm_launches / args.steps)
     kms = {k: round(sum(v) / args.steps, 4) for k, v in per.items()}
-    mem_bytes = {k: v for k, v in _mem_bytes(w, P, tc).items() if k in per}
+    mem_bytes = {k: v for k, v in _mem_bytes(w, P, tc, shared=Fs > 0).items() if k in per}
     # from the rounded per-kernel times of the line, so the figure can be recomputed from it
     mem_ms = sum(kms[k] for k in mem_bytes)
     mem_gbs = (w.layers * sum(mem_bytes.values()) / (mem_ms * 1e-3) / 1e9 if mem_ms > 0
