@@ -362,6 +362,36 @@ def _mem_bytes(w, P, tc, shared=False, splits_hint=None):
     }
 
 
+def _gemm_rooflines(w, P, kms, hbm, burst):
+    """Each expert-GEMM phase against its own roofline: FLOPs and algorithmic DRAM bytes per
+    step (operands, weights and outputs once each; fp32 weight gradients), their ratio, the
+    attainable rate min(burst peak, ratio x copy bandwidth) and the fraction of it reached.
+    Only for the tensor-core (bf16) path."""
+    if w.dtype != "bf16":
+        return None
+    b, d, F, E, L = 2, w.d, w.d_ff, w.E, w.layers
+    work = {   # phase: (FLOP, bytes) per layer
+        "gemm_gate_up_swiglu": (4 * P * d * F, P * d * b + 2 * E * d * F * b + 3 * P * F * b),
+        "gemm_down": (2 * P * d * F, P * F * b + E * F * d * b + P * d * b),
+        "gemm_dgrad_up_swiglu": (2 * P * d * F, P * d * b + E * F * d * b + 4 * P * F * b),
+        "gemm_dgrad_h": (4 * P * d * F, 2 * P * F * b + 2 * E * d * F * b + P * d * b),
+        "gemm_wgrad": (6 * P * d * F, (P * d * b + 2 * P * F * b + 2 * E * d * F * 4)
+                       + (P * F * b + P * d * b + E * F * d * 4)),
+    }
+    out = {}
+    for k, (fl, by) in work.items():
+        ms = kms.get(k)
+        if not ms:
+            continue
+        fl, by = fl * L, by * L
+        att = min(burst, fl / by * hbm / 1e3)   # TFLOP/s (hbm in GB/s)
+        ach = fl / (ms * 1e-3) / 1e12
+        out[k] = {"ms": ms, "tflops": round(ach, 1), "gbytes": round(by / 1e9, 3),
+                  "flop_per_byte": round(fl / by, 1), "attainable_tflops": round(att, 1),
+                  "frac_of_attainable": round(ach / att, 3)}
+    return out
+
+
 def _timestep_schedule(w, n, seed=12345):
     """Per-step capacities of a timestep workload: each step draws a new masking ratio per
     sequence and takes k_g by the workload's FLOPs-matched rule (the sum stays G k_base)."""
@@ -651,6 +681,7 @@ def measure(w, args, device, ws, local, headline):
         "routing_kernels": sorted(mem_bytes),
         "gpu_launches": int(launches),
         "kernel_ms_per_step": kms,
+        "gemm_rooflines": _gemm_rooflines(w, P, kms, hbm, bf16_burst),
         "clocks": clk,
         "graph_ms": graph_ms, "coverage": coverage, "rows": rows, "tc_cap": tc_cap,
         "shared_ms": shared_ms, "Fs": Fs,
@@ -734,6 +765,7 @@ def run_ours(args):
     out["coverage"] = res["coverage"]
     out["gpu_launches"] = res["gpu_launches"]
     out["kernel_ms_per_step"] = res["kernel_ms_per_step"]
+    out["gemm_rooflines"] = res["gemm_rooflines"]
     out["clocks"] = res["clocks"]
     # the other workloads, each in the same run (single GPU, default expert-choice line)
     extra = [] if (ws > 1 or tc or args.shared_experts or args.seqs
@@ -763,6 +795,7 @@ def run_ours(args):
             "routing_hbm_gbs": res["routing_hbm_gbs"], "routing_hbm_frac": res["routing_hbm_frac"],
             "gpu_launches": res["gpu_launches"],
             "kernel_ms_per_step": res["kernel_ms_per_step"],
+            "gemm_rooflines": res["gemm_rooflines"],
             "clocks": res["clocks"],
         }
     if rank == 0 and not args.no_cpu_baseline:
